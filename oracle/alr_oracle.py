@@ -1,0 +1,267 @@
+"""CPU oracle for the ALR slot-loss hot path.  TEST INFRASTRUCTURE ONLY.
+
+This module is the plain, slow, fp64 statement of what the GPU path computes.  Only the
+test suite, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may import
+or call it; the product path (the CUDA library and its Python binding) never does, and this
+module imports nothing from the product package.
+
+Every function takes the already-rounded inputs (bf16 or fp32 values) widened to float64 and
+accumulates in float64.  Library primitives used as single steps: ``numpy.matmul`` (the
+head projection and the gradient products), ``numpy.argmax`` (first index of the maximum).
+
+Notation follows the paper ("Recovering Off-Policy Supervision for Speculative Decoding"):
+an anchor block has slots k = 1..K predicted in parallel (Sec. 3).  A batch holds A anchors
+with B rows each; buffer row r = a*B + s holds paper slot k = s + 1.  z_d = H_d W are the
+drafter logits (q = softmax z_d), z_t = H_t W the target logits whose softmax p is the label
+distribution pi_{a,k} (Eq. 3 for ALR rows, the corpus-prefix KD label of Sec. 3.1 otherwise).
+
+Parity status: every function below is pinned by tests/test_oracle_pins.py against closed
+forms, textbook special cases, finite differences or brute-force enumeration.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+MODE_ALR = 0          # omega = w_k (Sec. 3.2: ALR keeps the envelope and omits the gate)
+MODE_ERASE_SOFT = 1   # omega = w_k * g_{a,k}, soft survival gate (Eq. 2)
+MODE_ERASE_HARD = 2   # omega = w_k * prod 1[x = greedy target]  (hard variant under Eq. 2)
+
+
+def _f64(x):
+    return np.asarray(x, dtype=np.float64)
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 1: slot envelope w_k = exp(-(k-1)/gamma)
+# ----------------------------------------------------------------------------------------
+def slot_envelope(B: int, gamma: float) -> np.ndarray:
+    """Envelope of Eq. 1 for buffer slots s = 0..B-1 (paper slot k = s+1): exp(-s/gamma)."""
+    k = np.arange(1, B + 1, dtype=np.float64)
+    return np.exp(-(k - 1.0) / float(gamma))
+
+
+# ----------------------------------------------------------------------------------------
+# Head projection and the full-vocabulary normaliser
+# ----------------------------------------------------------------------------------------
+def head_logits(H, W) -> np.ndarray:
+    """z = H W for H [N, d] and the vocabulary head W [d, V] (one matmul)."""
+    return _f64(H) @ _f64(W)
+
+
+def log_sum_exp(z) -> np.ndarray:
+    """Row-wise log sum_v exp(z[r, v]), shifted by the row maximum for range safety."""
+    z = _f64(z)
+    m = z.max(axis=1, keepdims=True)
+    return (m + np.log(np.exp(z - m).sum(axis=1, keepdims=True)))[:, 0]
+
+
+def softmax(z) -> np.ndarray:
+    z = _f64(z)
+    return np.exp(z - log_sum_exp(z)[:, None])
+
+
+# ----------------------------------------------------------------------------------------
+# Soft cross-entropy l(pi, q) of Eq. 1, in its full-vocabulary form
+# ----------------------------------------------------------------------------------------
+def soft_cross_entropy(p, z_d) -> np.ndarray:
+    """l_r = -sum_v p[r, v] log q[r, v] with log q = z_d - LSE(z_d)."""
+    p = _f64(p)
+    log_q = _f64(z_d) - log_sum_exp(z_d)[:, None]
+    return -(p * log_q).sum(axis=1)
+
+
+def entropy(p) -> np.ndarray:
+    """H(p)_r = -sum_v p log p (terms with p = 0 contribute 0)."""
+    p = _f64(p)
+    safe = np.where(p > 0, p, 1.0)
+    return -(p * np.log(safe)).sum(axis=1)
+
+
+# ----------------------------------------------------------------------------------------
+# Greedy choice with the paper's tie rule (App. A: greedy ties go to the lower token id)
+# ----------------------------------------------------------------------------------------
+def greedy(z):
+    """Per row: the smallest index attaining the maximum, and the gap top1 - top2.
+
+    top2 is the largest value at any other index, so an exact tie gives gap 0.  With V = 1
+    there is no second value and the gap is +inf.
+    """
+    z = _f64(z)
+    idx = np.argmax(z, axis=1)                  # numpy returns the first maximal index
+    rows = np.arange(z.shape[0])
+    top1 = z[rows, idx]
+    if z.shape[1] == 1:
+        return idx.astype(np.int64), np.full(z.shape[0], np.inf)
+    rest = z.copy()
+    rest[rows, idx] = -np.inf
+    return idx.astype(np.int64), top1 - rest.max(axis=1)
+
+
+# ----------------------------------------------------------------------------------------
+# Eq. 2: survival gate of the erase comparator
+# ----------------------------------------------------------------------------------------
+def erase_gate(B, logp_x=None, corpus_tok=None, argmax_t=None, hard=False) -> np.ndarray:
+    """g_{a,k} = prod_{1<=j<k} f_{a,j} per buffer row (Eq. 2).
+
+    Buffer row s of anchor a carries the label of paper slot k = s+1, conditioned on the
+    corpus prefix before position a+k, and corpus_tok[a*B+s] is the corpus token x_{a+k}
+    that this label predicts.  So the factor for paper position a+j (j = s'+1) comes from
+    row s' = j-1:
+      soft: f = p_T(x_{a+j} | x_{<a+j}) = exp(logp_x[a*B+s'])
+      hard: f = 1[x_{a+j} == greedy target after x_{<a+j}] = 1[corpus_tok == argmax_t] of row s'
+    and row s multiplies the factors of rows s' < s; row 0 (slot 1) has the empty product 1.
+    """
+    if hard:
+        f = (np.asarray(corpus_tok) == np.asarray(argmax_t)).astype(np.float64)
+    else:
+        f = np.exp(_f64(logp_x))
+    f = f.reshape(-1, B)
+    g = np.ones_like(f)
+    for s in range(1, B):
+        g[:, s] = g[:, s - 1] * f[:, s - 1]
+    return g.reshape(-1)
+
+
+def slot_weights(mode, B, gamma, N, row_mask=None, logp_x=None, corpus_tok=None,
+                 argmax_t=None) -> np.ndarray:
+    """omega_r of Eq. 1: envelope w_k, times the termination / IRA validity mask, times the
+    erase gate of Eq. 2 in the erase modes (ALR omits the gate, Sec. 3.2)."""
+    w = np.tile(slot_envelope(B, gamma), N // B)
+    if row_mask is not None:
+        w = w * _f64(row_mask)
+    if mode == MODE_ERASE_SOFT:
+        w = w * erase_gate(B, logp_x=logp_x)
+    elif mode == MODE_ERASE_HARD:
+        w = w * erase_gate(B, corpus_tok=corpus_tok, argmax_t=argmax_t, hard=True)
+    return w
+
+
+def weighted_loss(loss_row, weight, lam):
+    """Eq. 1 scaled by the KD factor lambda: L = lam * sum omega l / sum omega (0 if sum omega = 0)."""
+    weight = _f64(weight)
+    wsum = weight.sum()
+    if wsum == 0.0:
+        return 0.0, 0.0
+    return float(lam * (weight * _f64(loss_row)).sum() / wsum), float(wsum)
+
+
+# ----------------------------------------------------------------------------------------
+# Forward pass of the slot loss
+# ----------------------------------------------------------------------------------------
+def slot_loss_forward(Hd, Ht, W, B, mode=MODE_ALR, gamma=2.0, lam=1.0, row_mask=None,
+                      corpus_tok=None):
+    """All forward outputs of the slot loss for N = A*B rows.
+
+    Returns a dict with z_d, z_t (kept for the backward), lse_d, lse_t, loss_row (l_r),
+    ent_row (H(p_r)), argmax_d / argmax_t and gap_d / gap_t, logp_x (erase modes), weight
+    (omega_r), loss_total (L) and weight_sum (sum omega).
+    """
+    Hd, Ht, W = _f64(Hd), _f64(Ht), _f64(W)
+    N = Hd.shape[0]
+    assert N % B == 0
+    z_d = head_logits(Hd, W)
+    z_t = head_logits(Ht, W)
+    lse_d = log_sum_exp(z_d)
+    lse_t = log_sum_exp(z_t)
+    p = np.exp(z_t - lse_t[:, None])
+    loss_row = soft_cross_entropy(p, z_d)
+    ent_row = entropy(p)
+    am_d, gap_d = greedy(z_d)
+    am_t, gap_t = greedy(z_t)
+    logp_x = None
+    if mode in (MODE_ERASE_SOFT, MODE_ERASE_HARD):
+        x = np.asarray(corpus_tok, dtype=np.int64)
+        logp_x = z_t[np.arange(N), x] - lse_t
+    weight = slot_weights(mode, B, gamma, N, row_mask=row_mask, logp_x=logp_x,
+                          corpus_tok=corpus_tok, argmax_t=am_t)
+    L, wsum = weighted_loss(loss_row, weight, lam)
+    return dict(z_d=z_d, z_t=z_t, lse_d=lse_d, lse_t=lse_t, loss_row=loss_row,
+                ent_row=ent_row, argmax_d=am_d, argmax_t=am_t, gap_d=gap_d, gap_t=gap_t,
+                logp_x=logp_x, weight=weight, loss_total=L, weight_sum=wsum)
+
+
+# ----------------------------------------------------------------------------------------
+# Backward pass: gradient of L with respect to the drafter logits, H_d and W
+# ----------------------------------------------------------------------------------------
+def logit_grad(z_d, z_t, weight, lam) -> np.ndarray:
+    """dL/dz_d[r, v] = lam * omega_r / sum omega * (q[r, v] - p[r, v]).
+
+    From l_r = LSE(z_d) - sum_v p_v z_d,v: d l_r / d z_d,v = q_v - p_v.  The label p, the
+    weights omega and the erase gate are target-side quantities and carry no gradient.
+    """
+    weight = _f64(weight)
+    wsum = weight.sum()
+    if wsum == 0.0:
+        return np.zeros_like(_f64(z_d))
+    q = softmax(z_d)
+    p = softmax(z_t)
+    return (lam * weight / wsum)[:, None] * (q - p)
+
+
+def slot_loss_backward(Hd, W, G, dW_in=None):
+    """dH_d = G W^T and dW = dW_in + H_d^T G (the drafter path of z_d = H_d W)."""
+    G, Hd, W = _f64(G), _f64(Hd), _f64(W)
+    dHd = G @ W.T
+    dW = Hd.T @ G
+    if dW_in is not None:
+        dW = dW + _f64(dW_in)
+    return dHd, dW
+
+
+# ----------------------------------------------------------------------------------------
+# Accepted length (Sec. 3.2 and the MAT definition of Sec. 4)
+# ----------------------------------------------------------------------------------------
+def accept_len(argmax_d, argmax_t, B, active=None):
+    """acc[a] = number of leading rows s with active[a*B+s] and argmax_d == argmax_t.
+
+    A slot contributes only when every earlier slot matched, so the count stops at the first
+    mismatch or inactive (masked) row.  hist[n] = #{a : acc[a] = n}, n = 0..B.
+    """
+    am_d = np.asarray(argmax_d).reshape(-1, B)
+    am_t = np.asarray(argmax_t).reshape(-1, B)
+    ok = am_d == am_t
+    if active is not None:
+        ok &= np.asarray(active).reshape(-1, B) > 0
+    A = ok.shape[0]
+    acc = np.zeros(A, dtype=np.int64)
+    for a in range(A):
+        n = 0
+        while n < B and ok[a, n]:
+            n += 1
+        acc[a] = n
+    hist = np.bincount(acc, minlength=B + 1).astype(np.int64)
+    return acc, hist
+
+
+# ----------------------------------------------------------------------------------------
+# IRA placement (Eq. 4): gather slot features from a rollout feature buffer
+# ----------------------------------------------------------------------------------------
+def gather_ira_blocks(F, seq, pos, B, valid_len=None):
+    """out[a*B+s] = F[seq_a, pos_a + s] and row_valid = 1 when that position exists.
+
+    A row is invalid (zero features, row_valid 0) when seq_a is outside [0, S), pos_a < 0,
+    or pos_a + s >= min(valid_len_a, L).  For an IRA secondary block at offset j inside a
+    primary block's stored rows [K, d], pos = j and valid_len = K give exactly the indicator
+    1[j + k <= K] of Eq. 4 (row s is paper slot k = s + 1 and reads primary row j + s).
+    """
+    F = np.asarray(F)
+    S, L, d = F.shape
+    A = len(seq)
+    out = np.zeros((A * B, d), dtype=F.dtype)
+    valid = np.zeros(A * B, dtype=np.float32)
+    for a in range(A):
+        sq, p0 = int(seq[a]), int(pos[a])
+        lim = L if valid_len is None else min(int(valid_len[a]), L)
+        if sq < 0 or sq >= S or p0 < 0:
+            continue
+        for s in range(B):
+            if p0 + s < lim:
+                out[a * B + s] = F[sq, p0 + s]
+                valid[a * B + s] = 1.0
+    return out, valid
+
+
+def ira_supervised_slots(K: int, j: int) -> int:
+    """Number of supervised slots of a secondary block at offset j (Eq. 4): #{k : j+k <= K}."""
+    return sum(1 for k in range(1, K + 1) if j + k <= K)
