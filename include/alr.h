@@ -1,0 +1,189 @@
+/*
+ * libalr — GB300 (sm_103a) hot path of Anchor-Label Relabelling with In-Rollout Anchors.
+ *
+ * The operations follow "Recovering Off-Policy Supervision for Speculative Decoding":
+ *   - the weighted, normalised soft cross-entropy of Eq. 1 with the slot envelope
+ *     w_k = exp(-(k-1)/gamma), evaluated over the full vocabulary;
+ *   - the ALR label distribution pi = p_T(. | ...) read through the vocabulary head (Eq. 3);
+ *   - the erase comparator's survival gate (Eq. 2, soft and hard variants);
+ *   - the IRA placement of blocks inside a rollout, with weights w_k 1[j+k <= K] (Eq. 4);
+ *   - the greedy accepted length behind the MAT metric (Sec. 3.2, Sec. 4), ties to the
+ *     lower token id (App. A, rollout implementation).
+ *
+ * Conventions shared by every entry point
+ *   Rows.      A batch holds A anchors with B rows each, N = A*B; row r = a*B + s holds the
+ *              paper's slot k = s+1 of anchor a.  1 <= B <= 32.
+ *   Memory.    Every pointer is a DEVICE pointer owned by the caller, unless stated.  The
+ *              library allocates no device memory; scratch comes from a caller workspace whose
+ *              size the matching *_workspace_size function returns.  Matrices are row-major
+ *              and dense; every base pointer must be 16-byte aligned.
+ *   Streams.   `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *              Every call only enqueues work on it and returns without synchronising.
+ *   Errors.    Every call returns an int status (ALR_OK = 0) and never throws.  Arguments
+ *              are validated before anything is enqueued; on failure nothing is launched and
+ *              alr_last_error() (per host thread) describes the problem.  Kernels that wait
+ *              on on-chip pipelines give up after a bounded time and record ALR_ERR_TIMEOUT
+ *              in a per-device status word that alr_device_status() reads.
+ *   Inputs.    Outputs are unspecified when the inputs contain NaN or Inf.
+ */
+#ifndef ALR_H
+#define ALR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define ALR_OK 0
+#define ALR_ERR_INVALID_ARG 1   /* null pointer, bad size, misalignment, workspace too small */
+#define ALR_ERR_UNSUPPORTED 2   /* dtype / mode not supported, or the device is not sm_103 */
+#define ALR_ERR_CUDA 3          /* a CUDA runtime or driver call failed (launch, encode)   */
+#define ALR_ERR_TIMEOUT 4       /* a device-side bounded wait expired (alr_device_status)  */
+
+/* Element types of H_d, H_t, W (and the feature buffer of the gather). */
+#define ALR_BF16 0              /* bfloat16 inputs, bf16 tensor-core products, fp32 accumulate */
+#define ALR_F32 1               /* fp32 inputs, tf32 tensor-core products, fp32 accumulate     */
+
+/* Slot-weight modes of the loss (omega_{a,k} of Eq. 1). */
+#define ALR_MODE_ALR 0          /* omega = w_k * mask             (ALR / IRA, Sec. 3.2)        */
+#define ALR_MODE_ERASE_SOFT 1   /* omega = w_k * mask * g_{a,k}   (soft survival gate, Eq. 2)  */
+#define ALR_MODE_ERASE_HARD 2   /* omega = w_k * mask * prod 1[x == greedy target] (Eq. 2)     */
+
+/* Problem description shared by the forward and backward calls. */
+typedef struct {
+    int64_t N;       /* rows, N = A*B, N >= 1                                                 */
+    int32_t d;       /* hidden size (contraction length), d >= 8, d % 8 == 0                  */
+    int32_t V;       /* vocabulary size, V >= 2, V % 8 == 0                                   */
+    int32_t B;       /* rows per anchor, 1 <= B <= 32, N % B == 0                             */
+    int32_t dtype;   /* ALR_BF16 or ALR_F32                                                   */
+    int32_t mode;    /* ALR_MODE_*                                                            */
+    float lambda;    /* KD loss scale lambda multiplying Eq. 1 (App. A: 1.013441 VL, 1.0 text) */
+    float gamma;     /* envelope constant gamma of Eq. 1, > 0 (default 2)                     */
+} alr_params;
+
+/* Forward outputs, all device pointers, length N unless stated. */
+typedef struct {
+    float* loss_row;     /* l_r = -sum_v p log q (required)                                    */
+    float* ent_row;      /* H(p_r), the label entropy (nullable)                               */
+    float* lse_d;        /* log-sum-exp of the drafter logits z_d = H_d W (required)           */
+    float* lse_t;        /* log-sum-exp of the target logits z_t = H_t W (required)            */
+    int32_t* argmax_d;   /* greedy drafter token, lowest id on ties (required)                 */
+    int32_t* argmax_t;   /* greedy target token, lowest id on ties (required)                  */
+    float* gap_d;        /* top-1 minus top-2 drafter logit, 0 on an exact tie (nullable)      */
+    float* gap_t;        /* same for the target logits (nullable)                              */
+    float* logp_x;       /* erase modes: log p_t(corpus_tok_r); other modes untouched (nullable) */
+    float* weight;       /* omega_r, the final slot weight (required)                          */
+    float* loss_total;   /* [1] L = lambda * sum omega l / sum omega, 0 when sum omega = 0     */
+    float* weight_sum;   /* [1] sum omega (the backward's normaliser)                          */
+} alr_fwd_outputs;
+
+/* Library version string (static storage). */
+const char* alr_version(void);
+
+/* Description of the last failed call on this host thread (static thread-local storage). */
+const char* alr_last_error(void);
+
+/* ALR_OK when the current device is compute capability 10.3 (sm_103), else ALR_ERR_UNSUPPORTED. */
+int alr_device_supported(void);
+
+/*
+ * Synchronises `stream`, then reads the current device's status word: ALR_OK, or
+ * ALR_ERR_TIMEOUT if any kernel of this library gave up a bounded wait since the last clear.
+ * clear != 0 resets the word to ALR_OK.
+ */
+int alr_device_status(void* stream, int clear);
+
+/*
+ * IRA gather (Eq. 4; App. A: rollout features stored for y*_1..y*_13).
+ *   feat      [S, L, d] features of S rollout sequences of length L, element type `dtype`.
+ *   seq, pos  [A] int32: anchor a reads sequence seq[a] from position pos[a].
+ *   valid_len [A] int32 or NULL (= L): positions >= min(valid_len[a], L) are not supervised.
+ *   out       [A*B, d] (same dtype): out[a*B+s] = feat[seq[a], pos[a]+s] for a valid row,
+ *             zeros otherwise.
+ *   row_valid [A*B] float or NULL: 1 for a valid row, 0 otherwise.  A row is invalid when
+ *             seq[a] is outside [0, S), pos[a] < 0, or pos[a]+s >= min(valid_len[a], L).
+ * A secondary IRA block at offset j inside a primary block's K stored rows is the gather
+ * with L = K, pos = j and valid_len = K, whose row_valid is 1[j + k <= K].
+ * Requires d * elemsize % 16 == 0.
+ */
+int alr_gather_ira_blocks(const void* feat, int32_t S, int32_t L, int32_t d, int32_t dtype,
+                          const int32_t* seq, const int32_t* pos, const int32_t* valid_len,
+                          int32_t A, int32_t B, void* out, float* row_valid, void* stream);
+
+/* Workspace bytes alr_slot_loss_fwd needs for `p` (0 on invalid params). */
+size_t alr_fwd_workspace_size(const alr_params* p);
+
+/*
+ * Forward pass of the slot loss (Eq. 1 with labels from Eq. 3, gate from Eq. 2).
+ *   Hd, Ht     [N, d] drafter and target hidden states (dtype p->dtype).
+ *   W          [d, V] vocabulary head shared by both sides (row-major, V contiguous).
+ *   row_mask   [N] float or NULL (= all ones): multiplies omega (termination, IRA validity).
+ *   corpus_tok [N] int32, required in the erase modes: the corpus token x that row r's
+ *              label predicts; must lie in [0, V).  Ignored in ALR mode.
+ *   out        output pointers (see alr_fwd_outputs).
+ * The logits are produced tile by tile in tensor memory and reduced on chip; they are never
+ * written to global memory.
+ */
+int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                      const float* row_mask, const int32_t* corpus_tok,
+                      const alr_fwd_outputs* out, void* workspace, size_t ws_bytes,
+                      void* stream);
+
+/* Workspace bytes alr_slot_loss_bwd needs for `p` (includes the logit gradient, N*V*elem). */
+size_t alr_bwd_workspace_size(const alr_params* p);
+
+/*
+ * Backward pass of the slot loss.  The label p, the weights and the gate are constants, so
+ * the gradient reaches z_d only: G = lambda * omega_r / sum omega * (q - p), recomputed
+ * tile by tile from Hd, Ht, W and the forward's lse_d, lse_t.
+ *   weight, weight_sum, lse_d, lse_t   forward outputs (device).
+ *   dHd  [N, d] float, overwritten with G W^T.
+ *   dW   [d, V] float or NULL; when given, H_d^T G is ADDED to it (gradient accumulation).
+ */
+int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                      const float* weight, const float* weight_sum, const float* lse_d,
+                      const float* lse_t, float* dHd, float* dW, void* workspace,
+                      size_t ws_bytes, void* stream);
+
+/*
+ * Greedy accepted length per anchor (Sec. 3.2: slot k counts only when slots 1..k-1 were
+ * accepted; MAT tau = acc + 1, Sec. 4).
+ *   argmax_d, argmax_t [A*B] int32; active [A*B] float or NULL (rows with active <= 0 stop
+ *   the count).  acc_len [A] int32 output; hist [B+1] int64 or NULL, overwritten with
+ *   hist[n] = #{a : acc_len[a] = n}.
+ */
+int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,
+                   int32_t A, int32_t B, int32_t* acc_len, int64_t* hist, void* stream);
+
+/*
+ * Slot weights of the erase comparator (Eq. 2) from per-row target statistics.
+ *   logp_x   [A*B] float: log p_T of the corpus token row r's label predicts (soft gate).
+ *   corpus_tok, argmax_t [A*B] int32 (hard gate; may be NULL when hard == 0).
+ *   row_mask [A*B] float or NULL.
+ *   weight   [A*B] output: w_k * mask * g, g = prod over earlier rows of the anchor of
+ *            exp(logp_x) (soft) or 1[corpus_tok == argmax_t] (hard); 1 for the first row.
+ */
+int alr_erase_weights(const float* logp_x, const int32_t* corpus_tok, const int32_t* argmax_t,
+                      const float* row_mask, int32_t A, int32_t B, float gamma, int32_t hard,
+                      float* weight, void* stream);
+
+/*
+ * The tensor-core GEMM the backward pass runs on, exposed on its own:
+ *   C[M, Nc] = A B   (accumulate == 0)   or   C[M, Nc] += A B   (accumulate != 0)
+ * with fp32 C (row-major, leading dimension Nc) and A, B of element type `dtype`:
+ *   a_mn == 0: A stored [M, K] row-major;  a_mn != 0: A stored [K, M] row-major.
+ *   b_mn == 0: B stored [Nc, K] row-major; b_mn != 0: B stored [K, Nc] row-major.
+ * dH_d = G W^T is (a_mn, b_mn) = (0, 0) and dW += H_d^T G is (1, 1).  Row strides must be
+ * multiples of 16 bytes and Nc % 4 == 0.
+ */
+int alr_gemm(int32_t dtype, int32_t a_mn, int32_t b_mn, int32_t accumulate, const void* A,
+             const void* B, float* C, int32_t M, int32_t Nc, int32_t K, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ALR_H */

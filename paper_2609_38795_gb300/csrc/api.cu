@@ -1,0 +1,482 @@
+// C ABI of libalr (declared in include/alr.h): argument validation, tensor-map encoding,
+// work planning and kernel launches.  No entry point allocates device memory.
+#include <cudaTypedefs.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "alr.h"
+#include "kernels.h"
+
+namespace {
+
+thread_local char g_err[1024] = "";
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(ALR_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+std::mutex g_mu;
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+struct DevInfo {
+  int sms = 0;
+  int cc = 0;
+};
+
+int device_info(DevInfo* out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  static DevInfo cache[64];
+  if (dev < 0 || dev >= 64) return fail(ALR_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (cache[dev].sms == 0) {
+    int sms = 0, major = 0, minor = 0;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) !=
+            cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess)
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    cache[dev].sms = sms;
+    cache[dev].cc = major * 10 + minor;
+  }
+  *out = cache[dev];
+  return ALR_OK;
+}
+
+int require_sm103(DevInfo* info) {
+  int rc = device_info(info);
+  if (rc != ALR_OK) return rc;
+  if (info->cc != 103)
+    return fail(ALR_ERR_UNSUPPORTED,
+                "libalr kernels are built for sm_103a only; current device is sm_%d", info->cc);
+  return ALR_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t elem_size(int dtype) { return dtype == ALR_BF16 ? 2 : 4; }
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// 2-D tiled tensor map with 128-byte swizzle: `inner` contiguous elements per row, `outer`
+// rows `row_bytes` apart; boxes of box_inner x box_outer elements.
+int make_map(CUtensorMap* m, const void* ptr, int dtype, uint64_t inner, uint64_t outer,
+             uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  auto enc = encode_fn();
+  if (enc == nullptr) return fail(ALR_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, dtype == ALR_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                   2, const_cast<void*>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(ALR_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d) for %llu x %llu", int(r),
+                (unsigned long long)inner, (unsigned long long)outer);
+  return ALR_OK;
+}
+
+// K elements per 128-byte swizzle row, and MN elements per 128-byte chunk.
+uint32_t k_per_row(int dtype) { return uint32_t(128 / elem_size(dtype)); }
+
+int check_params(const alr_params* p) {
+  if (p == nullptr) return fail(ALR_ERR_INVALID_ARG, "params is NULL");
+  if (p->dtype != ALR_BF16 && p->dtype != ALR_F32)
+    return fail(ALR_ERR_UNSUPPORTED, "dtype %d is not ALR_BF16 or ALR_F32", p->dtype);
+  if (p->mode < ALR_MODE_ALR || p->mode > ALR_MODE_ERASE_HARD)
+    return fail(ALR_ERR_UNSUPPORTED, "mode %d is not an ALR_MODE_* value", p->mode);
+  if (p->B < 1 || p->B > 32) return fail(ALR_ERR_INVALID_ARG, "B = %d must lie in [1, 32]", p->B);
+  if (p->N < 1 || p->N % p->B != 0)
+    return fail(ALR_ERR_INVALID_ARG, "N = %lld must be a positive multiple of B = %d",
+                (long long)p->N, p->B);
+  if (p->N > (int64_t(1) << 30)) return fail(ALR_ERR_INVALID_ARG, "N = %lld too large", (long long)p->N);
+  if (p->d < 8 || p->d % 8 != 0) return fail(ALR_ERR_INVALID_ARG, "d = %d must be a positive multiple of 8", p->d);
+  if (p->V < 2 || p->V % 8 != 0) return fail(ALR_ERR_INVALID_ARG, "V = %d must be >= 2 and a multiple of 8", p->V);
+  if (!(p->gamma > 0.f)) return fail(ALR_ERR_INVALID_ARG, "gamma must be > 0");
+  if (!(p->lambda == p->lambda)) return fail(ALR_ERR_INVALID_ARG, "lambda is NaN");
+  return ALR_OK;
+}
+
+alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
+  alr::LossPlan P{};
+  P.N = int(p->N);
+  P.d = p->d;
+  P.V = p->V;
+  P.B = p->B;
+  P.n_rb = int((p->N + 127) / 128);
+  P.n_vt = (p->V + 127) / 128;
+  P.group_rows = P.n_rb < 8 ? P.n_rb : 8;
+  if (bwd) {
+    P.n_vs = P.n_vt;  // one tile per unit
+  } else {
+    int vs = sms / P.group_rows;
+    if (vs < 1) vs = 1;
+    P.n_vs = vs < P.n_vt ? vs : P.n_vt;
+  }
+  P.n_units = P.n_rb * P.n_vs;
+  P.grid = sms < P.n_units ? sms : P.n_units;
+  return P;
+}
+
+// fp32 inputs run tf32 products, which take K-major operands only: the head is then read from
+// a transposed copy W^T [V, d] placed in the workspace.
+struct FwdLayout {
+  size_t part_off, anchor_off, wt_off, total;
+};
+
+FwdLayout fwd_layout(const alr_params* p, int sms) {
+  const alr::LossPlan P = loss_plan(p, sms, false);
+  FwdLayout L{};
+  L.part_off = 0;
+  L.anchor_off = round_up(size_t(alr::kPFields) * P.n_vs * size_t(P.N) * sizeof(float), 1024);
+  L.wt_off = L.anchor_off + round_up(2 * sizeof(double) * size_t(P.N / P.B), 1024);
+  L.total = L.wt_off;
+  if (p->dtype == ALR_F32) L.total += round_up(size_t(p->V) * p->d * sizeof(float), 1024);
+  return L;
+}
+
+// Backward workspace: G [N, V]; for fp32 also W^T [V, d], G^T [V, N'] and H_d^T [d, N'] with
+// N' = N rounded up to 4 (16-byte rows).
+struct BwdLayout {
+  size_t g_off, wt_off, gt_off, hdt_off, total;
+  int64_t ld_n;
+};
+
+BwdLayout bwd_layout(const alr_params* p) {
+  BwdLayout L{};
+  const size_t es = p->dtype == ALR_BF16 ? 2 : 4;
+  L.g_off = 0;
+  L.total = round_up(size_t(p->N) * size_t(p->V) * es, 1024);
+  L.ld_n = (p->N + 3) / 4 * 4;
+  if (p->dtype == ALR_F32) {
+    L.wt_off = L.total;
+    L.gt_off = L.wt_off + round_up(size_t(p->V) * p->d * 4, 1024);
+    L.hdt_off = L.gt_off + round_up(size_t(p->V) * L.ld_n * 4, 1024);
+    L.total = L.hdt_off + round_up(size_t(p->d) * L.ld_n * 4, 1024);
+  }
+  return L;
+}
+
+alr::GemmArgs gemm_plan(int M, int Nc, int K, float* C, int64_t ldc, int sms) {
+  alr::GemmArgs g{};
+  g.M = M;
+  g.Nc = Nc;
+  g.K = K;
+  g.C = C;
+  g.ldc = ldc;
+  g.n_mb = (M + 127) / 128;
+  g.n_nb = (Nc + 255) / 256;
+  g.group_m = g.n_mb < 16 ? g.n_mb : 16;
+  g.n_tiles = g.n_mb * g.n_nb;
+  g.grid = sms < g.n_tiles ? sms : g.n_tiles;
+  return g;
+}
+
+// Tensor map of the head operand of the fused loss kernels: MN-major tiles straight from
+// W [d, V] for bf16; for fp32, W is first transposed into `wt` and read K-major.
+int head_map(CUtensorMap* m, const alr_params* p, const void* W, void* wt, cudaStream_t s) {
+  const uint32_t kke = k_per_row(p->dtype);
+  if (p->dtype == ALR_BF16) return make_map(m, W, ALR_BF16, p->V, p->d, uint64_t(p->V) * 2, kke, kke);
+  cudaError_t e = alr::launch_transpose32(static_cast<const float*>(W), static_cast<float*>(wt),
+                                          p->d, p->V, p->d, s);
+  if (e != cudaSuccess) return cuda_fail(e, "head transpose launch");
+  return make_map(m, wt, ALR_F32, p->d, p->V, uint64_t(p->d) * 4, kke, 128);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* alr_version(void) { return "libalr 0.1 (sm_103a)"; }
+
+const char* alr_last_error(void) { return g_err; }
+
+int alr_device_supported(void) {
+  DevInfo info;
+  return require_sm103(&info);
+}
+
+int alr_device_status(void* stream, int clear) {
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int* w = alr::device_status_ptr();
+  if (w == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  int v = 0;
+  if ((e = cudaMemcpy(&v, w, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "reading the status word");
+  if (clear) {
+    const int z = 0;
+    if ((e = cudaMemcpy(w, &z, sizeof(int), cudaMemcpyHostToDevice)) != cudaSuccess)
+      return cuda_fail(e, "clearing the status word");
+  }
+  if (v != 0) return fail(ALR_ERR_TIMEOUT, "a device pipeline wait timed out");
+  return ALR_OK;
+}
+
+int alr_gather_ira_blocks(const void* feat, int32_t S, int32_t L, int32_t d, int32_t dtype,
+                          const int32_t* seq, const int32_t* pos, const int32_t* valid_len,
+                          int32_t A, int32_t B, void* out, float* row_valid, void* stream) {
+  if (dtype != ALR_BF16 && dtype != ALR_F32) return fail(ALR_ERR_UNSUPPORTED, "dtype %d", dtype);
+  if (S < 1 || L < 1 || d < 1 || A < 0 || B < 1)
+    return fail(ALR_ERR_INVALID_ARG, "bad sizes S=%d L=%d d=%d A=%d B=%d", S, L, d, A, B);
+  if ((size_t(d) * elem_size(dtype)) % 16 != 0)
+    return fail(ALR_ERR_INVALID_ARG, "d * element size must be a multiple of 16 bytes");
+  if (A == 0) return ALR_OK;
+  if (feat == nullptr || seq == nullptr || pos == nullptr || out == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "feat, seq, pos and out must be non-NULL");
+  if (!aligned16(feat) || !aligned16(out))
+    return fail(ALR_ERR_INVALID_ARG, "feat and out must be 16-byte aligned");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  cudaError_t e = alr::launch_gather(feat, S, L, d, int(elem_size(dtype)), seq, pos, valid_len, A,
+                                     B, out, row_valid, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  return ALR_OK;
+}
+
+size_t alr_fwd_workspace_size(const alr_params* p) {
+  if (check_params(p) != ALR_OK) return 0;
+  DevInfo info;
+  if (device_info(&info) != ALR_OK) return 0;
+  return fwd_layout(p, info.sms).total;
+}
+
+int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                      const float* row_mask, const int32_t* corpus_tok, const alr_fwd_outputs* out,
+                      void* workspace, size_t ws_bytes, void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || Ht == nullptr || W == nullptr || out == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht, W and out must be non-NULL");
+  if (!aligned16(Hd) || !aligned16(Ht) || !aligned16(W))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht and W must be 16-byte aligned");
+  if (out->loss_row == nullptr || out->lse_d == nullptr || out->lse_t == nullptr ||
+      out->argmax_d == nullptr || out->argmax_t == nullptr || out->weight == nullptr ||
+      out->loss_total == nullptr || out->weight_sum == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required forward output pointer is NULL");
+  if (p->mode != ALR_MODE_ALR && corpus_tok == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "the erase modes need corpus_tok");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  const FwdLayout lay = fwd_layout(p, info.sms);
+  if (workspace == nullptr || ws_bytes < lay.total)
+    return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
+                ws_bytes, lay.total);
+  if (!aligned16(workspace)) return fail(ALR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  const uint32_t kke = k_per_row(dt);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  CUtensorMap m_hd, m_ht, m_w;
+  if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
+
+  alr::LossArgs args{};
+  args.plan = loss_plan(p, info.sms, false);
+  args.part = reinterpret_cast<float*>(ws + lay.part_off);
+  args.corpus_tok = p->mode != ALR_MODE_ALR ? corpus_tok : nullptr;
+  args.lam = p->lambda;
+  args.status = alr::device_status_ptr();
+  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  e = alr::launch_loss_fwd(dt, m_hd, m_ht, m_w, args, s);
+  if (e != cudaSuccess) return cuda_fail(e, "forward loss kernel launch");
+  double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
+  e = alr::launch_combine(args.plan, args.part, p->mode, p->gamma, row_mask, args.corpus_tok,
+                          out->loss_row, out->ent_row, out->lse_d, out->lse_t, out->argmax_d,
+                          out->argmax_t, out->gap_d, out->gap_t, out->logp_x, out->weight, anchor,
+                          s);
+  if (e != cudaSuccess) return cuda_fail(e, "combine launch");
+  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
+  return ALR_OK;
+}
+
+size_t alr_bwd_workspace_size(const alr_params* p) {
+  if (check_params(p) != ALR_OK) return 0;
+  return bwd_layout(p).total;
+}
+
+int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                      const float* weight, const float* weight_sum, const float* lse_d,
+                      const float* lse_t, float* dHd, float* dW, void* workspace, size_t ws_bytes,
+                      void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || Ht == nullptr || W == nullptr || weight == nullptr ||
+      weight_sum == nullptr || lse_d == nullptr || lse_t == nullptr || dHd == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required backward pointer is NULL");
+  if (!aligned16(Hd) || !aligned16(Ht) || !aligned16(W) || !aligned16(dHd) ||
+      (dW != nullptr && !aligned16(dW)))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht, W, dHd and dW must be 16-byte aligned");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  const size_t need = alr_bwd_workspace_size(p);
+  if (workspace == nullptr || ws_bytes < need)
+    return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
+                ws_bytes, need);
+  if (!aligned16(workspace)) return fail(ALR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  const uint32_t kke = k_per_row(dt);
+  const BwdLayout lay = bwd_layout(p);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  void* G = ws + lay.g_off;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  CUtensorMap m_hd, m_ht, m_w, m_gs;
+  if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_gs, G, dt, p->V, p->N, p->V * es, kke, 32)) != ALR_OK) return rc;
+
+  alr::LossArgs args{};
+  args.plan = loss_plan(p, info.sms, true);
+  args.lse_d = lse_d;
+  args.lse_t = lse_t;
+  args.weight = weight;
+  args.weight_sum = weight_sum;
+  args.lam = p->lambda;
+  args.status = alr::device_status_ptr();
+  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, m_gs, args, s);
+  if (e != cudaSuccess) return cuda_fail(e, "backward logit-gradient kernel launch");
+
+  // dH_d = G W^T: A = G [N, V] K-major, B = W [d, V] K-major.
+  CUtensorMap m_ga, m_wk;
+  if ((rc = make_map(&m_ga, G, dt, p->V, p->N, p->V * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_wk, W, dt, p->V, p->d, p->V * es, kke, 256)) != ALR_OK) return rc;
+  alr::GemmArgs gh = gemm_plan(int(p->N), p->d, p->V, dHd, p->d, info.sms);
+  gh.status = args.status;
+  e = alr::launch_plain_gemm(dt, false, false, false, m_ga, m_wk, gh, s);
+  if (e != cudaSuccess) return cuda_fail(e, "dH GEMM launch");
+
+  if (dW != nullptr) {
+    alr::GemmArgs gw = gemm_plan(p->d, p->V, int(p->N), dW, p->V, info.sms);
+    gw.status = args.status;
+    CUtensorMap m_ha, m_gb;
+    if (dt == ALR_BF16) {
+      // dW += H_d^T G: A = H_d read as [K = N, M = d] (MN-major), B = G [K = N, V] (MN-major).
+      if ((rc = make_map(&m_ha, Hd, dt, p->d, p->N, p->d * es, kke, kke)) != ALR_OK) return rc;
+      if ((rc = make_map(&m_gb, G, dt, p->V, p->N, p->V * es, kke, kke)) != ALR_OK) return rc;
+      e = alr::launch_plain_gemm(dt, true, true, true, m_ha, m_gb, gw, s);
+    } else {
+      // K-major operands from transposed copies H_d^T [d, N'] and G^T [V, N'].
+      float* hdt = reinterpret_cast<float*>(ws + lay.hdt_off);
+      float* gt = reinterpret_cast<float*>(ws + lay.gt_off);
+      if ((e = alr::launch_transpose32(static_cast<const float*>(Hd), hdt, int(p->N), p->d,
+                                       int(lay.ld_n), s)) != cudaSuccess)
+        return cuda_fail(e, "H_d transpose launch");
+      if ((e = alr::launch_transpose32(static_cast<const float*>(G), gt, int(p->N), p->V,
+                                       int(lay.ld_n), s)) != cudaSuccess)
+        return cuda_fail(e, "G transpose launch");
+      if ((rc = make_map(&m_ha, hdt, dt, p->N, p->d, lay.ld_n * 4, kke, 128)) != ALR_OK) return rc;
+      if ((rc = make_map(&m_gb, gt, dt, p->N, p->V, lay.ld_n * 4, kke, 256)) != ALR_OK) return rc;
+      e = alr::launch_plain_gemm(dt, false, false, true, m_ha, m_gb, gw, s);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "dW GEMM launch");
+  }
+  return ALR_OK;
+}
+
+int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,
+                   int32_t A, int32_t B, int32_t* acc_len, int64_t* hist, void* stream) {
+  if (A < 0 || B < 1 || B > 32) return fail(ALR_ERR_INVALID_ARG, "bad sizes A=%d B=%d", A, B);
+  if (A > 0 && (argmax_d == nullptr || argmax_t == nullptr || acc_len == nullptr))
+    return fail(ALR_ERR_INVALID_ARG, "argmax_d, argmax_t and acc_len must be non-NULL");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  if (A == 0 && hist == nullptr) return ALR_OK;
+  cudaError_t e = alr::launch_accept_len(argmax_d, argmax_t, active, A, B, acc_len, hist,
+                                         static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "accept_len launch");
+  return ALR_OK;
+}
+
+int alr_erase_weights(const float* logp_x, const int32_t* corpus_tok, const int32_t* argmax_t,
+                      const float* row_mask, int32_t A, int32_t B, float gamma, int32_t hard,
+                      float* weight, void* stream) {
+  if (A < 0 || B < 1 || B > 32) return fail(ALR_ERR_INVALID_ARG, "bad sizes A=%d B=%d", A, B);
+  if (!(gamma > 0.f)) return fail(ALR_ERR_INVALID_ARG, "gamma must be > 0");
+  if (A == 0) return ALR_OK;
+  if (weight == nullptr) return fail(ALR_ERR_INVALID_ARG, "weight must be non-NULL");
+  if (hard ? (corpus_tok == nullptr || argmax_t == nullptr) : (logp_x == nullptr))
+    return fail(ALR_ERR_INVALID_ARG, "the %s gate needs %s", hard ? "hard" : "soft",
+                hard ? "corpus_tok and argmax_t" : "logp_x");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  cudaError_t e = alr::launch_erase_weights(logp_x, corpus_tok, argmax_t, row_mask, A, B, gamma,
+                                            hard, weight, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "erase_weights launch");
+  return ALR_OK;
+}
+
+int alr_gemm(int32_t dtype, int32_t a_mn, int32_t b_mn, int32_t accumulate, const void* A,
+             const void* B, float* C, int32_t M, int32_t Nc, int32_t K, void* stream) {
+  if (dtype != ALR_BF16 && dtype != ALR_F32) return fail(ALR_ERR_UNSUPPORTED, "dtype %d", dtype);
+  if (M < 1 || Nc < 1 || K < 1) return fail(ALR_ERR_INVALID_ARG, "bad sizes M=%d Nc=%d K=%d", M, Nc, K);
+  if (A == nullptr || B == nullptr || C == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "A, B and C must be non-NULL");
+  if (!aligned16(A) || !aligned16(B) || !aligned16(C))
+    return fail(ALR_ERR_INVALID_ARG, "A, B and C must be 16-byte aligned");
+  if (dtype == ALR_F32 && (a_mn || b_mn))
+    return fail(ALR_ERR_UNSUPPORTED, "fp32 (tf32) operands must be K-major");
+  const size_t es = elem_size(dtype);
+  const int64_t a_inner = a_mn ? M : K, b_inner = b_mn ? Nc : K;
+  if ((a_inner * es) % 16 != 0 || (b_inner * es) % 16 != 0 || Nc % 4 != 0)
+    return fail(ALR_ERR_INVALID_ARG, "row strides must be multiples of 16 bytes and Nc %% 4 == 0");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  const uint32_t kke = k_per_row(dtype);
+  CUtensorMap ma, mb;
+  if (a_mn) rc = make_map(&ma, A, dtype, M, K, M * es, kke, kke);
+  else rc = make_map(&ma, A, dtype, K, M, K * es, kke, 128);
+  if (rc != ALR_OK) return rc;
+  if (b_mn) rc = make_map(&mb, B, dtype, Nc, K, Nc * es, kke, kke);
+  else rc = make_map(&mb, B, dtype, K, Nc, K * es, kke, 256);
+  if (rc != ALR_OK) return rc;
+  alr::GemmArgs g = gemm_plan(M, Nc, K, C, Nc, info.sms);
+  g.status = alr::device_status_ptr();
+  if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  cudaError_t e = alr::launch_plain_gemm(dtype, a_mn != 0, b_mn != 0, accumulate != 0, ma, mb, g,
+                                         static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
+  return ALR_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,107 @@
+// Internal launch interface between the C-ABI layer (api.cu) and the kernel translation units.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace alr {
+
+// Row-block x vocabulary-split work plan of the fused loss kernels.
+//   A "unit" is one 128-row block times one contiguous range of 128-column vocabulary tiles.
+//   Units are numbered group by group: a group holds `group_rows` consecutive row blocks,
+//   and inside a group the row block varies fastest, so the CTAs running at the same time
+//   share both their hidden-state tiles and their head tiles through L2.
+struct LossPlan {
+  int N, d, V, B;
+  int n_rb;        // ceil(N / 128)
+  int n_vt;        // ceil(V / 128)
+  int n_vs;        // vocabulary splits (partial statistics per row and split)
+  int group_rows;  // row blocks per group
+  int n_units;     // n_rb * n_vs
+  int grid;        // persistent CTAs
+};
+
+// Partial statistics of one row over one vocabulary split (structure of arrays, field-major:
+// part[f * n_vs * N + vs * N + row]).
+enum PartField {
+  kPMd = 0,   // running max of z_d
+  kPSd,       // sum exp(z_d - m_d)
+  kPMt,       // running max of z_t
+  kPSt,       // sum exp(z_t - m_t)
+  kPU,        // sum exp(z_t - m_t) * z_d
+  kPW,        // sum exp(z_t - m_t) * z_t
+  kPBd,       // best z_d
+  kPId,       // its index (int bits)
+  kPSecd,     // second-best z_d (any other index)
+  kPBt,
+  kPIt,
+  kPSect,
+  kPZx,       // z_t at the corpus token if it lies in the split, else NaN
+  kPFields
+};
+
+struct LossArgs {
+  LossPlan plan;
+  float* part;                // forward: partial statistics
+  const int32_t* corpus_tok;  // forward: nullable
+  const float* lse_d;         // backward
+  const float* lse_t;
+  const float* weight;
+  const float* weight_sum;
+  float lam;
+  int* status;
+};
+
+// Fused dual-GEMM kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
+cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
+                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s);
+cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
+                            const CUtensorMap& w, const CUtensorMap& g_store,
+                            const LossArgs& args, cudaStream_t s);
+size_t loss_fwd_smem_bytes(int dtype);
+size_t loss_bwd_smem_bytes(int dtype);
+
+// Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm.cu).
+struct GemmArgs {
+  int M, Nc, K;
+  float* C;
+  int64_t ldc;
+  int n_mb, n_nb;   // 128-row and 256-column tile counts
+  int group_m;      // m-blocks per raster group
+  int n_tiles;
+  int grid;
+  int* status;
+};
+// a_mn / b_mn: operand stored MN-major (A as [K, M], B as [K, Nc]) instead of K-major
+// (A as [M, K], B as [Nc, K]).  accumulate: C += A B instead of C = A B.
+cudaError_t launch_plain_gemm(int dtype, bool a_mn, bool b_mn, bool accumulate,
+                              const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,
+                              cudaStream_t s);
+size_t plain_gemm_smem_bytes(int dtype);
+
+// Row-level kernels (row_kernels.cu).
+cudaError_t launch_gather(const void* feat, int S, int L, int d, int elem_bytes,
+                          const int32_t* seq, const int32_t* pos, const int32_t* valid_len,
+                          int A, int B, void* out, float* row_valid, cudaStream_t s);
+cudaError_t launch_combine(const LossPlan& plan, const float* part, int mode, float gamma,
+                           const float* row_mask, const int32_t* corpus_tok, float* loss_row,
+                           float* ent_row, float* lse_d, float* lse_t, int32_t* argmax_d,
+                           int32_t* argmax_t, float* gap_d, float* gap_t, float* logp_x,
+                           float* weight, double* anchor_part, cudaStream_t s);
+cudaError_t launch_finalize(const double* anchor_part, int A, float lam, float* loss_total,
+                            float* weight_sum, cudaStream_t s);
+cudaError_t launch_accept_len(const int32_t* am_d, const int32_t* am_t, const float* active,
+                              int A, int B, int32_t* acc, int64_t* hist, cudaStream_t s);
+cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,
+                                 const int32_t* argmax_t, const float* row_mask, int A, int B,
+                                 float gamma, int hard, float* weight, cudaStream_t s);
+
+// out[c, r] = in[r, c] for an fp32 [R, C] matrix; out rows are ld_out elements apart.
+cudaError_t launch_transpose32(const float* in, float* out, int R, int C, int ld_out,
+                               cudaStream_t s);
+
+// Per-device status word (status.cu).
+int* device_status_ptr();
+
+}  // namespace alr

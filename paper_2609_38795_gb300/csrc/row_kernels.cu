@@ -1,0 +1,335 @@
+// Row-level kernels of the slot-loss path: the IRA gather, the merge of per-split forward
+// statistics into the per-row loss terms and slot weights, the batch reduction of Eq. 1,
+// the accepted-length statistic and the erase-gate weights.
+#include <cfloat>
+
+#include "kernels.h"
+#include "tc_common.cuh"
+
+namespace alr {
+namespace {
+
+__device__ __forceinline__ float quiet_nan() { return __int_as_float(0x7fc00000); }
+
+// ------------------------------------------------------------------ IRA gather ---
+// One warp per output row; each lane moves 16-byte vectors, issuing a batch of loads before
+// the matching stores so that many requests are in flight per SM.
+constexpr int kGatherBatch = 8;
+
+__global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ feat, int S, int L,
+                                                     int vec_per_row,
+                                                     const int32_t* __restrict__ seq,
+                                                     const int32_t* __restrict__ pos,
+                                                     const int32_t* __restrict__ valid_len,
+                                                     int A, int B, uint4* __restrict__ out,
+                                                     float* __restrict__ row_valid) {
+  const long long r = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (r >= (long long)A * B) return;
+  const int a = int(r / B), s = int(r - (long long)a * B);
+  const int sq = seq[a], p0 = pos[a];
+  int lim = L;
+  if (valid_len != nullptr) lim = min(lim, valid_len[a]);
+  const bool ok = sq >= 0 && sq < S && p0 >= 0 && p0 + s < lim;
+  uint4* dst = out + r * vec_per_row;
+  if (lane == 0 && row_valid != nullptr) row_valid[r] = ok ? 1.f : 0.f;
+  if (!ok) {
+    const uint4 z = make_uint4(0, 0, 0, 0);
+    for (int i = lane; i < vec_per_row; i += 32) dst[i] = z;
+    return;
+  }
+  const uint4* src = feat + ((long long)sq * L + p0 + s) * vec_per_row;
+  for (int base = 0; base < vec_per_row; base += 32 * kGatherBatch) {
+    uint4 v[kGatherBatch];
+#pragma unroll
+    for (int j = 0; j < kGatherBatch; ++j) {
+      const int i = base + j * 32 + lane;
+      if (i < vec_per_row) v[j] = __ldg(src + i);
+    }
+#pragma unroll
+    for (int j = 0; j < kGatherBatch; ++j) {
+      const int i = base + j * 32 + lane;
+      if (i < vec_per_row) dst[i] = v[j];
+    }
+  }
+}
+
+// ------------------------------------------------------------- gate (Eq. 2) ---
+// Warp-level survival gate for one anchor: lane s holds row a*B+s (lanes >= B inactive).
+// soft: g_s = exp(sum_{s'<s} logp_x[s']); hard: g_s = prod_{s'<s} 1[x == argmax_t].
+__device__ __forceinline__ float gate_for_lane(bool active, int lane, bool hard, float logp,
+                                               bool match) {
+  if (hard) {
+    const unsigned bad = __ballot_sync(0xffffffffu, active && !match);
+    const unsigned below = (lane == 0) ? 0u : (0xffffffffu >> (32 - lane));
+    return (bad & below) ? 0.f : 1.f;
+  }
+  float v = active ? logp : 0.f;
+  float incl = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float t = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += t;
+  }
+  return expf(incl - v);
+}
+
+// --------------------------------------------------------------- combine ---
+// One warp per anchor.  Merges the per-split statistics of each row into the log-sum-exps,
+// l_r = LSE_d - (sum_v e^{z_t - m_t} z_d) / (sum_v e^{z_t - m_t}), the label entropy,
+// the greedy tokens with their top-1/top-2 gaps, log p_t(x), and the slot weight omega_r of
+// Eq. 1 (envelope w_k, mask, optional gate of Eq. 2).  Writes the anchor's sum omega l and
+// sum omega for the batch reduction.
+__global__ void __launch_bounds__(256) combine_kernel(
+    LossPlan P, const float* __restrict__ part, int mode, float gamma,
+    const float* __restrict__ row_mask, const int32_t* __restrict__ corpus_tok,
+    float* __restrict__ loss_row, float* __restrict__ ent_row, float* __restrict__ lse_d_out,
+    float* __restrict__ lse_t_out, int32_t* __restrict__ argmax_d, int32_t* __restrict__ argmax_t,
+    float* __restrict__ gap_d, float* __restrict__ gap_t, float* __restrict__ logp_x_out,
+    float* __restrict__ weight, double* __restrict__ anchor_part) {
+  const int A = P.N / P.B;
+  const int a = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (a >= A) return;
+  const bool active = lane < P.B;
+  const int r = a * P.B + (active ? lane : 0);
+  const size_t fs = size_t(P.n_vs) * P.N;
+
+  float Md = -INFINITY, Sd = 0.f, Mt = -INFINITY, St = 0.f, U = 0.f, Wt = 0.f;
+  float bd = -INFINITY, secd = -INFINITY, bt = -INFINITY, sect = -INFINITY, zx = quiet_nan();
+  int id = 0x7fffffff, it = 0x7fffffff;
+  if (active) {
+    for (int vs = 0; vs < P.n_vs; ++vs) {
+      const float* p = part + size_t(vs) * P.N + r;
+      const float md = p[kPMd * fs], sd = p[kPSd * fs];
+      const float nmd = fmaxf(Md, md);
+      Sd = Sd * ex2((Md - nmd) * kLog2e) + sd * ex2((md - nmd) * kLog2e);
+      Md = nmd;
+      const float mt = p[kPMt * fs];
+      const float nmt = fmaxf(Mt, mt);
+      const float so = ex2((Mt - nmt) * kLog2e), sn = ex2((mt - nmt) * kLog2e);
+      St = St * so + p[kPSt * fs] * sn;
+      U = U * so + p[kPU * fs] * sn;
+      Wt = Wt * so + p[kPW * fs] * sn;
+      Mt = nmt;
+      // top-2 merge: the earlier split holds the lower indices, so ties keep the incumbent
+      const float b2 = p[kPBd * fs], s2 = p[kPSecd * fs];
+      const int i2 = __float_as_int(p[kPId * fs]);
+      if (b2 > bd) {
+        secd = fmaxf(bd, s2);
+        bd = b2;
+        id = i2;
+      } else {
+        secd = fmaxf(secd, b2);
+      }
+      const float b3 = p[kPBt * fs], s3 = p[kPSect * fs];
+      const int i3 = __float_as_int(p[kPIt * fs]);
+      if (b3 > bt) {
+        sect = fmaxf(bt, s3);
+        bt = b3;
+        it = i3;
+      } else {
+        sect = fmaxf(sect, b3);
+      }
+      const float z = p[kPZx * fs];
+      if (z == z) zx = z;
+    }
+  }
+  const float lse_d = Md + logf(Sd);
+  const float lse_t = Mt + logf(St);
+  const float loss = lse_d - U / St;
+  const float logp = zx - lse_t;
+  const bool erase = mode != 0;
+  const int x = (erase && active) ? corpus_tok[r] : -1;
+  const float gate = erase ? gate_for_lane(active, lane, mode == 2, logp, x == it) : 1.f;
+  float w = 0.f;
+  if (active) {
+    w = expf(-float(lane) / gamma) * gate;
+    if (row_mask != nullptr) w *= row_mask[r];
+    loss_row[r] = loss;
+    if (ent_row) ent_row[r] = lse_t - Wt / St;
+    lse_d_out[r] = lse_d;
+    lse_t_out[r] = lse_t;
+    argmax_d[r] = id;
+    argmax_t[r] = it;
+    if (gap_d) gap_d[r] = bd - secd;
+    if (gap_t) gap_t[r] = bt - sect;
+    if (erase && logp_x_out) logp_x_out[r] = logp;
+    weight[r] = w;
+  }
+  double wl = active ? double(w) * double(loss) : 0.0;
+  double ws = active ? double(w) : 0.0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    wl += __shfl_xor_sync(0xffffffffu, wl, off);
+    ws += __shfl_xor_sync(0xffffffffu, ws, off);
+  }
+  if (lane == 0) {
+    anchor_part[2 * a] = wl;
+    anchor_part[2 * a + 1] = ws;
+  }
+}
+
+// Batch reduction of Eq. 1 in a fixed order (one block, deterministic).
+__global__ void __launch_bounds__(1024) finalize_kernel(const double* __restrict__ anchor_part,
+                                                        int A, float lam,
+                                                        float* __restrict__ loss_total,
+                                                        float* __restrict__ weight_sum) {
+  __shared__ double s_wl[32], s_ws[32];
+  double wl = 0.0, ws = 0.0;
+  for (int a = threadIdx.x; a < A; a += blockDim.x) {
+    wl += anchor_part[2 * a];
+    ws += anchor_part[2 * a + 1];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    wl += __shfl_xor_sync(0xffffffffu, wl, off);
+    ws += __shfl_xor_sync(0xffffffffu, ws, off);
+  }
+  const int warp = threadIdx.x / 32, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    s_wl[warp] = wl;
+    s_ws[warp] = ws;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    wl = lane < int(blockDim.x / 32) ? s_wl[lane] : 0.0;
+    ws = lane < int(blockDim.x / 32) ? s_ws[lane] : 0.0;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      wl += __shfl_xor_sync(0xffffffffu, wl, off);
+      ws += __shfl_xor_sync(0xffffffffu, ws, off);
+    }
+    if (lane == 0) {
+      *loss_total = ws > 0.0 ? float(double(lam) * wl / ws) : 0.f;
+      *weight_sum = float(ws);
+    }
+  }
+}
+
+// ------------------------------------------------------------- accepted length ---
+// One warp per anchor: the count of leading slots whose greedy drafter token equals the
+// greedy target token (and whose row is active).
+__global__ void __launch_bounds__(256) accept_len_kernel(const int32_t* __restrict__ am_d,
+                                                         const int32_t* __restrict__ am_t,
+                                                         const float* __restrict__ active_w,
+                                                         int A, int B, int32_t* __restrict__ acc,
+                                                         unsigned long long* __restrict__ hist) {
+  const int a = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (a >= A) return;
+  bool ok = false;
+  if (lane < B) {
+    const int r = a * B + lane;
+    ok = am_d[r] == am_t[r];
+    if (active_w != nullptr) ok = ok && active_w[r] > 0.f;
+  }
+  const unsigned bal = __ballot_sync(0xffffffffu, ok);
+  const int n = (bal == 0xffffffffu) ? 32 : (__ffs(~bal) - 1);
+  if (lane == 0) {
+    acc[a] = n;
+    if (hist != nullptr) atomicAdd(hist + n, 1ull);
+  }
+}
+
+// ---------------------------------------------------------- erase weights ---
+__global__ void __launch_bounds__(256) erase_weights_kernel(
+    const float* __restrict__ logp_x, const int32_t* __restrict__ corpus_tok,
+    const int32_t* __restrict__ argmax_t, const float* __restrict__ row_mask, int A, int B,
+    float gamma, int hard, float* __restrict__ weight) {
+  const int a = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (a >= A) return;
+  const bool active = lane < B;
+  const int r = a * B + (active ? lane : 0);
+  float logp = 0.f;
+  bool match = true;
+  if (active) {
+    if (hard) match = corpus_tok[r] == argmax_t[r];
+    else logp = logp_x[r];
+  }
+  const float g = gate_for_lane(active, lane, hard != 0, logp, match);
+  if (active) {
+    float w = expf(-float(lane) / gamma) * g;
+    if (row_mask != nullptr) w *= row_mask[r];
+    weight[r] = w;
+  }
+}
+
+// ------------------------------------------------------------------ transpose ---
+// out[c * ld_out + r] = in[r * C + c] for 32-bit elements, 32 x 32 tiles through shared memory.
+__global__ void __launch_bounds__(256) transpose32_kernel(const float* __restrict__ in,
+                                                          float* __restrict__ out, int R, int C,
+                                                          int ld_out) {
+  __shared__ float tile[32][33];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + threadIdx.x;
+    if (r < R && c < C) tile[i][threadIdx.x] = in[(long long)r * C + c];
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + threadIdx.x;
+    if (r < R && c < C) out[(long long)c * ld_out + r] = tile[threadIdx.x][i];
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_transpose32(const float* in, float* out, int R, int C, int ld_out,
+                               cudaStream_t s) {
+  dim3 grid((C + 31) / 32, (R + 31) / 32);
+  transpose32_kernel<<<grid, dim3(32, 8), 0, s>>>(in, out, R, C, ld_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const void* feat, int S, int L, int d, int elem_bytes,
+                          const int32_t* seq, const int32_t* pos, const int32_t* valid_len,
+                          int A, int B, void* out, float* row_valid, cudaStream_t s) {
+  const long long rows = (long long)A * B;
+  const int vec = int((long long)d * elem_bytes / 16);
+  const long long blocks = (rows + 7) / 8;
+  gather_kernel<<<dim3(unsigned(blocks)), 256, 0, s>>>(
+      static_cast<const uint4*>(feat), S, L, vec, seq, pos, valid_len, A, B,
+      static_cast<uint4*>(out), row_valid);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const LossPlan& plan, const float* part, int mode, float gamma,
+                           const float* row_mask, const int32_t* corpus_tok, float* loss_row,
+                           float* ent_row, float* lse_d, float* lse_t, int32_t* argmax_d,
+                           int32_t* argmax_t, float* gap_d, float* gap_t, float* logp_x,
+                           float* weight, double* anchor_part, cudaStream_t s) {
+  const int A = plan.N / plan.B;
+  combine_kernel<<<(A + 7) / 8, 256, 0, s>>>(plan, part, mode, gamma, row_mask, corpus_tok,
+                                             loss_row, ent_row, lse_d, lse_t, argmax_d, argmax_t,
+                                             gap_d, gap_t, logp_x, weight, anchor_part);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(const double* anchor_part, int A, float lam, float* loss_total,
+                            float* weight_sum, cudaStream_t s) {
+  finalize_kernel<<<1, 1024, 0, s>>>(anchor_part, A, lam, loss_total, weight_sum);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_accept_len(const int32_t* am_d, const int32_t* am_t, const float* active,
+                              int A, int B, int32_t* acc, int64_t* hist, cudaStream_t s) {
+  if (hist != nullptr) {
+    cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(int64_t) * size_t(B + 1), s);
+    if (e != cudaSuccess) return e;
+  }
+  accept_len_kernel<<<(A + 7) / 8, 256, 0, s>>>(am_d, am_t, active, A, B, acc,
+                                                reinterpret_cast<unsigned long long*>(hist));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,
+                                 const int32_t* argmax_t, const float* row_mask, int A, int B,
+                                 float gamma, int hard, float* weight, cudaStream_t s) {
+  erase_weights_kernel<<<(A + 7) / 8, 256, 0, s>>>(logp_x, corpus_tok, argmax_t, row_mask, A, B,
+                                                   gamma, hard, weight);
+  return cudaGetLastError();
+}
+
+}  // namespace alr

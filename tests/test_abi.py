@@ -1,0 +1,70 @@
+"""The C-ABI library builds, loads, and exports every function include/alr.h declares.
+
+No kernel is launched here (these run without a GPU)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_38795_gb300 import alr, build_lib
+
+HEADER = os.path.join(build_lib.ROOT, "include", "alr.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(alr_[a-z0-9_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def libalr():
+    build_lib.build()
+    return ctypes.CDLL(build_lib.LIB)
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for need in ("alr_gather_ira_blocks", "alr_slot_loss_fwd", "alr_slot_loss_bwd",
+                 "alr_accept_len", "alr_erase_weights"):
+        assert need in names
+
+
+def test_every_declared_symbol_is_exported(libalr):
+    missing = [n for n in _declared() if not hasattr(libalr, n)]
+    assert not missing, missing
+
+
+def test_binding_covers_the_header():
+    assert sorted(alr.SIGNATURES) == _declared()
+
+
+def test_struct_layouts_match_the_header():
+    # alr_params: int64 N, five int32, two floats -> 8 + 20 + 8 = 36, padded to 40
+    assert ctypes.sizeof(alr.AlrParams) == 40
+    assert alr.AlrParams.lam.offset == 28 and alr.AlrParams.gamma.offset == 32
+    assert ctypes.sizeof(alr.AlrFwdOutputs) == 12 * 8
+
+
+def test_argument_errors_are_reported_without_a_launch(libalr):
+    lib = alr.lib()
+    assert lib.alr_version().decode().startswith("libalr")
+    bad = alr.make_params(N=30, d=64, V=128, B=16)          # N not a multiple of B
+    assert lib.alr_fwd_workspace_size(ctypes.byref(bad)) == 0
+    out = alr.AlrFwdOutputs()
+    rc = lib.alr_slot_loss_fwd(ctypes.byref(bad), None, None, None, None, None,
+                               ctypes.byref(out), None, 0, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    assert "multiple of B" in lib.alr_last_error().decode()
+    bad_b = alr.make_params(N=66, d=64, V=128, B=33)
+    rc = lib.alr_slot_loss_bwd(ctypes.byref(bad_b), *([None] * 10), 0, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    rc = lib.alr_accept_len(None, None, None, 4, 0, None, None, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    rc = lib.alr_erase_weights(None, None, None, None, 4, 8, 0.0, 0, None, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    rc = lib.alr_gather_ira_blocks(None, 1, 8, 12, alr.ALR_BF16, None, None, None, 2, 4, None,
+                                   None, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG                   # 12 * 2 bytes is not a multiple of 16

@@ -1,0 +1,235 @@
+"""GPU path (through the C ABI) against the CPU oracle, element by element, on seeded inputs
+that span several tiles and ragged tails, plus the degenerate cases of the method."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import alr_oracle as orc
+from paper_2609_38795_gb300 import alr, build_lib, synthetic
+from tests import parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    build_lib.build()
+    alr.lib()
+    assert alr.alr_device_supported() == alr.ALR_OK, alr.alr_last_error()
+
+
+def _inputs(d, V, A, B, sigma, dtype, seed):
+    b = synthetic.slot_batch(d, V, A, B, sigma, dtype=dtype, device="cuda", seed=seed)
+    return b["Hd"], b["Ht"], b["W"]
+
+
+def _oracle_fwd(Hd, Ht, W, B, **kw):
+    return orc.slot_loss_forward(P.np64(Hd), P.np64(Ht), P.np64(W), B, **kw)
+
+
+def _erase_tokens(Ht, W, rate, seed):
+    """Corpus tokens: the oracle's greedy target token, replaced at `rate` by a random one."""
+    greedy = np.argmax(P.np64(Ht) @ P.np64(W), axis=1)
+    mask, tok = synthetic.corpus_replacement(len(greedy), W.shape[1], rate, seed=seed)
+    return synthetic.corpus_tokens(torch.from_numpy(greedy), mask, tok).cuda()
+
+
+# ------------------------------------------------------------------------- gather ---
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_gather_matches_oracle_bit_for_bit(dtype):
+    g = torch.Generator().manual_seed(3)
+    S, L, d, A, B = 5, 70, 264, 37, 16
+    F = torch.randn(S, L, d, generator=g).to(dtype)
+    seq = torch.randint(-1, S + 1, (A,), generator=g, dtype=torch.int32)      # some invalid
+    pos = torch.randint(-2, L - 4, (A,), generator=g, dtype=torch.int32)      # some past L-B
+    vlen = torch.randint(0, L + 3, (A,), generator=g, dtype=torch.int32)
+    for use_vlen in (False, True):
+        out = torch.full((A * B, d), 7.0, dtype=dtype, device="cuda")
+        valid = torch.full((A * B,), -1.0, device="cuda")
+        alr.alr_gather_ira_blocks(F.cuda(), seq.cuda(), pos.cuda(), B, out, valid,
+                                  valid_len=vlen.cuda() if use_vlen else None)
+        ref, rv = orc.gather_ira_blocks(F.float().numpy(), seq.numpy(), pos.numpy(), B,
+                                        valid_len=vlen.numpy() if use_vlen else None)
+        assert np.array_equal(out.float().cpu().numpy(), ref)
+        assert np.array_equal(valid.cpu().numpy(), rv)
+
+
+def test_gather_ira_secondary_blocks_mask():
+    """Secondary blocks at offsets j in 2..14 of 15 stored rows: valid rows are 1[j+k <= K]."""
+    K, d, A = 15, 64, 13
+    prim = torch.randn(A, K, d).to(torch.bfloat16).cuda()
+    seq = torch.arange(A, dtype=torch.int32).cuda()
+    j = torch.arange(2, K, dtype=torch.int32).cuda()
+    out = torch.empty(A * K, d, dtype=torch.bfloat16, device="cuda")
+    valid = torch.empty(A * K, device="cuda")
+    alr.alr_gather_ira_blocks(prim, seq, j, K, out, valid,
+                              valid_len=torch.full((A,), K, dtype=torch.int32, device="cuda"))
+    v = valid.cpu().numpy().reshape(A, K)
+    for a in range(A):
+        jj = a + 2
+        assert v[a].tolist() == [1.0 if jj + k <= K else 0.0 for k in range(1, K + 1)]
+    assert v.sum(axis=1).mean() == 7.0
+
+
+def test_gather_empty_batch():
+    F = torch.zeros(1, 4, 8, dtype=torch.bfloat16, device="cuda")
+    e = torch.empty(0, dtype=torch.int32, device="cuda")
+    out = torch.empty(0, 8, dtype=torch.bfloat16, device="cuda")
+    alr.alr_gather_ira_blocks(F, e, e, 4, out)
+
+
+# ------------------------------------------------------------------------ forward ---
+def test_tiny_fp32_forward_backward_full_parity():
+    """The tiny fp32 workload (d=256, V=4096, B=8, 64 anchors), every row and gradient."""
+    wl = synthetic.WORKLOADS["tiny"]
+    Hd, Ht, W = _inputs(wl.d, wl.V, wl.A, wl.B, 0.5, torch.float32, seed=0)
+    sl = P.gpu_forward(Hd, Ht, W, wl.B)
+    g = P.fwd_to_numpy(sl)
+    r = _oracle_fwd(Hd, Ht, W, wl.B)
+    P.compare_forward(g, r)
+    acc, hist = sl.accept()
+    acc_r, _ = orc.accept_len(r["argmax_d"], r["argmax_t"], wl.B)
+    P.compare_accept(P.npi(acc), P.npi(hist), acc_r, r["gap_d"], r["gap_t"], wl.B)
+    dH = torch.empty(wl.N, wl.d, device="cuda")
+    dW0 = torch.randn(wl.d, wl.V, device="cuda") * 1e-3
+    dW = dW0.clone()
+    sl.backward(Hd, Ht, W, dH, dW)
+    torch.cuda.synchronize()
+    G = orc.logit_grad(r["z_d"], r["z_t"], r["weight"], 1.0)
+    dH_r, dW_r = orc.slot_loss_backward(P.np64(Hd), P.np64(W), G)
+    assert P.max_norm_rel(P.np64(dH), dH_r) <= P.GRAD_RTOL
+    assert P.max_norm_rel(P.np64(dW - dW0), dW_r) <= P.GRAD_RTOL
+    assert alr.alr_device_status() == alr.ALR_OK
+
+
+@pytest.mark.parametrize("mode", [alr.ALR_MODE_ALR, alr.ALR_MODE_ERASE_SOFT, alr.ALR_MODE_ERASE_HARD])
+def test_ragged_bf16_forward_backward(mode):
+    """Ragged everywhere: N = 160 rows (1.25 row tiles), d = 200 (K tail), V = 1000 (7.8
+    vocabulary tiles), a masked row per anchor, lambda and gamma off their defaults."""
+    A, B, d, V, lam, gamma = 10, 16, 200, 1000, 1.013441, 0.5
+    Hd, Ht, W = _inputs(d, V, A, B, 0.5, torch.bfloat16, seed=11 + mode)
+    mask = torch.ones(A * B, device="cuda")
+    mask[5::B] = 0.0
+    tok = _erase_tokens(Ht, W, 0.2, seed=5) if mode != alr.ALR_MODE_ALR else None
+    sl = P.gpu_forward(Hd, Ht, W, B, mode=mode, lam=lam, gamma=gamma, row_mask=mask, corpus_tok=tok)
+    g = P.fwd_to_numpy(sl)
+    r = _oracle_fwd(Hd, Ht, W, B, mode=mode, gamma=gamma, lam=lam, row_mask=P.np64(mask),
+                    corpus_tok=None if tok is None else P.npi(tok))
+    P.compare_forward(g, r, mode=mode)
+    dH = torch.empty(A * B, d, device="cuda")
+    dW = torch.zeros(d, V, device="cuda")
+    sl.backward(Hd, Ht, W, dH, dW)
+    torch.cuda.synchronize()
+    G = orc.logit_grad(r["z_d"], r["z_t"], r["weight"], lam)
+    dH_r, dW_r = orc.slot_loss_backward(P.np64(Hd), P.np64(W), G)
+    assert P.max_norm_rel(P.np64(dH), dH_r) <= P.GRAD_RTOL
+    assert P.max_norm_rel(P.np64(dW), dW_r) <= P.GRAD_RTOL
+    assert np.all(P.np64(dH)[5::B] == 0)                   # masked rows get no gradient
+
+
+def test_small_bf16_forward_full_parity():
+    """The small workload (d=2048, V=32000, B=16, 256 anchors): every row, forward only."""
+    wl = synthetic.WORKLOADS["small"]
+    Hd, Ht, W = _inputs(wl.d, wl.V, wl.A, wl.B, wl.sigma, torch.bfloat16, seed=0)
+    sl = P.gpu_forward(Hd, Ht, W, wl.B)
+    g = P.fwd_to_numpy(sl)
+    r = _oracle_fwd(Hd, Ht, W, wl.B)
+    near = P.compare_forward(g, r)
+    acc, hist = sl.accept()
+    acc_r, _ = orc.accept_len(r["argmax_d"], r["argmax_t"], wl.B)
+    excluded = P.compare_accept(P.npi(acc), P.npi(hist), acc_r, r["gap_d"], r["gap_t"], wl.B)
+    # near-ties are a property of the data (top-2 gaps of 32000 logits of std ~0.9); the
+    # count is reported, and every other row matched exactly
+    print(f"small: {near} near-tie rows of {wl.N}, {excluded} anchors excluded from acc-len")
+    assert near < wl.N // 4
+
+
+@pytest.mark.parametrize("B", [1, 3, 32])
+def test_degenerate_shapes(B):
+    """Vocabulary smaller than one tile, hidden size below one pipeline stage, B = 1 and 32."""
+    A, d, V = 7, 8, 24
+    Hd, Ht, W = _inputs(d, V, A, B, 1.0, torch.bfloat16, seed=B)
+    W = (W.float() * 20).to(torch.bfloat16)                  # sharpen the tiny problem
+    sl = P.gpu_forward(Hd, Ht, W, B)
+    r = _oracle_fwd(Hd, Ht, W, B)
+    P.compare_forward(P.fwd_to_numpy(sl), r)
+
+
+def test_identical_hidden_states_give_entropy_and_full_acceptance():
+    """H_d = H_t: the loss equals the label entropy (Gibbs equality) and every slot is
+    accepted; the gradient vanishes up to rounding."""
+    A, B, d, V = 8, 16, 128, 640
+    Hd, _, W = _inputs(d, V, A, B, 0.5, torch.bfloat16, seed=21)
+    sl = P.gpu_forward(Hd, Hd, W, B)
+    g = P.fwd_to_numpy(sl)
+    np.testing.assert_allclose(g["loss_row"], g["ent_row"], rtol=1e-5, atol=1e-5)
+    acc, hist = sl.accept()
+    assert P.npi(hist)[B] == A
+    dH = torch.empty(A * B, d, device="cuda")
+    sl.backward(Hd, Hd, W, dH)
+    torch.cuda.synchronize()
+    assert dH.abs().max().item() < 1e-4
+
+
+def test_zero_total_weight():
+    A, B, d, V = 4, 8, 64, 256
+    Hd, Ht, W = _inputs(d, V, A, B, 0.5, torch.bfloat16, seed=31)
+    sl = P.gpu_forward(Hd, Ht, W, B, row_mask=torch.zeros(A * B, device="cuda"))
+    assert sl.out["loss_total"].item() == 0.0 and sl.out["weight_sum"].item() == 0.0
+    dH = torch.full((A * B, d), 5.0, device="cuda")
+    dW = torch.zeros(d, V, device="cuda")
+    sl.backward(Hd, Ht, W, dH, dW)
+    torch.cuda.synchronize()
+    assert dH.abs().max().item() == 0.0 and dW.abs().max().item() == 0.0
+
+
+def test_constructed_exact_ties_take_the_lower_id():
+    """Head columns 3 and 9 identical (and dominant): both logits tie exactly, id 3 wins."""
+    A, B, d, V = 2, 8, 64, 256
+    Hd, Ht, W = _inputs(d, V, A, B, 0.5, torch.bfloat16, seed=41)
+    Hd = Hd.abs().to(torch.bfloat16)
+    Ht = Ht.abs().to(torch.bfloat16)
+    W[:, 3] = 1.0
+    W[:, 9] = 1.0
+    W[:, 200] = 1.0
+    sl = P.gpu_forward(Hd, Ht, W, B)
+    assert torch.all(sl.out["argmax_d"] == 3) and torch.all(sl.out["argmax_t"] == 3)
+    assert torch.all(sl.out["gap_d"] == 0)
+
+
+# ------------------------------------------------------------- row-level kernels ---
+@pytest.mark.parametrize("B", [1, 5, 16, 32])
+def test_accept_len_bit_exact(B):
+    g = torch.Generator().manual_seed(B)
+    A = 301
+    am_t = torch.randint(0, 3, (A * B,), generator=g, dtype=torch.int32)
+    am_d = torch.where(torch.rand(A * B, generator=g) < 0.85, am_t,
+                       torch.randint(0, 3, (A * B,), generator=g, dtype=torch.int32))
+    active = (torch.rand(A * B, generator=g) < 0.95).float()
+    acc = torch.empty(A, dtype=torch.int32, device="cuda")
+    hist = torch.full((B + 1,), 99, dtype=torch.int64, device="cuda")
+    alr.alr_accept_len(am_d.cuda(), am_t.cuda(), B, acc, hist, active=active.cuda())
+    acc_r, hist_r = orc.accept_len(am_d.numpy(), am_t.numpy(), B, active=active.numpy())
+    assert np.array_equal(P.npi(acc), acc_r)
+    assert np.array_equal(P.npi(hist), hist_r)
+
+
+@pytest.mark.parametrize("hard", [0, 1])
+def test_erase_weights_kernel(hard):
+    g = torch.Generator().manual_seed(7 + hard)
+    A, B, gamma = 50, 16, 2.0
+    logp = -torch.rand(A * B, generator=g) * 3
+    am_t = torch.randint(0, 4, (A * B,), generator=g, dtype=torch.int32)
+    tok = torch.where(torch.rand(A * B, generator=g) < 0.8, am_t,
+                      torch.randint(0, 4, (A * B,), generator=g, dtype=torch.int32))
+    mask = (torch.rand(A * B, generator=g) < 0.9).float()
+    w = torch.empty(A * B, device="cuda")
+    alr.alr_erase_weights(B, gamma, hard, w, logp_x=logp.cuda(), corpus_tok=tok.cuda(),
+                          argmax_t=am_t.cuda(), row_mask=mask.cuda())
+    gate = orc.erase_gate(B, logp_x=logp.double().numpy(), corpus_tok=tok.numpy(),
+                          argmax_t=am_t.numpy(), hard=bool(hard))
+    ref = np.tile(orc.slot_envelope(B, gamma), A) * mask.double().numpy() * gate
+    np.testing.assert_allclose(P.np64(w), ref, rtol=1e-5, atol=1e-7)
