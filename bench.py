@@ -1,0 +1,402 @@
+#!/usr/bin/env python3
+"""Throughput of the ALR slot-loss hot path on GB300.
+
+One step = the whole path over one batch of the 8B-text workload (d=4096, V=151936, B=16,
+2048 anchors = 32768 slot rows; seeded synthetic inputs, rollout feature buffer of 16
+sequences x 4096 positions):
+    IRA gather of the target hidden rows  ->  fused forward (logits, online LSE, soft CE,
+    greedy argmaxes, slot weights, Eq. 1)  ->  accepted length  ->  logit gradient G
+    (recomputed tiles)  ->  dH_d = G W^T  ->  dW += H_d^T G.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
+
+Prints one JSON line (rank 0).  `value` is slot rows per second over all ranks with inputs
+resident in HBM; `e2e` repeats the measurement with the step's inputs copied from pinned host
+memory and the loss / acceptance histogram read back inside the timed region.  Under
+torchrun every rank runs its own batch (weak scaling, no collective on the data path).
+`--impl reference` times the CPU oracle on a bounded sample of the same workload.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ALR slot-loss fwd+bwd rows/s and % bf16 tensor peak (d=4096,V=151936,B=16)"
+UNIT = "rows/s"
+WORKLOAD = "text8b"
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["gpu", "reference"], default="gpu")
+    ap.add_argument("--sigma", type=float, default=0.5)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-anchors", type=int, default=1)
+    ap.add_argument("--anchors", type=int, default=0,
+                    help="profiling only: fewer anchors than the workload (config says so)")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return dict(bf16=j["bf16_tflops"], bf16_sustained=j["bf16_tflops_sustained"],
+                    hbm=j["hbm_gbs"], source="measured")
+    return dict(bf16=1900.0, bf16_sustained=1700.0, hbm=6800.0, source="fallback")
+
+
+# ------------------------------------------------------------------ clocks sampler ---
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------- CPU oracle ---
+def oracle_sample(wl, inputs, n_anchors):
+    """Rows of the workload for the CPU oracle: the first n_anchors anchors' rows and W."""
+    import numpy as np
+    rows = n_anchors * wl.B
+    Hd = inputs["Hd"][:rows].float().cpu().numpy()
+    Ht = inputs["Ht"][:rows].float().cpu().numpy()
+    W = inputs["W"].float().cpu().numpy()
+    mask = inputs["row_valid"][:rows].float().cpu().numpy().astype(np.float64)
+    return Hd, Ht, W, mask
+
+
+def oracle_step(wl, Hd, Ht, W, mask):
+    """The oracle's fwd + bwd over its sample (as it stands; its own fp64 conversions)."""
+    from oracle import alr_oracle as orc
+    out = orc.slot_loss_forward(Hd, Ht, W, wl.B, row_mask=mask)
+    G = orc.logit_grad(out["z_d"], out["z_t"], out["weight"], 1.0)
+    orc.slot_loss_backward(Hd, W, G)
+    return out["loss_total"]
+
+
+def cores_used():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def time_oracle(wl, inputs, n_anchors, reps, budget_s=30.0):
+    Hd, Ht, W, mask = oracle_sample(wl, inputs, n_anchors)
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        oracle_step(wl, Hd, Ht, W, mask)
+        times.append(time.perf_counter() - t0)
+        if sum(times) > budget_s:
+            break
+    rows = n_anchors * wl.B
+    return rows * len(times) / sum(times), times
+
+
+# ------------------------------------------------------------------------ GPU arm ---
+def make_inputs(wl, sigma, device, seed):
+    import torch
+    from paper_2609_38795_gb300 import synthetic
+    b = synthetic.rollout_batch(wl.d, wl.V, wl.A, wl.B, wl.S, wl.L, sigma, dtype=torch.bfloat16,
+                                device=device, seed=seed)
+    b["Ht"] = torch.empty(wl.N, wl.d, dtype=torch.bfloat16, device=device)
+    b["row_valid"] = torch.empty(wl.N, dtype=torch.float32, device=device)
+    return b
+
+
+class Step:
+    """Buffers and the sequence of C-ABI calls of one step."""
+    N_PHASES = 6
+    PHASES = ["gather", "fwd", "accept_len", "logit_grad", "dH_gemm", "dW_gemm"]
+    KERNELS_PER_STEP = 8   # gather, fwd (loss, combine, finalize), accept, logit grad, dH, dW
+
+    def __init__(self, wl, inputs, device):
+        import torch
+        from paper_2609_38795_gb300 import alr
+        self.alr, self.wl, self.x = alr, wl, inputs
+        self.sl = alr.SlotLoss(wl.N, wl.d, wl.V, wl.B, dtype=torch.bfloat16, device=device)
+        self.G = torch.empty(wl.N, wl.V, dtype=torch.bfloat16, device=device)
+        self.dH = torch.empty(wl.N, wl.d, dtype=torch.float32, device=device)
+        self.dW = torch.zeros(wl.d, wl.V, dtype=torch.float32, device=device)
+
+    def run(self, events=None):
+        alr, x, sl, wl = self.alr, self.x, self.sl, self.wl
+        rec = (lambda i: events[i].record()) if events is not None else (lambda i: None)
+        rec(0)
+        alr.alr_gather_ira_blocks(x["F"], x["seq"], x["pos"], wl.B, x["Ht"], x["row_valid"])
+        rec(1)
+        sl.forward(x["Hd"], x["Ht"], x["W"], row_mask=x["row_valid"])
+        rec(2)
+        sl.accept(active=x["row_valid"])
+        rec(3)
+        o = sl.out
+        alr.alr_logit_grad(sl.params, x["Hd"], x["Ht"], x["W"], o["weight"], o["weight_sum"],
+                           o["lse_d"], o["lse_t"], self.G)
+        rec(4)
+        alr.alr_gemm(self.G, x["W"], self.dH, wl.N, wl.d, wl.V)                    # G W^T
+        rec(5)
+        alr.alr_gemm(x["Hd"], self.G, self.dW, wl.d, wl.V, wl.N, a_mn=True, b_mn=True,
+                     accumulate=True)                                               # H_d^T G
+        rec(6)
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_38795_gb300 import alr, build_lib, synthetic
+
+    torch.cuda.set_device(local_rank)
+    device = f"cuda:{local_rank}"
+    build_lib.build()
+    alr.lib()
+    if alr.alr_device_supported() != alr.ALR_OK:
+        raise RuntimeError(alr.alr_last_error())
+    wl = synthetic.WORKLOADS[WORKLOAD]
+    if args.anchors:
+        import dataclasses
+        wl = dataclasses.replace(wl, A=args.anchors, S=max(1, args.anchors // 128))
+    x = make_inputs(wl, args.sigma, device, seed=rank)
+    step = Step(wl, x, device)
+    for _ in range(args.warmup):
+        step.run()
+    torch.cuda.synchronize()
+    if alr.alr_device_status() != alr.ALR_OK:
+        raise RuntimeError("device status: " + alr.alr_last_error())
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(K)]
+    clocks = Clocks(local_rank)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_stop = torch.cuda.Event(enable_timing=True)
+    t_start.record()
+    for k in range(K):
+        step.run(ev[k])
+    t_stop.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_stop)
+    phase_ms = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
+                for i, p in enumerate(Step.PHASES)}
+    if alr.alr_device_status() != alr.ALR_OK:
+        raise RuntimeError("device status: " + alr.alr_last_error())
+    acc_hist = step.sl.hist.cpu().tolist()
+    loss = step.sl.out["loss_total"].item()
+
+    # ---- end to end through host buffers (pinned), copies inside the timed region ----
+    e2e = None
+    if not args.no_e2e:
+        host = {k: x[k].cpu().pin_memory() for k in ("Hd", "F", "seq", "pos")}
+        res = {"loss": torch.empty(2, dtype=torch.float32).pin_memory(),
+               "hist": torch.empty(wl.B + 1, dtype=torch.int64).pin_memory()}
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = 2 * 4 + (wl.B + 1) * 8
+
+        def e2e_step():
+            for k in host:
+                x[k].copy_(host[k], non_blocking=True)
+            step.run()
+            res["loss"][0:1].copy_(step.sl.out["loss_total"], non_blocking=True)
+            res["loss"][1:2].copy_(step.sl.out["weight_sum"], non_blocking=True)
+            res["hist"].copy_(step.sl.hist, non_blocking=True)
+
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(K):
+            e2e_step()
+        b.record()
+        torch.cuda.synchronize()
+        e2e_ms = a.elapsed_time(b)
+        if world > 1:
+            dist.barrier()
+        e2e = {"ms": e2e_ms, "h2d": h2d, "d2h": d2h}
+
+    # ---- max over ranks ----
+    times = torch.tensor([total_ms, e2e["ms"] if e2e else 0.0], device=device, dtype=torch.float64)
+    if world > 1:
+        dist.all_reduce(times, op=dist.ReduceOp.MAX)
+    total_ms, e2e_ms = times.tolist()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rps, ts = time_oracle(wl, x, args.cpu_sample_anchors, reps=3)
+        cpu = {"value": rps, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+               "sample": f"{args.cpu_sample_anchors} anchor(s) x {wl.B} rows of the {WORKLOAD} "
+                         f"workload, full d={wl.d} and V={wl.V}, fwd+bwd in fp64, "
+                         f"{len(ts)} repetition(s), {sum(ts):.1f} s"}
+    if rank != 0:
+        return None
+
+    pk = peaks()
+    NdV = wl.N * wl.d * wl.V
+    ms_step = total_ms / K
+    rows_per_s = world * wl.N * K / (total_ms / 1e3)
+    exec_tf = 12 * NdV / (ms_step / 1e3) / 1e12
+    algo_tf = 8 * NdV / (ms_step / 1e3) / 1e12
+    # dominant kernel by measured time; its algorithmic flops per launch
+    flops = {"fwd": 4 * NdV, "logit_grad": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
+    dom = max(flops, key=lambda p: phase_ms[p])
+    achieved = flops[dom] / (phase_ms[dom] / 1e3) / 1e12
+    out = {
+        "metric": METRIC, "value": rows_per_s, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{WORKLOAD}{' PROFILING SUBSET' if args.anchors else ''}: d={wl.d} V={wl.V} B={wl.B} A={wl.A} rows={wl.N} "
+                               f"sigma={args.sigma} feature buffer {wl.S}x{wl.L}",
+                   "global_batch_rows": world * wl.N, "l2": "inputs larger than L2 "
+                   "(W 1.24 GB, H 268 MB each, G 10 GB)", "parallelism": f"replicas{world}"},
+        "tensor_tflops": {"executed_12NdV": exec_tf, "algorithmic_8NdV": algo_tf,
+                          "pct_peak_executed": exec_tf / pk["bf16"],
+                          "pct_peak_algorithmic": algo_tf / pk["bf16"],
+                          "peak_tflops": pk["bf16"], "peak_source": pk["source"]},
+        "phase_ms": phase_ms,
+        "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved,
+                     "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+                     "frac": achieved / pk["bf16_sustained"],
+                     "frac_of_burst_peak": achieved / pk["bf16"], "traffic": None,
+                     "peak_note": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
+                     "flops_per_launch": flops[dom]},
+        "gpu_launches": Step.KERNELS_PER_STEP * K,
+        "loss": loss, "acc_hist": acc_hist,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+    }
+    if e2e is not None:
+        out["e2e"] = {"value": world * wl.N * K / (e2e_ms / 1e3), "unit": UNIT,
+                      "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
+                      "ms_per_step": e2e_ms / K}
+    return out
+
+
+# ---------------------------------------------------------------- reference arm ---
+def run_reference(args):
+    import torch
+    from paper_2609_38795_gb300 import synthetic
+    wl = synthetic.WORKLOADS[WORKLOAD]
+    n_a = args.cpu_sample_anchors
+    rows = n_a * wl.B
+    # the sample's inputs, drawn on the CPU with the same recipe (first n_a anchors)
+    g = torch.Generator().manual_seed(0)
+    W = (torch.randn(wl.d, wl.V, generator=g) * synthetic.HEAD_STD).to(torch.bfloat16)
+    Ht = torch.randn(rows, wl.d, generator=g).to(torch.bfloat16)
+    Hd = (Ht.float() + args.sigma * torch.randn(rows, wl.d, generator=g)).to(torch.bfloat16)
+    x = {"Hd": Hd, "Ht": Ht, "W": W, "row_valid": torch.ones(rows)}
+    Hd_n, Ht_n, W_n, mask = oracle_sample(wl, x, n_a)
+    for _ in range(args.warmup):
+        oracle_step(wl, Hd_n, Ht_n, W_n, mask)
+    ts = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_step(wl, Hd_n, Ht_n, W_n, mask)
+        ts.append(time.perf_counter() - t0)
+    total = sum(ts)
+    v = rows * len(ts) / total
+    sample = (f"{n_a} anchor(s) x {wl.B} rows of the {WORKLOAD} workload per step, full d={wl.d} "
+              f"and V={wl.V}, fwd+bwd in fp64")
+    return {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(ts),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": f"{WORKLOAD}{' PROFILING SUBSET' if args.anchors else ''}: d={wl.d} V={wl.V} B={wl.B} (CPU oracle sample)"},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    out = run_gpu(args, rank, world, local_rank)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -148,6 +148,20 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
                       const float* lse_t, float* dHd, float* dW, void* workspace,
                       size_t ws_bytes, void* stream);
 
+/* Workspace bytes alr_logit_grad needs for `p` (0 for bf16; W^T for fp32). */
+size_t alr_logit_grad_workspace_size(const alr_params* p);
+
+/*
+ * The first step of alr_slot_loss_bwd on its own: the gradient of Eq. 1 with respect to the
+ * drafter logits, G[r, v] = lambda * omega_r / sum omega * (q[r, v] - p[r, v]), recomputed
+ * tile by tile from Hd, Ht, W and the forward's lse_d, lse_t, written to G [N, V] (element
+ * type p->dtype, row-major).  dH_d = G W^T and dW += H_d^T G then follow with alr_gemm
+ * (bf16: layouts (0, 0) and (1, 1)).
+ */
+int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                   const float* weight, const float* weight_sum, const float* lse_d,
+                   const float* lse_t, void* G, void* workspace, size_t ws_bytes, void* stream);
+
 /*
  * Greedy accepted length per anchor (Sec. 3.2: slot k counts only when slots 1..k-1 were
  * accepted; MAT tau = acc + 1, Sec. 4).

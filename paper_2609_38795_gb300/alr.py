@@ -53,6 +53,9 @@ SIGNATURES = {
     "alr_bwd_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_slot_loss_bwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_logit_grad_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
+    "alr_logit_grad": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
     "alr_erase_weights": (_c_int, [_c_p, _c_p, _c_p, _c_p, _c_i32, _c_i32, _c_f, _c_i32, _c_p,
                                    _c_p]),
@@ -159,6 +162,18 @@ def alr_slot_loss_bwd(params, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, dHd, 
                                    _ptr(weight), _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t),
                                    _ptr(dHd), _ptr(dW), _ptr(workspace),
                                    workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def alr_logit_grad_workspace_size(params) -> int:
+    return lib().alr_logit_grad_workspace_size(ctypes.byref(params))
+
+
+def alr_logit_grad(params, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, workspace=None,
+                   stream=None):
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().alr_logit_grad(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W), _ptr(weight),
+                                _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t), _ptr(G),
+                                _ptr(workspace), nbytes, _stream(stream)))
 
 
 def alr_accept_len(argmax_d, argmax_t, B, acc_len, hist=None, active=None, stream=None):

@@ -328,20 +328,85 @@ size_t alr_bwd_workspace_size(const alr_params* p) {
   return bwd_layout(p).total;
 }
 
+}  // extern "C"
+
+namespace {
+
+// Checks shared by the backward entry points; fills `info`.
+int check_bwd_args(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                   const float* weight, const float* weight_sum, const float* lse_d,
+                   const float* lse_t, DevInfo* info) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || Ht == nullptr || W == nullptr || weight == nullptr ||
+      weight_sum == nullptr || lse_d == nullptr || lse_t == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required backward input pointer is NULL");
+  if (!aligned16(Hd) || !aligned16(Ht) || !aligned16(W))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht and W must be 16-byte aligned");
+  return require_sm103(info);
+}
+
+// G = lambda omega / sum omega (q - p), recomputing the logit tiles (the fused backward kernel).
+int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                    const float* weight, const float* weight_sum, const float* lse_d,
+                    const float* lse_t, void* G, void* wt, const DevInfo& info, cudaStream_t s) {
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  const uint32_t kke = k_per_row(dt);
+  int rc;
+  CUtensorMap m_hd, m_ht, m_w, m_gs;
+  if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = head_map(&m_w, p, W, wt, s)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_gs, G, dt, p->V, p->N, p->V * es, kke, 32)) != ALR_OK) return rc;
+  alr::LossArgs args{};
+  args.plan = loss_plan(p, info.sms, true);
+  args.lse_d = lse_d;
+  args.lse_t = lse_t;
+  args.weight = weight;
+  args.weight_sum = weight_sum;
+  args.lam = p->lambda;
+  args.status = alr::device_status_ptr();
+  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  cudaError_t e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, m_gs, args, s);
+  if (e != cudaSuccess) return cuda_fail(e, "logit-gradient kernel launch");
+  return ALR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t alr_logit_grad_workspace_size(const alr_params* p) {
+  if (check_params(p) != ALR_OK) return 0;
+  return p->dtype == ALR_F32 ? round_up(size_t(p->V) * p->d * 4, 1024) : 0;
+}
+
+int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+                   const float* weight, const float* weight_sum, const float* lse_d,
+                   const float* lse_t, void* G, void* workspace, size_t ws_bytes, void* stream) {
+  DevInfo info;
+  int rc = check_bwd_args(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, &info);
+  if (rc != ALR_OK) return rc;
+  if (G == nullptr || !aligned16(G)) return fail(ALR_ERR_INVALID_ARG, "G must be non-NULL and 16-byte aligned");
+  const size_t need = alr_logit_grad_workspace_size(p);
+  if (need > 0 && (workspace == nullptr || ws_bytes < need || !aligned16(workspace)))
+    return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
+                ws_bytes, need);
+  return logit_grad_impl(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, workspace, info,
+                         static_cast<cudaStream_t>(stream));
+}
+
 int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
                       const float* weight, const float* weight_sum, const float* lse_d,
                       const float* lse_t, float* dHd, float* dW, void* workspace, size_t ws_bytes,
                       void* stream) {
-  int rc = check_params(p);
-  if (rc != ALR_OK) return rc;
-  if (Hd == nullptr || Ht == nullptr || W == nullptr || weight == nullptr ||
-      weight_sum == nullptr || lse_d == nullptr || lse_t == nullptr || dHd == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "a required backward pointer is NULL");
-  if (!aligned16(Hd) || !aligned16(Ht) || !aligned16(W) || !aligned16(dHd) ||
-      (dW != nullptr && !aligned16(dW)))
-    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht, W, dHd and dW must be 16-byte aligned");
   DevInfo info;
-  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  int rc = check_bwd_args(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, &info);
+  if (rc != ALR_OK) return rc;
+  if (dHd == nullptr) return fail(ALR_ERR_INVALID_ARG, "dHd is NULL");
+  if (!aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
+    return fail(ALR_ERR_INVALID_ARG, "dHd and dW must be 16-byte aligned");
   const size_t need = alr_bwd_workspace_size(p);
   if (workspace == nullptr || ws_bytes < need)
     return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
@@ -356,36 +421,22 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
   void* G = ws + lay.g_off;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;
-  CUtensorMap m_hd, m_ht, m_w, m_gs;
-  if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_gs, G, dt, p->V, p->N, p->V * es, kke, 32)) != ALR_OK) return rc;
-
-  alr::LossArgs args{};
-  args.plan = loss_plan(p, info.sms, true);
-  args.lse_d = lse_d;
-  args.lse_t = lse_t;
-  args.weight = weight;
-  args.weight_sum = weight_sum;
-  args.lam = p->lambda;
-  args.status = alr::device_status_ptr();
-  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, m_gs, args, s);
-  if (e != cudaSuccess) return cuda_fail(e, "backward logit-gradient kernel launch");
+  rc = logit_grad_impl(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, ws + lay.wt_off, info, s);
+  if (rc != ALR_OK) return rc;
+  int* status = alr::device_status_ptr();
 
   // dH_d = G W^T: A = G [N, V] K-major, B = W [d, V] K-major.
   CUtensorMap m_ga, m_wk;
   if ((rc = make_map(&m_ga, G, dt, p->V, p->N, p->V * es, kke, 128)) != ALR_OK) return rc;
   if ((rc = make_map(&m_wk, W, dt, p->V, p->d, p->V * es, kke, 256)) != ALR_OK) return rc;
   alr::GemmArgs gh = gemm_plan(int(p->N), p->d, p->V, dHd, p->d, info.sms);
-  gh.status = args.status;
+  gh.status = status;
   e = alr::launch_plain_gemm(dt, false, false, false, m_ga, m_wk, gh, s);
   if (e != cudaSuccess) return cuda_fail(e, "dH GEMM launch");
 
   if (dW != nullptr) {
     alr::GemmArgs gw = gemm_plan(p->d, p->V, int(p->N), dW, p->V, info.sms);
-    gw.status = args.status;
+    gw.status = status;
     CUtensorMap m_ha, m_gb;
     if (dt == ALR_BF16) {
       // dW += H_d^T G: A = H_d read as [K = N, M = d] (MN-major), B = G [K = N, V] (MN-major).
