@@ -132,6 +132,34 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
                       const alr_fwd_outputs* out, void* workspace, size_t ws_bytes,
                       void* stream);
 
+/*
+ * Forward pass for callers that cannot allocate device memory.  The paper has no counterpart:
+ * this is a deployment variant of alr_slot_loss_fwd.
+ *
+ * Who needs it: a caller whose host process has handed all device memory to its own pool at
+ * start-up and allows no further allocation, or a caller on a latency-critical path where a
+ * device allocation (which can synchronise the whole device) is not acceptable, cannot
+ * provide the workspace alr_slot_loss_fwd asks for.  This call takes the same arguments minus
+ * the workspace and runs the same kernels; their scratch lives in a fixed array of
+ * ALR_NOALLOC_SCRATCH_BYTES bytes in device global memory that belongs to the library image.
+ * It calls no cudaMalloc, cudaFree or other allocating routine.
+ *
+ *   - Limit: problems whose alr_fwd_workspace_size exceeds ALR_NOALLOC_SCRATCH_BYTES are
+ *     rejected with ALR_ERR_INVALID_ARG and a message naming both sizes (bf16 at d=4096,
+ *     B=16 on a 152-SM GB300: about 16 900 rows).
+ *   - Memory: every device that loads the library holds the array until the process exits.
+ *   - Set-up: the first call on a device (with that device current) looks up the array's
+ *     device address; make that first call before any stream capture.
+ *   - Sharing: all calls on a device share the one array and it keeps the last call's
+ *     contents.  Nothing in it needs clearing (the kernels overwrite what they read), but
+ *     calls whose work overlaps on the GPU (different streams, or different host threads
+ *     without ordering) race on it and give undefined results: serialise them.
+ */
+#define ALR_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+int alr_slot_loss_fwd_noalloc(const alr_params* p, const void* Hd, const void* Ht,
+                              const void* W, const float* row_mask, const int32_t* corpus_tok,
+                              const alr_fwd_outputs* out, void* stream);
+
 /* Workspace bytes alr_slot_loss_bwd needs for `p` (includes the logit gradient, N*V*elem). */
 size_t alr_bwd_workspace_size(const alr_params* p);
 

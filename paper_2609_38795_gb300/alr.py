@@ -50,6 +50,8 @@ SIGNATURES = {
     "alr_fwd_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_slot_loss_fwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p,
                                    ctypes.POINTER(AlrFwdOutputs), _c_p, _c_sz, _c_p]),
+    "alr_slot_loss_fwd_noalloc": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
+                                           _c_p, ctypes.POINTER(AlrFwdOutputs), _c_p]),
     "alr_bwd_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_slot_loss_bwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
@@ -154,6 +156,15 @@ def alr_slot_loss_fwd(params, Hd, Ht, W, out: dict, workspace, row_mask=None, co
                                    _ptr(row_mask), _ptr(corpus_tok), ctypes.byref(o),
                                    _ptr(workspace), workspace.numel() * workspace.element_size(),
                                    _stream(stream)))
+
+
+def alr_slot_loss_fwd_noalloc(params, Hd, Ht, W, out: dict, row_mask=None, corpus_tok=None,
+                              stream=None):
+    """alr_slot_loss_fwd without a workspace (scratch in the library's fixed device array)."""
+    o = AlrFwdOutputs(**{f: _ptr(out.get(f)) for f in _FWD_FIELDS})
+    _check(lib().alr_slot_loss_fwd_noalloc(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W),
+                                           _ptr(row_mask), _ptr(corpus_tok), ctypes.byref(o),
+                                           _stream(stream)))
 
 
 def alr_slot_loss_bwd(params, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, dHd, dW, workspace,

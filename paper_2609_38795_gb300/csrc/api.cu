@@ -212,6 +212,10 @@ int head_map(CUtensorMap* m, const alr_params* p, const void* W, void* wt, cudaS
 
 }  // namespace
 
+namespace alr {
+int set_last_error(int code, const char* msg) { return fail(code, "%s", msg); }
+}  // namespace alr
+
 extern "C" {
 
 const char* alr_version(void) { return "libalr 0.1 (sm_103a)"; }

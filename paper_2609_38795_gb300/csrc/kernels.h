@@ -101,6 +101,9 @@ cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,
 cudaError_t launch_transpose32(const float* in, float* out, int R, int C, int ld_out,
                                cudaStream_t s);
 
+// Record `msg` as this host thread's alr_last_error() text and return `code` (api.cu).
+int set_last_error(int code, const char* msg);
+
 // Per-device status word (status.cu).
 int* device_status_ptr();
 
