@@ -155,6 +155,38 @@ def time_oracle(wl, inputs, n_anchors, reps, budget_s=30.0):
     return rows * len(times) / sum(times), times
 
 
+# ------------------------------------------------------------- gather bandwidth ---
+def gather_bandwidth(device, reps=20, warmup=3):
+    """IRA gather at the vl7b shape (F [32, 2048, 3584] bf16, 512 anchors x 16 rows): each
+    repetition is timed alone with CUDA events after a 256 MB write that flushes L2."""
+    import torch
+    from paper_2609_38795_gb300 import alr, synthetic
+    wl = synthetic.WORKLOADS["vl7b"]
+    g = torch.Generator(device=device).manual_seed(5)
+    F = torch.randn(wl.S, wl.L, wl.d, generator=g, device=device).to(torch.bfloat16)
+    seq, pos = synthetic.anchor_positions(wl.A, wl.S, wl.L, wl.B, device=device, g=g)
+    out = torch.empty(wl.N, wl.d, dtype=torch.bfloat16, device=device)
+    valid = torch.empty(wl.N, dtype=torch.float32, device=device)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    ts = []
+    for i in range(warmup + reps):
+        flush.fill_(i & 0xFF)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        alr.alr_gather_ira_blocks(F, seq, pos, wl.B, out, valid)
+        b.record()
+        torch.cuda.synchronize()
+        if i >= warmup:
+            ts.append(a.elapsed_time(b))
+    ms = statistics.median(ts)
+    nbytes = 2 * wl.N * wl.d * 2 + wl.N * 4       # rows read + rows written + row_valid
+    gbs = nbytes / (ms / 1e3) / 1e9
+    return {"workload": f"vl7b: {wl.A} anchors x {wl.B} rows, d={wl.d}, feature buffer "
+                        f"{wl.S}x{wl.L}", "bytes": nbytes, "us_median": ms * 1e3,
+            "GB/s": gbs, "l2": "flushed (256 MB write) before each repetition", "reps": reps}
+
+
 # ------------------------------------------------------------------------ GPU arm ---
 def make_inputs(wl, sigma, device, seed):
     import torch
@@ -290,6 +322,8 @@ def run_gpu(args, rank, world, local_rank):
         dist.all_reduce(times, op=dist.ReduceOp.MAX)
     total_ms, e2e_ms = times.tolist()
 
+    gather = gather_bandwidth(device) if rank == 0 else None
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rps, ts = time_oracle(wl, x, args.cpu_sample_anchors, reps=3)
@@ -330,6 +364,7 @@ def run_gpu(args, rank, world, local_rank):
                      "peak_note": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
                      "flops_per_launch": flops[dom]},
         "gpu_launches": Step.KERNELS_PER_STEP * K,
+        "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
         "loss": loss, "acc_hist": acc_hist,
         "clocks": clk,
         "cpu_baseline": cpu,

@@ -184,14 +184,16 @@ def slot_loss_forward(Hd, Ht, W, B, mode=MODE_ALR, gamma=2.0, lam=1.0, row_mask=
 # ----------------------------------------------------------------------------------------
 # Backward pass: gradient of L with respect to the drafter logits, H_d and W
 # ----------------------------------------------------------------------------------------
-def logit_grad(z_d, z_t, weight, lam) -> np.ndarray:
+def logit_grad(z_d, z_t, weight, lam, weight_sum=None) -> np.ndarray:
     """dL/dz_d[r, v] = lam * omega_r / sum omega * (q[r, v] - p[r, v]).
 
     From l_r = LSE(z_d) - sum_v p_v z_d,v: d l_r / d z_d,v = q_v - p_v.  The label p, the
     weights omega and the erase gate are target-side quantities and carry no gradient.
+    weight_sum: the normaliser sum omega of Eq. 1 over the whole batch, when only some of its
+    rows are passed (default: the sum of the given weights).
     """
     weight = _f64(weight)
-    wsum = weight.sum()
+    wsum = weight.sum() if weight_sum is None else float(weight_sum)
     if wsum == 0.0:
         return np.zeros_like(_f64(z_d))
     q = softmax(z_d)

@@ -124,14 +124,20 @@ int check_params(const alr_params* p) {
   return ALR_OK;
 }
 
+// Vocabulary tile width of the fused loss kernels (columns of z_d and of z_t per tile).
+#ifndef ALR_LOSS_BN
+#define ALR_LOSS_BN 256
+#endif
+
 alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
   alr::LossPlan P{};
   P.N = int(p->N);
   P.d = p->d;
   P.V = p->V;
   P.B = p->B;
+  P.bn = ALR_LOSS_BN;
   P.n_rb = int((p->N + 127) / 128);
-  P.n_vt = (p->V + 127) / 128;
+  P.n_vt = (p->V + P.bn - 1) / P.bn;
   P.group_rows = P.n_rb < 8 ? P.n_rb : 8;
   if (bwd) {
     P.n_vs = P.n_vt;  // one tile per unit
@@ -140,6 +146,7 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
     if (vs < 1) vs = 1;
     P.n_vs = vs < P.n_vt ? vs : P.n_vt;
   }
+  P.n_parts = P.n_vs * (P.bn / 128);
   P.n_units = P.n_rb * P.n_vs;
   P.grid = sms < P.n_units ? sms : P.n_units;
   return P;
@@ -155,7 +162,7 @@ FwdLayout fwd_layout(const alr_params* p, int sms) {
   const alr::LossPlan P = loss_plan(p, sms, false);
   FwdLayout L{};
   L.part_off = 0;
-  L.anchor_off = round_up(size_t(alr::kPFields) * P.n_vs * size_t(P.N) * sizeof(float), 1024);
+  L.anchor_off = round_up(size_t(alr::kPFields) * P.n_parts * size_t(P.N) * sizeof(float), 1024);
   L.wt_off = L.anchor_off + round_up(2 * sizeof(double) * size_t(P.N / P.B), 1024);
   L.total = L.wt_off;
   if (p->dtype == ALR_F32) L.total += round_up(size_t(p->V) * p->d * sizeof(float), 1024);
@@ -207,7 +214,7 @@ int head_map(CUtensorMap* m, const alr_params* p, const void* W, void* wt, cudaS
   cudaError_t e = alr::launch_transpose32(static_cast<const float*>(W), static_cast<float*>(wt),
                                           p->d, p->V, p->d, s);
   if (e != cudaSuccess) return cuda_fail(e, "head transpose launch");
-  return make_map(m, wt, ALR_F32, p->d, p->V, uint64_t(p->d) * 4, kke, 128);
+  return make_map(m, wt, ALR_F32, p->d, p->V, uint64_t(p->d) * 4, kke, ALR_LOSS_BN);
 }
 
 }  // namespace
@@ -358,13 +365,13 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
   const size_t es = elem_size(dt);
   const uint32_t kke = k_per_row(dt);
   int rc;
-  CUtensorMap m_hd, m_ht, m_w, m_gs;
+  CUtensorMap m_hd, m_ht, m_w;
   if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
   if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
   if ((rc = head_map(&m_w, p, W, wt, s)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_gs, G, dt, p->V, p->N, p->V * es, kke, 32)) != ALR_OK) return rc;
   alr::LossArgs args{};
   args.plan = loss_plan(p, info.sms, true);
+  args.G = G;
   args.lse_d = lse_d;
   args.lse_t = lse_t;
   args.weight = weight;
@@ -372,7 +379,7 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
   args.lam = p->lambda;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, m_gs, args, s);
+  cudaError_t e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "logit-gradient kernel launch");
   return ALR_OK;
 }

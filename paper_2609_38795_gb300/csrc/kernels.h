@@ -14,16 +14,18 @@ namespace alr {
 //   share both their hidden-state tiles and their head tiles through L2.
 struct LossPlan {
   int N, d, V, B;
+  int bn;          // vocabulary columns per tile (128 or 256)
   int n_rb;        // ceil(N / 128)
-  int n_vt;        // ceil(V / 128)
-  int n_vs;        // vocabulary splits (partial statistics per row and split)
+  int n_vt;        // ceil(V / bn)
+  int n_vs;        // vocabulary splits
+  int n_parts;     // partial records per row: n_vs * (bn / 128), one per split and half
   int group_rows;  // row blocks per group
   int n_units;     // n_rb * n_vs
   int grid;        // persistent CTAs
 };
 
-// Partial statistics of one row over one vocabulary split (structure of arrays, field-major:
-// part[f * n_vs * N + vs * N + row]).
+// Partial statistics of one row over the columns of one vocabulary split seen by one
+// epilogue thread (structure of arrays, field-major: part[f * n_parts * N + part * N + row]).
 enum PartField {
   kPMd = 0,   // running max of z_d
   kPSd,       // sum exp(z_d - m_d)
@@ -45,6 +47,7 @@ struct LossArgs {
   LossPlan plan;
   float* part;                // forward: partial statistics
   const int32_t* corpus_tok;  // forward: nullable
+  void* G;                    // backward: logit gradient [N, V] (element type of the inputs)
   const float* lse_d;         // backward
   const float* lse_t;
   const float* weight;
@@ -57,10 +60,7 @@ struct LossArgs {
 cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
                             const CUtensorMap& w, const LossArgs& args, cudaStream_t s);
 cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const CUtensorMap& g_store,
-                            const LossArgs& args, cudaStream_t s);
-size_t loss_fwd_smem_bytes(int dtype);
-size_t loss_bwd_smem_bytes(int dtype);
+                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s);
 
 // Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm.cu).
 struct GemmArgs {

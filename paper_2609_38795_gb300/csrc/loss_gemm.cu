@@ -1,19 +1,24 @@
 // Fused dual-GEMM kernels of the slot loss on the sm_103a tensor cores.
 //
-// Both kernels compute, for a 128-row block of H_d and H_t and a 128-column tile of the
+// Both kernels compute, for a 128-row block of H_d and H_t and a kBN-column tile of the
 // vocabulary head W, the two logit tiles z_d = H_d W and z_t = H_t W with tcgen05.mma into
-// tensor memory (fp32 accumulators, 2 x 128 columns per tile, double-buffered so the epilogue
-// of one tile overlaps the products of the next).  The logits never leave the SM:
+// tensor memory (fp32 accumulators; the two tiles share every W stage).  The logits never
+// leave the SM:
 //   forward  - the epilogue folds each tile into running per-row statistics (online max /
 //              sum-exp for both sides, the label-weighted sums behind the soft cross-entropy
 //              of Eq. 1, greedy top-2 with lowest-index ties, z_t at the corpus token) and
-//              writes one partial record per row and vocabulary split;
+//              writes one partial record per row, vocabulary split and 128-column half;
 //   backward - the epilogue forms G = lambda omega_r / sum omega (q - p) for the tile
-//              (the gradient of Eq. 1 with respect to z_d) and streams it out with TMA.
+//              (the gradient of Eq. 1 with respect to z_d) and stores it to global memory.
 //
-// Warp roles (256 threads): warp 0 issues TMA loads, warp 1 owns tensor memory and issues
-// the MMAs from one lane, warps 4-7 run the epilogue (warp w reads TMEM lanes 32(w%4)..+31,
-// one row per thread).  Every pipeline wait is bounded (tc_common.cuh).
+// Tile widths: kBN = 256 (default) uses all 512 TMEM columns for one tile (z_d | z_t) and
+// 64 KB pipeline stages (1024 tensor cycles of work each); kBN = 128 double-buffers the
+// accumulators with 48 KB stages (512 cycles each).
+//
+// Warp roles: warp 0 issues TMA loads, warp 1 owns tensor memory and issues the MMAs from one
+// lane, warps 2-3 idle, warps 4.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one
+// row per thread) and columns [128 h, 128 h + 128) of the tile, h = (w-4)/4.  Every pipeline
+// wait is bounded (tc_common.cuh).
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -21,13 +26,10 @@ namespace alr {
 namespace {
 
 constexpr int kBM = 128;                 // rows per tile = TMEM lanes
-constexpr int kBN = 128;                 // vocabulary columns per tile (per GEMM)
-constexpr int kThreads = 256;
 constexpr int kEpiWarp0 = 4;
-constexpr int kEpiThreads = 128;
-constexpr int kTileBytes = kBM * 128;    // a 128-extent operand over 128 bytes of K
-constexpr int kStageBytes = 3 * kTileBytes;  // H_d tile, H_t tile, W tile
+constexpr int kATileBytes = kBM * 128;   // a 128-row operand over 128 bytes of K
 constexpr int kCtrlBytes = 256;
+constexpr int kSmemBudget = 227 * 1024;
 
 template <typename Elem>
 struct Geo {
@@ -35,20 +37,27 @@ struct Geo {
   static constexpr int kKE = 128 / kElem;          // K elements per pipeline stage
   static constexpr int kMmaK = 32 / kElem;         // K per MMA instruction
   static constexpr int kChunkMN = 128 / kElem;     // MN elements per 128-byte chunk
-  static constexpr int kNChunks = kBN / kChunkMN;  // W chunks per tile
   static constexpr uint32_t kChunkBytes = kKE * 128;
   static constexpr bool kTf32 = (kElem == 4);
 };
 
-template <bool kBwd>
-constexpr int stages() { return kBwd ? 3 : 4; }
+template <int kBN>
+struct Shape {
+  static constexpr int kBTileBytes = kBN * 128;
+  static constexpr int kStageBytes = 2 * kATileBytes + kBTileBytes;
+  static constexpr int kAccCols = 2 * kBN;           // z_d columns, then z_t columns
+  static constexpr int kAccBufs = 512 / kAccCols;    // 2 for kBN = 128, 1 for kBN = 256
+  static constexpr int kHalves = kBN / 128;          // epilogue warps per TMEM lane quarter
+  static constexpr int kEpiWarps = 4 * kHalves;
+  static constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
+  static constexpr int kFit = (kSmemBudget - 1024 - kCtrlBytes) / kStageBytes;
+  static constexpr int kStages = kFit < 4 ? kFit : 4;
+  static constexpr size_t kSmem = 1024 + size_t(kStages) * kStageBytes + kCtrlBytes;
+};
 
-template <typename Elem, bool kBwd>
-constexpr size_t smem_bytes() {
-  return 1024 + size_t(stages<kBwd>()) * kStageBytes + (kBwd ? size_t(kBM) * kBN * sizeof(Elem) : 0) +
-         kCtrlBytes;
-}
-
+// Unit u -> (row block, vocabulary split).  Units go group by group (group_rows row blocks);
+// inside a group the row block varies fastest, and the split index is rotated by the group
+// number so that every CTA of a static round-robin sees every split size in turn.
 ALR_DEV void decode_unit(const LossPlan& p, int u, int& rb, int& vs) {
   const int per_group = p.group_rows * p.n_vs;
   const int full = p.n_rb / p.group_rows;
@@ -62,8 +71,9 @@ ALR_DEV void decode_unit(const LossPlan& p, int u, int& rb, int& vs) {
     w = u - full * per_group;
     gr = p.n_rb - full * p.group_rows;
   }
-  vs = w / gr;
-  rb = g * p.group_rows + (w - vs * gr);
+  const int k = w / gr;
+  rb = g * p.group_rows + (w - k * gr);
+  vs = (k + g) % p.n_vs;
 }
 
 ALR_DEV int split_begin(const LossPlan& p, int vs) {
@@ -72,7 +82,7 @@ ALR_DEV int split_begin(const LossPlan& p, int vs) {
 
 ALR_DEV float f32(uint32_t x) { return __uint_as_float(x); }
 
-// Running statistics of one row (forward epilogue).
+// Running statistics of one row over the columns one thread sees (forward epilogue).
 struct RowStats {
   float m_d, s_d, m_t, s_t, u, w;
   float b_d, sec_d, b_t, sec_t, zx;
@@ -178,21 +188,19 @@ ALR_DEV bool warp_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
 
 // kWMN: the head tile is read MN-major straight from W [d, V] (bf16), or K-major from a
 // transposed copy W^T [V, d] (fp32 inputs, whose tf32 products take K-major operands only).
-template <typename Elem, bool kBwd, bool kWMN>
-__global__ void __launch_bounds__(kThreads, 1)
+template <typename Elem, bool kBwd, bool kWMN, int kBN>
+__global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
     loss_gemm_kernel(const __grid_constant__ CUtensorMap tm_hd,
                      const __grid_constant__ CUtensorMap tm_ht,
-                     const __grid_constant__ CUtensorMap tm_w,
-                     const __grid_constant__ CUtensorMap tm_g, const LossArgs args) {
+                     const __grid_constant__ CUtensorMap tm_w, const LossArgs args) {
   using G = Geo<Elem>;
-  constexpr int kStages = stages<kBwd>();
-  constexpr int kGStageBytes = kBwd ? kBM * kBN * int(sizeof(Elem)) : 0;
+  using S = Shape<kBN>;
+  constexpr int kStages = S::kStages;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_1024(smem_raw);
   uint8_t* stage_mem = smem;
-  uint8_t* gstage = smem + kStages * kStageBytes;
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(gstage + kGStageBytes);
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kStages * S::kStageBytes);
   uint64_t* empty_bar = full_bar + kStages;
   uint64_t* tfull_bar = empty_bar + kStages;
   uint64_t* tempty_bar = tfull_bar + 2;
@@ -210,9 +218,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&full_bar[i], 1);
       mbar_init(&empty_bar[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < S::kAccBufs; ++i) {
       mbar_init(&tfull_bar[i], 1);
-      mbar_init(&tempty_bar[i], kEpiThreads / 32);
+      mbar_init(&tempty_bar[i], S::kEpiWarps);
     }
     mbar_init(drain_bar, 1);
     *abort_word = 0;
@@ -222,7 +230,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm_hd);
     tma_prefetch_desc(&tm_ht);
     tma_prefetch_desc(&tm_w);
-    if (kBwd) tma_prefetch_desc(&tm_g);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
@@ -250,17 +257,17 @@ __global__ void __launch_bounds__(kThreads, 1)
               ok = false;
               break;
             }
-            uint8_t* sb = stage_mem + stage * kStageBytes;
-            mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
+            uint8_t* sb = stage_mem + stage * S::kStageBytes;
+            mbar_arrive_expect_tx(&full_bar[stage], S::kStageBytes);
             tma_load_2d(sb, &tm_hd, &full_bar[stage], kb * G::kKE, rb * kBM);
-            tma_load_2d(sb + kTileBytes, &tm_ht, &full_bar[stage], kb * G::kKE, rb * kBM);
+            tma_load_2d(sb + kATileBytes, &tm_ht, &full_bar[stage], kb * G::kKE, rb * kBM);
             if constexpr (kWMN) {
 #pragma unroll
-              for (int c = 0; c < G::kNChunks; ++c)
-                tma_load_2d(sb + 2 * kTileBytes + c * G::kChunkBytes, &tm_w, &full_bar[stage],
+              for (int c = 0; c < kBN / G::kChunkMN; ++c)
+                tma_load_2d(sb + 2 * kATileBytes + c * G::kChunkBytes, &tm_w, &full_bar[stage],
                             vt * kBN + c * G::kChunkMN, kb * G::kKE);
             } else {
-              tma_load_2d(sb + 2 * kTileBytes, &tm_w, &full_bar[stage], kb * G::kKE, vt * kBN);
+              tma_load_2d(sb + 2 * kATileBytes, &tm_w, &full_bar[stage], kb * G::kKE, vt * kBN);
             }
             armed |= 1u << stage;
             armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
@@ -293,21 +300,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d_acc = tmem_base + uint32_t(abuf * 2 * kBN);
+          const uint32_t d_acc = tmem_base + uint32_t(abuf * S::kAccCols);
           for (int kb = 0; kb < n_kb; ++kb) {
             if (!mbar_wait(&full_bar[stage], phase, ab)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_u32(stage_mem + stage * kStageBytes);
+            const uint32_t sa = smem_u32(stage_mem + stage * S::kStageBytes);
 #pragma unroll
             for (int kk = 0; kk < G::kKE / G::kMmaK; ++kk) {
               const uint64_t ad = sdesc_sw128(sa + kk * 32, 16, 1024);
-              const uint64_t at = sdesc_sw128(sa + kTileBytes + kk * 32, 16, 1024);
+              const uint64_t at = sdesc_sw128(sa + kATileBytes + kk * 32, 16, 1024);
               const uint64_t bd =
-                  kWMN ? sdesc_sw128(sa + 2 * kTileBytes + kk * G::kMmaK * 128, G::kChunkBytes, 1024)
-                       : sdesc_sw128(sa + 2 * kTileBytes + kk * 32, 16, 1024);
+                  kWMN ? sdesc_sw128(sa + 2 * kATileBytes + kk * G::kMmaK * 128, G::kChunkBytes, 1024)
+                       : sdesc_sw128(sa + 2 * kATileBytes + kk * 32, 16, 1024);
               const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
               mma_issue<G::kTf32>(d_acc, ad, bd, idesc, acc);
               mma_issue<G::kTf32>(d_acc + kBN, at, bd, idesc, acc);
@@ -320,7 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (!ok) break;
           mma_commit(&tfull_bar[abuf]);
-          if (++abuf == 2) {
+          if (++abuf == S::kAccBufs) {
             abuf = 0;
             aphase ^= 1;
           }
@@ -333,8 +340,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= kEpiWarp0) {
     // -------------------------------------------------------------------- epilogue ---
     const int q = warp & 3;
+    const int h = (warp - kEpiWarp0) >> 2;
     const int row_in_tile = q * 32 + lane;
-    const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16);
+    const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(h * 128);
     int abuf = 0;
     uint32_t aphase = 0;
     bool ok = true;
@@ -354,11 +362,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t tb = lane_addr + uint32_t(abuf * 2 * kBN);
-          const int vbase = vt * kBN;
-          const bool full_tile = vbase + kBN <= P.V;
+          const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
+          const int vbase = vt * kBN + h * 128;
+          const bool full_tile = vbase + 128 <= P.V;
 #pragma unroll 1
-          for (int c = 0; c < kBN / 32; ++c) {
+          for (int c = 0; c < 4; ++c) {
             uint32_t rd[32], rt[32];
             tmem_ld32(tb + c * 32, rd);
             tmem_ld32(tb + kBN + c * 32, rt);
@@ -375,14 +383,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&tempty_bar[abuf]);
-          if (++abuf == 2) {
+          if (++abuf == S::kAccBufs) {
             abuf = 0;
             aphase ^= 1;
           }
         }
         if (ok && row_ok) {
-          const size_t fs = size_t(P.n_vs) * P.N;
-          float* o = args.part + size_t(vs) * P.N + row;
+          const size_t fs = size_t(P.n_parts) * P.N;
+          float* o = args.part + size_t(vs * S::kHalves + h) * P.N + row;
           o[kPMd * fs] = st.m_d;
           o[kPSd * fs] = st.s_d;
           o[kPMt * fs] = st.m_t;
@@ -405,73 +413,60 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float ws = *args.weight_sum;
           cw = ws > 0.f ? args.lam * args.weight[row] / ws : 0.f;
         }
+        Elem* grow = static_cast<Elem*>(args.G) + size_t(row_ok ? row : 0) * size_t(P.V);
         for (int vt = split_begin(P, vs); vt < vt1; ++vt) {
           if (!warp_wait(&tfull_bar[abuf], aphase, ab)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          // Each warp owns rows 32q..32q+31 of the staging tile and stores them itself, so
-          // the epilogue warps never wait on one another.  The slab is free once this
-          // warp's previous store has read it.
-          if (lane == 0) tma_store_wait_read_all();
-          __syncwarp();
-          const uint32_t tb = lane_addr + uint32_t(abuf * 2 * kBN);
+          const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
+          const int vbase = vt * kBN + h * 128;
 #pragma unroll 1
-          for (int c = 0; c < kBN / 32; ++c) {
+          for (int c = 0; c < 4; ++c) {
             uint32_t rd[32], rt[32];
             tmem_ld32(tb + c * 32, rd);
             tmem_ld32(tb + kBN + c * 32, rt);
             tmem_ld_wait();
             reg_fence(rd);
             reg_fence(rt);
-            float g[32];
+            const int v0 = vbase + c * 32;
+            if (row_ok && v0 < P.V) {
+              float g[32];
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-              g[j] = cw * (ex2(fmaf(f32(rd[j]), kLog2e, ad)) - ex2(fmaf(f32(rt[j]), kLog2e, at)));
-            if constexpr (sizeof(Elem) == 2) {
-              uint8_t* rowp = gstage + (c >> 1) * (kBM * 128) + row_in_tile * 128;
+              for (int j = 0; j < 32; ++j)
+                g[j] = cw * (ex2(fmaf(f32(rd[j]), kLog2e, ad)) - ex2(fmaf(f32(rt[j]), kLog2e, at)));
+              if constexpr (sizeof(Elem) == 2) {
 #pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                const int unit = ((c & 1) * 4 + i) ^ (row_in_tile & 7);
-                uint4 v;
-                v.x = pack_bf16x2(g[8 * i + 0], g[8 * i + 1]);
-                v.y = pack_bf16x2(g[8 * i + 2], g[8 * i + 3]);
-                v.z = pack_bf16x2(g[8 * i + 4], g[8 * i + 5]);
-                v.w = pack_bf16x2(g[8 * i + 6], g[8 * i + 7]);
-                *reinterpret_cast<uint4*>(rowp + unit * 16) = v;
-              }
-            } else {
-              uint8_t* rowp = gstage + c * (kBM * 128) + row_in_tile * 128;
+                for (int i = 0; i < 4; ++i) {
+                  if (v0 + 8 * i < P.V) {   // V % 8 == 0: a vector is all in or all out
+                    uint4 v;
+                    v.x = pack_bf16x2(g[8 * i + 0], g[8 * i + 1]);
+                    v.y = pack_bf16x2(g[8 * i + 2], g[8 * i + 3]);
+                    v.z = pack_bf16x2(g[8 * i + 4], g[8 * i + 5]);
+                    v.w = pack_bf16x2(g[8 * i + 6], g[8 * i + 7]);
+                    *reinterpret_cast<uint4*>(grow + v0 + 8 * i) = v;
+                  }
+                }
+              } else {
 #pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                const int unit = i ^ (row_in_tile & 7);
-                *reinterpret_cast<float4*>(rowp + unit * 16) =
-                    make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
+                for (int i = 0; i < 8; ++i) {
+                  if (v0 + 4 * i < P.V)
+                    *reinterpret_cast<float4*>(grow + v0 + 4 * i) =
+                        make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
+                }
               }
             }
           }
           tc_fence_before();
-          fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) {
-            mbar_arrive(&tempty_bar[abuf]);
-#pragma unroll
-            for (int b = 0; b < G::kNChunks; ++b)
-              tma_store_2d(&tm_g, gstage + b * (kBM * 128) + q * 32 * 128,
-                           vt * kBN + b * G::kChunkMN, rb * kBM + q * 32);
-            tma_store_commit();
-          }
-          if (++abuf == 2) {
+          if (lane == 0) mbar_arrive(&tempty_bar[abuf]);
+          if (++abuf == S::kAccBufs) {
             abuf = 0;
             aphase ^= 1;
           }
         }
-        if (!ok) break;
       }
-    }
-    if constexpr (kBwd) {
-      if (lane == 0) tma_store_wait_all();
     }
   }
 
@@ -483,37 +478,39 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <typename Elem, bool kBwd>
+template <typename Elem, bool kBwd, int kBN>
 cudaError_t launch_impl(const CUtensorMap& hd, const CUtensorMap& ht, const CUtensorMap& w,
-                        const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
-  auto kern = loss_gemm_kernel<Elem, kBwd, sizeof(Elem) == 2>;
-  const size_t smem = smem_bytes<Elem, kBwd>();
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+                        const LossArgs& args, cudaStream_t s) {
+  using S = Shape<kBN>;
+  auto kern = loss_gemm_kernel<Elem, kBwd, sizeof(Elem) == 2, kBN>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
   if (e != cudaSuccess) return e;
-  kern<<<args.plan.grid, kThreads, smem, s>>>(hd, ht, w, g, args);
+  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(hd, ht, w, args);
   return cudaGetLastError();
+}
+
+template <bool kBwd>
+cudaError_t dispatch(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
+                     const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
+  if (args.plan.bn == 128) {
+    if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 128>(hd, ht, w, args, s);
+    return launch_impl<float, kBwd, 128>(hd, ht, w, args, s);
+  }
+  if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 256>(hd, ht, w, args, s);
+  return launch_impl<float, kBwd, 256>(hd, ht, w, args, s);
 }
 
 }  // namespace
 
-size_t loss_fwd_smem_bytes(int dtype) {
-  return dtype == 0 ? smem_bytes<__nv_bfloat16, false>() : smem_bytes<float, false>();
-}
-size_t loss_bwd_smem_bytes(int dtype) {
-  return dtype == 0 ? smem_bytes<__nv_bfloat16, true>() : smem_bytes<float, true>();
-}
-
 cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
                             const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
-  if (dtype == 0) return launch_impl<__nv_bfloat16, false>(hd, ht, w, w, args, s);
-  return launch_impl<float, false>(hd, ht, w, w, args, s);
+  return dispatch<false>(dtype, hd, ht, w, args, s);
 }
 
 cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const CUtensorMap& g_store,
-                            const LossArgs& args, cudaStream_t s) {
-  if (dtype == 0) return launch_impl<__nv_bfloat16, true>(hd, ht, w, g_store, args, s);
-  return launch_impl<float, true>(hd, ht, w, g_store, args, s);
+                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
+  return dispatch<true>(dtype, hd, ht, w, args, s);
 }
 
 }  // namespace alr

@@ -14,7 +14,7 @@ __device__ __forceinline__ float quiet_nan() { return __int_as_float(0x7fc00000)
 // ------------------------------------------------------------------ IRA gather ---
 // One warp per output row; each lane moves 16-byte vectors, issuing a batch of loads before
 // the matching stores so that many requests are in flight per SM.
-constexpr int kGatherBatch = 8;
+constexpr int kGatherBatch = 16;
 
 __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ feat, int S, int L,
                                                      int vec_per_row,
@@ -49,7 +49,7 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ f
 #pragma unroll
     for (int j = 0; j < kGatherBatch; ++j) {
       const int i = base + j * 32 + lane;
-      if (i < vec_per_row) dst[i] = v[j];
+      if (i < vec_per_row) __stcs(dst + i, v[j]);
     }
   }
 }
@@ -93,14 +93,14 @@ __global__ void __launch_bounds__(256) combine_kernel(
   if (a >= A) return;
   const bool active = lane < P.B;
   const int r = a * P.B + (active ? lane : 0);
-  const size_t fs = size_t(P.n_vs) * P.N;
+  const size_t fs = size_t(P.n_parts) * P.N;
 
   float Md = -INFINITY, Sd = 0.f, Mt = -INFINITY, St = 0.f, U = 0.f, Wt = 0.f;
   float bd = -INFINITY, secd = -INFINITY, bt = -INFINITY, sect = -INFINITY, zx = quiet_nan();
   int id = 0x7fffffff, it = 0x7fffffff;
   if (active) {
-    for (int vs = 0; vs < P.n_vs; ++vs) {
-      const float* p = part + size_t(vs) * P.N + r;
+    for (int k = 0; k < P.n_parts; ++k) {
+      const float* p = part + size_t(k) * P.N + r;
       const float md = p[kPMd * fs], sd = p[kPSd * fs];
       const float nmd = fmaxf(Md, md);
       Sd = Sd * ex2((Md - nmd) * kLog2e) + sd * ex2((md - nmd) * kLog2e);
@@ -112,10 +112,10 @@ __global__ void __launch_bounds__(256) combine_kernel(
       U = U * so + p[kPU * fs] * sn;
       Wt = Wt * so + p[kPW * fs] * sn;
       Mt = nmt;
-      // top-2 merge: the earlier split holds the lower indices, so ties keep the incumbent
+      // top-2 merge; equal leaders go to the lower token id
       const float b2 = p[kPBd * fs], s2 = p[kPSecd * fs];
       const int i2 = __float_as_int(p[kPId * fs]);
-      if (b2 > bd) {
+      if (b2 > bd || (b2 == bd && i2 < id)) {
         secd = fmaxf(bd, s2);
         bd = b2;
         id = i2;
@@ -124,7 +124,7 @@ __global__ void __launch_bounds__(256) combine_kernel(
       }
       const float b3 = p[kPBt * fs], s3 = p[kPSect * fs];
       const int i3 = __float_as_int(p[kPIt * fs]);
-      if (b3 > bt) {
+      if (b3 > bt || (b3 == bt && i3 < it)) {
         sect = fmaxf(bt, s3);
         bt = b3;
         it = i3;
