@@ -97,6 +97,17 @@ int alr_device_supported(void);
 int alr_device_status(void* stream, int clear);
 
 /*
+ * Test hook for the failure-detection path (the paper has no counterpart).  With enable != 0,
+ * the next alr_slot_loss_fwd launch on any thread withholds the first pipeline stage of each
+ * CTA: nothing ever fills it, so the MMA issuer's bounded wait runs out after about 1.5 s, every
+ * role of the CTA leaves its loop (copies in flight are waited for, tensor memory is released)
+ * and the kernel records ALR_ERR_TIMEOUT in the device status word.  That call's outputs are
+ * meaningless; alr_device_status() then returns ALR_ERR_TIMEOUT and the context stays usable.
+ * Nothing faults, traps or hangs.  The hook disarms itself after one launch.
+ */
+int alr_debug_withhold_next_stage(int enable);
+
+/*
  * IRA gather (Eq. 4; App. A: rollout features stored for y*_1..y*_13).
  *   feat      [S, L, d] features of S rollout sequences of length L, element type `dtype`.
  *   seq, pos  [A] int32: anchor a reads sequence seq[a] from position pos[a].
@@ -155,7 +166,7 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
  *     calls whose work overlaps on the GPU (different streams, or different host threads
  *     without ordering) race on it and give undefined results: serialise them.
  */
-#define ALR_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+#define ALR_NOALLOC_SCRATCH_BYTES (64u * 1024u * 1024u)
 int alr_slot_loss_fwd_noalloc(const alr_params* p, const void* Hd, const void* Ht,
                               const void* W, const float* row_mask, const int32_t* corpus_tok,
                               const alr_fwd_outputs* out, void* stream);

@@ -45,6 +45,7 @@ SIGNATURES = {
     "alr_last_error": (ctypes.c_char_p, []),
     "alr_device_supported": (_c_int, []),
     "alr_device_status": (_c_int, [_c_p, _c_int]),
+    "alr_debug_withhold_next_stage": (_c_int, [_c_int]),
     "alr_gather_ira_blocks": (_c_int, [_c_p, _c_i32, _c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p,
                                        _c_i32, _c_i32, _c_p, _c_p, _c_p]),
     "alr_fwd_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
@@ -132,6 +133,10 @@ def alr_device_supported() -> int:
 
 def alr_device_status(clear=True, stream=None) -> int:
     return lib().alr_device_status(_stream(stream), int(clear))
+
+
+def alr_debug_withhold_next_stage(enable=True) -> int:
+    return lib().alr_debug_withhold_next_stage(int(enable))
 
 
 def alr_gather_ira_blocks(feat, seq, pos, B, out, row_valid=None, valid_len=None, stream=None):

@@ -2,6 +2,7 @@
 // work planning and kernel launches.  No entry point allocates device memory.
 #include <cudaTypedefs.h>
 
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -27,6 +28,9 @@ int cuda_fail(cudaError_t e, const char* what) {
 }
 
 std::mutex g_mu;
+
+// Test hook state: when set, the next forward launch withholds its first pipeline stage.
+std::atomic<int> g_withhold_next{0};
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -83,10 +87,11 @@ size_t elem_size(int dtype) { return dtype == ALR_BF16 ? 2 : 4; }
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// 2-D tiled tensor map with 128-byte swizzle: `inner` contiguous elements per row, `outer`
-// rows `row_bytes` apart; boxes of box_inner x box_outer elements.
+// 2-D tiled tensor map (128-byte swizzle unless stated): `inner` contiguous elements per row,
+// `outer` rows `row_bytes` apart; boxes of box_inner x box_outer elements.
 int make_map(CUtensorMap* m, const void* ptr, int dtype, uint64_t inner, uint64_t outer,
-             uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+             uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer,
+             CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   auto enc = encode_fn();
   if (enc == nullptr) return fail(ALR_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
   cuuint64_t dims[2] = {inner, outer};
@@ -95,7 +100,7 @@ int make_map(CUtensorMap* m, const void* ptr, int dtype, uint64_t inner, uint64_
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(m, dtype == ALR_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
                    2, const_cast<void*>(ptr), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS)
     return fail(ALR_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d) for %llu x %llu", int(r),
@@ -146,7 +151,7 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
     if (vs < 1) vs = 1;
     P.n_vs = vs < P.n_vt ? vs : P.n_vt;
   }
-  P.n_parts = P.n_vs * (P.bn / 128);
+  P.n_parts = P.n_vs * (P.bn / 64);
   P.n_units = P.n_rb * P.n_vs;
   P.grid = sms < P.n_units ? sms : P.n_units;
   return P;
@@ -226,6 +231,11 @@ int set_last_error(int code, const char* msg) { return fail(code, "%s", msg); }
 extern "C" {
 
 const char* alr_version(void) { return "libalr 0.1 (sm_103a)"; }
+
+int alr_debug_withhold_next_stage(int enable) {
+  g_withhold_next.store(enable ? 1 : 0);
+  return ALR_OK;
+}
 
 const char* alr_last_error(void) { return g_err; }
 
@@ -319,6 +329,7 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
   args.part = reinterpret_cast<float*>(ws + lay.part_off);
   args.corpus_tok = p->mode != ALR_MODE_ALR ? corpus_tok : nullptr;
   args.lam = p->lambda;
+  args.withhold_first_stage = g_withhold_next.exchange(0);
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
   e = alr::launch_loss_fwd(dt, m_hd, m_ht, m_w, args, s);
@@ -365,10 +376,14 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
   const size_t es = elem_size(dt);
   const uint32_t kke = k_per_row(dt);
   int rc;
-  CUtensorMap m_hd, m_ht, m_w;
+  CUtensorMap m_hd, m_ht, m_w, m_gs;
   if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
   if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
   if ((rc = head_map(&m_w, p, W, wt, s)) != ALR_OK) return rc;
+  m_gs = m_w;
+  if (dt == ALR_BF16 &&
+      (rc = make_map(&m_gs, G, dt, p->V, p->N, p->V * es, 16, 32, CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
+    return rc;
   alr::LossArgs args{};
   args.plan = loss_plan(p, info.sms, true);
   args.G = G;
@@ -379,7 +394,7 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
   args.lam = p->lambda;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, args, s);
+  cudaError_t e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, m_gs, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "logit-gradient kernel launch");
   return ALR_OK;
 }

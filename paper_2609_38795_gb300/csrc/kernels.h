@@ -18,7 +18,7 @@ struct LossPlan {
   int n_rb;        // ceil(N / 128)
   int n_vt;        // ceil(V / bn)
   int n_vs;        // vocabulary splits
-  int n_parts;     // partial records per row: n_vs * (bn / 128), one per split and half
+  int n_parts;     // partial records per row: n_vs * (bn / 64), one per split and 64-column group
   int group_rows;  // row blocks per group
   int n_units;     // n_rb * n_vs
   int grid;        // persistent CTAs
@@ -54,13 +54,16 @@ struct LossArgs {
   const float* weight_sum;
   float lam;
   int* status;
+  int withhold_first_stage;   // test hook: the producer never fills its first stage
 };
 
 // Fused dual-GEMM kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
 cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
                             const CUtensorMap& w, const LossArgs& args, cudaStream_t s);
+// g_store: bf16 G [N, V] as 16-column x 32-row boxes without swizzle (ignored for fp32).
 cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s);
+                            const CUtensorMap& w, const CUtensorMap& g_store,
+                            const LossArgs& args, cudaStream_t s);
 
 // Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm.cu).
 struct GemmArgs {

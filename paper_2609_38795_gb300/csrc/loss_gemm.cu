@@ -7,17 +7,19 @@
 //   forward  - the epilogue folds each tile into running per-row statistics (online max /
 //              sum-exp for both sides, the label-weighted sums behind the soft cross-entropy
 //              of Eq. 1, greedy top-2 with lowest-index ties, z_t at the corpus token) and
-//              writes one partial record per row, vocabulary split and 128-column half;
+//              writes one partial record per row, vocabulary split and 64-column group;
 //   backward - the epilogue forms G = lambda omega_r / sum omega (q - p) for the tile
-//              (the gradient of Eq. 1 with respect to z_d) and stores it to global memory.
+//              (the gradient of Eq. 1 with respect to z_d) and streams it to global memory
+//              (bf16: through per-warp shared staging and TMA stores).
 //
 // Tile widths: kBN = 256 (default) uses all 512 TMEM columns for one tile (z_d | z_t) and
 // 64 KB pipeline stages (1024 tensor cycles of work each); kBN = 128 double-buffers the
 // accumulators with 48 KB stages (512 cycles each).
 //
 // Warp roles: warp 0 issues TMA loads, warp 1 owns tensor memory and issues the MMAs from one
-// lane, warps 2-3 idle, warps 4.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one
-// row per thread) and columns [128 h, 128 h + 128) of the tile, h = (w-4)/4.  Every pipeline
+// lane, warps 2.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one row per thread)
+// and the 64 columns [64 g, 64 g + 64) of the tile, g = (w-2)/4, in 16-column sub-chunks.
+// Four epilogue warps per SM sub-partition keep the exposed epilogue short.  Every pipeline
 // wait is bounded (tc_common.cuh).
 #include "kernels.h"
 #include "tc_common.cuh"
@@ -26,10 +28,13 @@ namespace alr {
 namespace {
 
 constexpr int kBM = 128;                 // rows per tile = TMEM lanes
-constexpr int kEpiWarp0 = 4;
+constexpr int kEpiWarp0 = 2;
+constexpr int kColsPerWarp = 64;
+constexpr int kSub = 16;                 // columns per TMEM load / processing step
 constexpr int kATileBytes = kBM * 128;   // a 128-row operand over 128 bytes of K
 constexpr int kCtrlBytes = 256;
 constexpr int kSmemBudget = 227 * 1024;
+constexpr int kGStageBytes = 32 * kSub * 2;   // one warp's bf16 G sub-chunk: 32 rows x 16 cols
 
 template <typename Elem>
 struct Geo {
@@ -41,18 +46,19 @@ struct Geo {
   static constexpr bool kTf32 = (kElem == 4);
 };
 
-template <int kBN>
+template <int kBN, bool kStaged>
 struct Shape {
   static constexpr int kBTileBytes = kBN * 128;
   static constexpr int kStageBytes = 2 * kATileBytes + kBTileBytes;
-  static constexpr int kAccCols = 2 * kBN;           // z_d columns, then z_t columns
-  static constexpr int kAccBufs = 512 / kAccCols;    // 2 for kBN = 128, 1 for kBN = 256
-  static constexpr int kHalves = kBN / 128;          // epilogue warps per TMEM lane quarter
-  static constexpr int kEpiWarps = 4 * kHalves;
+  static constexpr int kAccCols = 2 * kBN;             // z_d columns, then z_t columns
+  static constexpr int kAccBufs = 512 / kAccCols;      // 2 for kBN = 128, 1 for kBN = 256
+  static constexpr int kColGroups = kBN / kColsPerWarp;
+  static constexpr int kEpiWarps = 4 * kColGroups;
   static constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
-  static constexpr int kFit = (kSmemBudget - 1024 - kCtrlBytes) / kStageBytes;
+  static constexpr int kStaging = kStaged ? kEpiWarps * 2 * kGStageBytes : 0;
+  static constexpr int kFit = (kSmemBudget - 1024 - kCtrlBytes - kStaging) / kStageBytes;
   static constexpr int kStages = kFit < 4 ? kFit : 4;
-  static constexpr size_t kSmem = 1024 + size_t(kStages) * kStageBytes + kCtrlBytes;
+  static constexpr size_t kSmem = 1024 + size_t(kStages) * kStageBytes + kStaging + kCtrlBytes;
 };
 
 // Unit u -> (row block, vocabulary split).  Units go group by group (group_rows row blocks);
@@ -82,96 +88,116 @@ ALR_DEV int split_begin(const LossPlan& p, int vs) {
 
 ALR_DEV float f32(uint32_t x) { return __uint_as_float(x); }
 
+// Load 16 consecutive 32-bit TMEM columns of this warp's 32 lanes (see tmem_ld32).
+ALR_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+// Maximum of 16 values by a balanced tree (depth 4).
+ALR_DEV float max16(const float (&z)[16]) {
+  float a[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) a[i] = fmaxf(z[2 * i], z[2 * i + 1]);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) a[i] = fmaxf(a[2 * i], a[2 * i + 1]);
+  a[0] = fmaxf(a[0], a[1]);
+  a[2] = fmaxf(a[2], a[3]);
+  return fmaxf(a[0], a[2]);
+}
+
 // Running statistics of one row over the columns one thread sees (forward epilogue).
+// best_x is both the greedy top-1 and the online-softmax reference of side x; s_x sums
+// exp(z_x - best_x); u and w sum exp(z_t - best_t) * z_d and * z_t.
 struct RowStats {
-  float m_d, s_d, m_t, s_t, u, w;
-  float b_d, sec_d, b_t, sec_t, zx;
+  float best_d, sec_d, s_d, best_t, sec_t, s_t, u, w, zx;
   int i_d, i_t;
 };
 
 ALR_DEV void stats_init(RowStats& st) {
-  st.m_d = st.m_t = -INFINITY;
+  st.best_d = st.sec_d = st.best_t = st.sec_t = -INFINITY;
   st.s_d = st.s_t = st.u = st.w = 0.f;
-  st.b_d = st.sec_d = st.b_t = st.sec_t = -INFINITY;
   st.i_d = st.i_t = 0x7fffffff;
   st.zx = __int_as_float(0x7fc00000);
 }
 
-// Greedy top-2 over a chunk in increasing column order; a strictly larger value is needed to
-// take the lead, so the lowest index wins exact ties.
-ALR_DEV void top2_scan(float& best, float& sec, int& idx, const uint32_t (&z)[32], int v0, int nv) {
+// Greedy top-2 with lowest-index ties, given the sub-chunk maximum cm.  Columns reach a
+// thread in increasing order, so an equal later value never takes the lead.
+ALR_DEV void top2_update(float& best, float& sec, int& idx, const float (&z)[16], float cm,
+                         int v0) {
+  sec = fmaxf(sec, fminf(cm, best));
+  if (cm > best) {  // a new leader in this sub-chunk: find its first position and runner-up
+    int jj = kSub - 1;
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    if (j < nv) {
-      const float v = f32(z[j]);
-      if (v > best) {
-        sec = best;
-        best = v;
-        idx = v0 + j;
-      } else if (v > sec) {
-        sec = v;
-      }
-    }
+    for (int j = kSub - 1; j >= 0; --j) jj = (z[j] == cm) ? j : jj;
+    float c2 = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < kSub; ++j) c2 = fmaxf(c2, j == jj ? -INFINITY : z[j]);
+    sec = fmaxf(best, c2);
+    best = cm;
+    idx = v0 + jj;
   }
 }
 
+// Fold one 16-column sub-chunk (nv valid columns) into the running statistics.
 template <bool kFull>
-ALR_DEV void stats_chunk(RowStats& st, const uint32_t (&rd)[32], const uint32_t (&rt)[32], int v0,
-                         int nv, int x) {
-  float cmd = -INFINITY, cmt = -INFINITY;
+ALR_DEV void stats_sub(RowStats& st, const uint32_t (&rd)[16], const uint32_t (&rt)[16], int v0,
+                       int nv, int x) {
+  float zd[16], zt[16];
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    if (kFull || j < nv) {
-      cmd = fmaxf(cmd, f32(rd[j]));
-      cmt = fmaxf(cmt, f32(rt[j]));
-    }
+  for (int j = 0; j < kSub; ++j) {
+    zd[j] = (kFull || j < nv) ? f32(rd[j]) : -INFINITY;
+    zt[j] = (kFull || j < nv) ? f32(rt[j]) : -INFINITY;
   }
-  if (cmd > st.sec_d) top2_scan(st.b_d, st.sec_d, st.i_d, rd, v0, kFull ? 32 : nv);
-  if (cmt > st.sec_t) top2_scan(st.b_t, st.sec_t, st.i_t, rt, v0, kFull ? 32 : nv);
-  const int xr = x - v0;
-  if (xr >= 0 && xr < (kFull ? 32 : nv)) {
-#pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if (j == xr) st.zx = f32(rt[j]);
-  }
-  // target side: sum e, sum e z_d, sum e z_t with e = exp(z_t - m_t)
-  const float nmt = fmaxf(st.m_t, cmt);
-  const float sct = ex2((st.m_t - nmt) * kLog2e);
-  const float bt = -nmt * kLog2e;
+  const float cd = max16(zd), ct = max16(zt);
+  // target side: rescale to the new running maximum, then add this sub-chunk
+  const float nbt = fmaxf(st.best_t, ct);
+  const float sct = ex2((st.best_t - nbt) * kLog2e);
+  const float bt = -nbt * kLog2e;
   float s0 = 0.f, s1 = 0.f, u0 = 0.f, u1 = 0.f, w0 = 0.f, w1 = 0.f;
 #pragma unroll
-  for (int j = 0; j < 32; j += 2) {
+  for (int j = 0; j < kSub; j += 2) {
     if (kFull || j < nv) {
-      const float zt = f32(rt[j]);
-      const float e = ex2(fmaf(zt, kLog2e, bt));
+      const float e = ex2(fmaf(zt[j], kLog2e, bt));
       s0 += e;
-      u0 = fmaf(e, f32(rd[j]), u0);
-      w0 = fmaf(e, zt, w0);
+      u0 = fmaf(e, zd[j], u0);
+      w0 = fmaf(e, zt[j], w0);
     }
     if (kFull || j + 1 < nv) {
-      const float zt = f32(rt[j + 1]);
-      const float e = ex2(fmaf(zt, kLog2e, bt));
+      const float e = ex2(fmaf(zt[j + 1], kLog2e, bt));
       s1 += e;
-      u1 = fmaf(e, f32(rd[j + 1]), u1);
-      w1 = fmaf(e, zt, w1);
+      u1 = fmaf(e, zd[j + 1], u1);
+      w1 = fmaf(e, zt[j + 1], w1);
     }
   }
   st.s_t = fmaf(st.s_t, sct, s0 + s1);
   st.u = fmaf(st.u, sct, u0 + u1);
   st.w = fmaf(st.w, sct, w0 + w1);
-  st.m_t = nmt;
-  // drafter side: sum exp(z_d - m_d)
-  const float nmd = fmaxf(st.m_d, cmd);
-  const float scd = ex2((st.m_d - nmd) * kLog2e);
-  const float bd = -nmd * kLog2e;
+  // drafter side
+  const float nbd = fmaxf(st.best_d, cd);
+  const float scd = ex2((st.best_d - nbd) * kLog2e);
+  const float bd = -nbd * kLog2e;
   float r0 = 0.f, r1 = 0.f;
 #pragma unroll
-  for (int j = 0; j < 32; j += 2) {
-    if (kFull || j < nv) r0 += ex2(fmaf(f32(rd[j]), kLog2e, bd));
-    if (kFull || j + 1 < nv) r1 += ex2(fmaf(f32(rd[j + 1]), kLog2e, bd));
+  for (int j = 0; j < kSub; j += 2) {
+    r0 += ex2(fmaf(zd[j], kLog2e, bd));      // masked columns are -inf: exp gives 0
+    r1 += ex2(fmaf(zd[j + 1], kLog2e, bd));
   }
   st.s_d = fmaf(st.s_d, scd, r0 + r1);
-  st.m_d = nmd;
+  // greedy top-2 of both sides (moves best_d / best_t to nbd / nbt)
+  top2_update(st.best_d, st.sec_d, st.i_d, zd, cd, v0);
+  top2_update(st.best_t, st.sec_t, st.i_t, zt, ct, v0);
+  const int xr = x - v0;
+  if (xr >= 0 && xr < (kFull ? kSub : nv)) {
+#pragma unroll
+    for (int j = 0; j < kSub; ++j)
+      if (j == xr) st.zx = zt[j];
+  }
 }
 
 ALR_DEV uint32_t pack_bf16x2(float a, float b) {
@@ -188,19 +214,23 @@ ALR_DEV bool warp_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
 
 // kWMN: the head tile is read MN-major straight from W [d, V] (bf16), or K-major from a
 // transposed copy W^T [V, d] (fp32 inputs, whose tf32 products take K-major operands only).
+// kStaged: the backward stores bf16 G through shared staging and TMA (tm_g), else directly.
 template <typename Elem, bool kBwd, bool kWMN, int kBN>
-__global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
+__global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThreads, 1)
     loss_gemm_kernel(const __grid_constant__ CUtensorMap tm_hd,
                      const __grid_constant__ CUtensorMap tm_ht,
-                     const __grid_constant__ CUtensorMap tm_w, const LossArgs args) {
+                     const __grid_constant__ CUtensorMap tm_w,
+                     const __grid_constant__ CUtensorMap tm_g, const LossArgs args) {
   using G = Geo<Elem>;
-  using S = Shape<kBN>;
+  constexpr bool kStaged = kBwd && sizeof(Elem) == 2;
+  using S = Shape<kBN, kStaged>;
   constexpr int kStages = S::kStages;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_1024(smem_raw);
   uint8_t* stage_mem = smem;
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kStages * S::kStageBytes);
+  uint8_t* gstage = smem + kStages * S::kStageBytes;
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(gstage + S::kStaging);
   uint64_t* empty_bar = full_bar + kStages;
   uint64_t* tfull_bar = empty_bar + kStages;
   uint64_t* tempty_bar = tfull_bar + 2;
@@ -230,6 +260,7 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
     tma_prefetch_desc(&tm_hd);
     tma_prefetch_desc(&tm_ht);
     tma_prefetch_desc(&tm_w);
+    if (kStaged) tma_prefetch_desc(&tm_g);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
@@ -256,6 +287,16 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, ab)) {
               ok = false;
               break;
+            }
+            if (args.withhold_first_stage && u == int(blockIdx.x) && vt == split_begin(P, vs) &&
+                kb == 0) {
+              // test hook: leave this stage empty, so the MMA issuer's bounded wait on it runs
+              // out and the whole CTA takes the timeout path
+              if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1;
+              }
+              continue;
             }
             uint8_t* sb = stage_mem + stage * S::kStageBytes;
             mbar_arrive_expect_tx(&full_bar[stage], S::kStageBytes);
@@ -337,12 +378,14 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
       mma_commit(drain_bar);
       mbar_wait_drain(drain_bar, 0);
     }
-  } else if (warp >= kEpiWarp0) {
+  } else {
     // -------------------------------------------------------------------- epilogue ---
     const int q = warp & 3;
-    const int h = (warp - kEpiWarp0) >> 2;
+    const int cg = (warp - kEpiWarp0) >> 2;
     const int row_in_tile = q * 32 + lane;
-    const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(h * 128);
+    const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(cg * kColsPerWarp);
+    uint8_t* my_stage = gstage + (warp - kEpiWarp0) * 2 * kGStageBytes;
+    uint32_t n_stores = 0;
     int abuf = 0;
     uint32_t aphase = 0;
     bool ok = true;
@@ -363,21 +406,20 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
           }
           tc_fence_after();
           const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
-          const int vbase = vt * kBN + h * 128;
-          const bool full_tile = vbase + 128 <= P.V;
+          const int vbase = vt * kBN + cg * kColsPerWarp;
 #pragma unroll 1
-          for (int c = 0; c < 4; ++c) {
-            uint32_t rd[32], rt[32];
-            tmem_ld32(tb + c * 32, rd);
-            tmem_ld32(tb + kBN + c * 32, rt);
+          for (int c = 0; c < kColsPerWarp / kSub; ++c) {
+            uint32_t rd[16], rt[16];
+            tmem_ld16(tb + c * kSub, rd);
+            tmem_ld16(tb + kBN + c * kSub, rt);
             tmem_ld_wait();
             reg_fence(rd);
             reg_fence(rt);
-            const int v0 = vbase + c * 32;
-            if (full_tile) {
-              stats_chunk<true>(st, rd, rt, v0, 32, x);
+            const int v0 = vbase + c * kSub;
+            if (v0 + kSub <= P.V) {
+              stats_sub<true>(st, rd, rt, v0, kSub, x);
             } else if (v0 < P.V) {
-              stats_chunk<false>(st, rd, rt, v0, min(32, P.V - v0), x);
+              stats_sub<false>(st, rd, rt, v0, P.V - v0, x);
             }
           }
           tc_fence_before();
@@ -390,17 +432,17 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
         }
         if (ok && row_ok) {
           const size_t fs = size_t(P.n_parts) * P.N;
-          float* o = args.part + size_t(vs * S::kHalves + h) * P.N + row;
-          o[kPMd * fs] = st.m_d;
+          float* o = args.part + size_t(vs * S::kColGroups + cg) * P.N + row;
+          o[kPMd * fs] = st.best_d;
           o[kPSd * fs] = st.s_d;
-          o[kPMt * fs] = st.m_t;
+          o[kPMt * fs] = st.best_t;
           o[kPSt * fs] = st.s_t;
           o[kPU * fs] = st.u;
           o[kPW * fs] = st.w;
-          o[kPBd * fs] = st.b_d;
+          o[kPBd * fs] = st.best_d;
           o[kPId * fs] = __int_as_float(st.i_d);
           o[kPSecd * fs] = st.sec_d;
-          o[kPBt * fs] = st.b_t;
+          o[kPBt * fs] = st.best_t;
           o[kPIt * fs] = __int_as_float(st.i_t);
           o[kPSect * fs] = st.sec_t;
           o[kPZx * fs] = st.zx;
@@ -421,40 +463,51 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
           }
           tc_fence_after();
           const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
-          const int vbase = vt * kBN + h * 128;
+          const int vbase = vt * kBN + cg * kColsPerWarp;
 #pragma unroll 1
-          for (int c = 0; c < 4; ++c) {
-            uint32_t rd[32], rt[32];
-            tmem_ld32(tb + c * 32, rd);
-            tmem_ld32(tb + kBN + c * 32, rt);
+          for (int c = 0; c < kColsPerWarp / kSub; ++c) {
+            uint32_t rd[16], rt[16];
+            tmem_ld16(tb + c * kSub, rd);
+            tmem_ld16(tb + kBN + c * kSub, rt);
             tmem_ld_wait();
             reg_fence(rd);
             reg_fence(rt);
-            const int v0 = vbase + c * 32;
-            if (row_ok && v0 < P.V) {
-              float g[32];
+            const int v0 = vbase + c * kSub;
+            if (v0 >= P.V) continue;   // warp-uniform
+            float g[16];
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                g[j] = cw * (ex2(fmaf(f32(rd[j]), kLog2e, ad)) - ex2(fmaf(f32(rt[j]), kLog2e, at)));
-              if constexpr (sizeof(Elem) == 2) {
+            for (int j = 0; j < kSub; ++j)
+              g[j] = cw * (ex2(fmaf(f32(rd[j]), kLog2e, ad)) - ex2(fmaf(f32(rt[j]), kLog2e, at)));
+            if constexpr (kStaged) {
+              // this warp's 32 x 16 sub-chunk -> shared staging -> one TMA store; the buffer
+              // used two stores ago must have been read before it is overwritten
+              uint8_t* buf = my_stage + (n_stores & 1u) * kGStageBytes;
+              if (lane == 0) tma_store_wait_read_le1();
+              __syncwarp();
+              uint4 v0v, v1v;
+              v0v.x = pack_bf16x2(g[0], g[1]);
+              v0v.y = pack_bf16x2(g[2], g[3]);
+              v0v.z = pack_bf16x2(g[4], g[5]);
+              v0v.w = pack_bf16x2(g[6], g[7]);
+              v1v.x = pack_bf16x2(g[8], g[9]);
+              v1v.y = pack_bf16x2(g[10], g[11]);
+              v1v.z = pack_bf16x2(g[12], g[13]);
+              v1v.w = pack_bf16x2(g[14], g[15]);
+              *reinterpret_cast<uint4*>(buf + lane * 32) = v0v;
+              *reinterpret_cast<uint4*>(buf + lane * 32 + 16) = v1v;
+              fence_proxy_async_smem();
+              __syncwarp();
+              if (lane == 0) {
+                tma_store_2d(&tm_g, buf, v0, rb * kBM + q * 32);
+                tma_store_commit();
+              }
+              ++n_stores;
+            } else if (row_ok) {
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                  if (v0 + 8 * i < P.V) {   // V % 8 == 0: a vector is all in or all out
-                    uint4 v;
-                    v.x = pack_bf16x2(g[8 * i + 0], g[8 * i + 1]);
-                    v.y = pack_bf16x2(g[8 * i + 2], g[8 * i + 3]);
-                    v.z = pack_bf16x2(g[8 * i + 4], g[8 * i + 5]);
-                    v.w = pack_bf16x2(g[8 * i + 6], g[8 * i + 7]);
-                    *reinterpret_cast<uint4*>(grow + v0 + 8 * i) = v;
-                  }
-                }
-              } else {
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                  if (v0 + 4 * i < P.V)
-                    *reinterpret_cast<float4*>(grow + v0 + 4 * i) =
-                        make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
-                }
+              for (int i = 0; i < kSub / 4; ++i) {
+                if (v0 + 4 * i < P.V)
+                  *reinterpret_cast<float4*>(grow + v0 + 4 * i) =
+                      make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
               }
             }
           }
@@ -468,6 +521,9 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
         }
       }
     }
+    if constexpr (kStaged) {
+      if (lane == 0) tma_store_wait_all();   // staging must stay valid until read
+    }
   }
 
   tc_fence_before();
@@ -480,37 +536,39 @@ __global__ void __launch_bounds__(Shape<kBN>::kThreads, 1)
 
 template <typename Elem, bool kBwd, int kBN>
 cudaError_t launch_impl(const CUtensorMap& hd, const CUtensorMap& ht, const CUtensorMap& w,
-                        const LossArgs& args, cudaStream_t s) {
-  using S = Shape<kBN>;
+                        const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
+  using S = Shape<kBN, kBwd && sizeof(Elem) == 2>;
   auto kern = loss_gemm_kernel<Elem, kBwd, sizeof(Elem) == 2, kBN>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
   if (e != cudaSuccess) return e;
-  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(hd, ht, w, args);
+  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(hd, ht, w, g, args);
   return cudaGetLastError();
 }
 
 template <bool kBwd>
 cudaError_t dispatch(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                     const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
+                     const CUtensorMap& w, const CUtensorMap& g, const LossArgs& args,
+                     cudaStream_t s) {
   if (args.plan.bn == 128) {
-    if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 128>(hd, ht, w, args, s);
-    return launch_impl<float, kBwd, 128>(hd, ht, w, args, s);
+    if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 128>(hd, ht, w, g, args, s);
+    return launch_impl<float, kBwd, 128>(hd, ht, w, g, args, s);
   }
-  if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 256>(hd, ht, w, args, s);
-  return launch_impl<float, kBwd, 256>(hd, ht, w, args, s);
+  if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 256>(hd, ht, w, g, args, s);
+  return launch_impl<float, kBwd, 256>(hd, ht, w, g, args, s);
 }
 
 }  // namespace
 
 cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
                             const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
-  return dispatch<false>(dtype, hd, ht, w, args, s);
+  return dispatch<false>(dtype, hd, ht, w, w, args, s);
 }
 
 cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
-  return dispatch<true>(dtype, hd, ht, w, args, s);
+                            const CUtensorMap& w, const CUtensorMap& g_store,
+                            const LossArgs& args, cudaStream_t s) {
+  return dispatch<true>(dtype, hd, ht, w, g_store, args, s);
 }
 
 }  // namespace alr

@@ -58,14 +58,19 @@ ALR_DEV void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
                : "memory");
 }
 
+// One bounded probe of the phase with the given parity.  A thread whose phase is not yet
+// complete is suspended in hardware until the phase completes or kSuspendHintNs elapses, so
+// waiting warps do not spin through issue slots (and power) while the tensor cores work.
+constexpr uint32_t kSuspendHintNs = 20000;
+
 ALR_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t done;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
       : "memory");
   return done != 0;
 }
@@ -82,15 +87,13 @@ struct AbortFlag {
 ALR_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
-  for (uint32_t it = 1;; ++it) {
+  for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 0) {
-      if (*ab.smem) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
-        *ab.smem = 1;
-        atomicExch(ab.status, kStatusTimeout);
-        return false;
-      }
+    if (*ab.smem) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      *ab.smem = 1;
+      atomicExch(ab.status, kStatusTimeout);
+      return false;
     }
   }
 }
@@ -128,6 +131,10 @@ ALR_DEV void tma_store_wait_read_all() {
   asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 ALR_DEV void tma_store_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Wait until at most the most recent bulk store group is still reading shared memory.
+ALR_DEV void tma_store_wait_read_le1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
 
 // Make generic-proxy shared-memory writes visible to the async proxy (TMA store reads).
 ALR_DEV void fence_proxy_async_smem() {

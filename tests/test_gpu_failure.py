@@ -1,0 +1,45 @@
+"""Failure detection without a GPU fault: a pipeline wait that nothing will satisfy runs out
+after its bounded time, the kernel records ALR_ERR_TIMEOUT, the host reads it through
+alr_device_status(), and the same context keeps computing correct results."""
+
+import time
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import alr_oracle as orc
+from paper_2609_38795_gb300 import alr, build_lib, synthetic
+from tests import parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    build_lib.build()
+    alr.lib()
+    assert alr.alr_device_supported() == alr.ALR_OK, alr.alr_last_error()
+
+
+def test_withheld_stage_times_out_and_context_survives():
+    A, B, d, V = 16, 16, 256, 1024
+    b = synthetic.slot_batch(d, V, A, B, 0.5, dtype=torch.bfloat16, device="cuda", seed=9)
+    sl = alr.SlotLoss(A * B, d, V, B)
+    assert alr.alr_device_status(clear=True) == alr.ALR_OK
+    alr.alr_debug_withhold_next_stage(True)
+    t0 = time.monotonic()
+    sl.forward(b["Hd"], b["Ht"], b["W"])          # enqueues; the kernel gives up on its own
+    rc = alr.alr_device_status(clear=True)
+    waited = time.monotonic() - t0
+    assert rc == alr.ALR_ERR_TIMEOUT, alr.alr_last_error()
+    assert "timed out" in alr.alr_last_error()
+    assert waited < 20.0
+    # the hook disarmed itself; the next call is normal and correct
+    sl.forward(b["Hd"], b["Ht"], b["W"])
+    torch.cuda.synchronize()
+    assert alr.alr_device_status() == alr.ALR_OK
+    r = orc.slot_loss_forward(P.np64(b["Hd"]), P.np64(b["Ht"]), P.np64(b["W"]), B)
+    P.compare_forward(P.fwd_to_numpy(sl), r)
