@@ -267,3 +267,71 @@ def gather_ira_blocks(F, seq, pos, B, valid_len=None):
 def ira_supervised_slots(K: int, j: int) -> int:
     """Number of supervised slots of a secondary block at offset j (Eq. 4): #{k : j+k <= K}."""
     return sum(1 for k in range(1, K + 1) if j + k <= K)
+
+
+# ----------------------------------------------------------------------------------------
+# Compact labels: top-k target probabilities plus a tail bin (Sec. 3.1 under Eq. 1; App. A,
+# KD loss and rollout label readout)
+# ----------------------------------------------------------------------------------------
+def label_readout(Ht, W, k=8, corpus_tok=None):
+    """The label a rollout step keeps: the k most probable target tokens (probability
+    descending, equal probabilities to the lower token id, App. A), their probabilities, the
+    remaining mass (the tail bin) and the greedy token y* (the first of them).
+
+    Returns idx [N, k] int64, prob [N, k], tail [N] (sum of p over the other tokens), lse_t,
+    argmax_t, gap_t, and logp_x (log p of corpus_tok, for the erase gate) when given.
+    """
+    z_t = head_logits(Ht, W)
+    N, V = z_t.shape
+    lse_t = log_sum_exp(z_t)
+    p = np.exp(z_t - lse_t[:, None])
+    order = np.argsort(-z_t, axis=1, kind="stable")   # stable: equal logits keep id order
+    idx = order[:, :k]
+    rows = np.arange(N)[:, None]
+    prob = p[rows, idx]
+    outside = np.ones_like(p, dtype=bool)
+    outside[rows, idx] = False
+    tail = np.where(outside, p, 0.0).sum(axis=1)
+    am_t, gap_t = greedy(z_t)
+    logp_x = None
+    if corpus_tok is not None:
+        x = np.asarray(corpus_tok, dtype=np.int64)
+        logp_x = z_t[np.arange(N), x] - lse_t
+    return dict(z_t=z_t, idx=idx.astype(np.int64), prob=prob, tail=tail, lse_t=lse_t,
+                argmax_t=am_t, gap_t=gap_t, logp_x=logp_x)
+
+
+def top_k_soft_cross_entropy(z_d, idx, prob, tail):
+    """l_r = -sum_i prob_i log q[idx_i] - tail * log(tail_q), the soft CE between the
+    (k+1)-bin label (prob, tail) and the drafter's (q[idx], tail_q), with tail_q the drafter
+    mass outside the label's k tokens.  A zero tail contributes nothing."""
+    z_d = _f64(z_d)
+    N, V = z_d.shape
+    rows = np.arange(N)[:, None]
+    log_q = z_d - log_sum_exp(z_d)[:, None]
+    outside = np.ones((N, V), dtype=bool)
+    outside[rows, idx] = False
+    tail_q = np.where(outside, np.exp(log_q), 0.0).sum(axis=1)
+    tail = _f64(tail)
+    tail_term = np.where(tail > 0, tail * np.log(np.where(tail > 0, tail_q, 1.0)), 0.0)
+    return -(_f64(prob) * log_q[rows, idx]).sum(axis=1) - tail_term, tail_q
+
+
+def top_k_logit_grad(z_d, idx, prob, tail, weight, lam, weight_sum=None):
+    """Gradient of Eq. 1 with the top-k + tail loss with respect to the drafter logits:
+    c_r * (q_v - prob at v) for a label token v, c_r * q_v * (1 - tail / tail_q) otherwise,
+    with c_r = lam * omega_r / sum omega (zero when sum omega = 0)."""
+    z_d = _f64(z_d)
+    N, V = z_d.shape
+    weight = _f64(weight)
+    wsum = weight.sum() if weight_sum is None else float(weight_sum)
+    if wsum == 0.0:
+        return np.zeros_like(z_d)
+    rows = np.arange(N)[:, None]
+    q = softmax(z_d)
+    _, tail_q = top_k_soft_cross_entropy(z_d, idx, prob, tail)
+    tail = _f64(tail)
+    beta = 1.0 - np.where(tail > 0, tail / np.where(tail > 0, tail_q, 1.0), 0.0)
+    G = q * beta[:, None]
+    G[rows, idx] = q[rows, idx] - _f64(prob)
+    return (lam * weight / wsum)[:, None] * G
