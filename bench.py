@@ -46,6 +46,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-anchors", type=int, default=1)
+    ap.add_argument("--no-topk", action="store_true",
+                    help="skip the compact-label (top-8 + tail) step measurement")
     ap.add_argument("--anchors", type=int, default=0,
                     help="profiling only: fewer anchors than the workload (config says so)")
     return ap.parse_args()
@@ -289,6 +291,82 @@ class Step:
         rec(6)
 
 
+class TopkStep:
+    """The compact-label step (the paper's own loss form): label readout of H_t (top-8 target
+    probabilities, tail, greedy token) -> top-8 + tail soft CE forward on H_d -> accepted
+    length -> logit gradient -> dH = G W^T -> dW += H_d^T G."""
+    PHASES = ["readout", "fwd", "accept_len", "logit_grad", "dH_gemm", "dW_gemm"]
+    KERNELS_PER_STEP = 8   # readout (+ merge), fwd (+ merge, finalize), accept, grad, dH, dW
+
+    def __init__(self, step):
+        import torch
+        from paper_2609_38795_gb300 import alr
+        self.s, self.alr = step, alr
+        wl, dev = step.wl, step.G.device
+        N = wl.N
+        self.params = alr.make_params(N, wl.d, wl.V, wl.B, torch.bfloat16)
+        f = lambda *sh: torch.empty(*sh, dtype=torch.float32, device=dev)  # noqa: E731
+        i = lambda *sh: torch.empty(*sh, dtype=torch.int32, device=dev)  # noqa: E731
+        self.lab = dict(top_idx=i(N, alr.ALR_TOPK), top_prob=f(N, alr.ALR_TOPK), tail=f(N),
+                        lse_t=f(N), argmax_t=i(N), gap_t=f(N))
+        self.out = dict(loss_row=f(N), lse_d=f(N), tail_q=f(N), argmax_d=i(N), gap_d=f(N),
+                        weight=f(N), loss_total=f(1), weight_sum=f(1))
+        self.ws_r = torch.empty(alr.alr_readout_workspace_size(self.params), dtype=torch.uint8,
+                                device=dev)
+        self.ws_f = torch.empty(alr.alr_topk_fwd_workspace_size(self.params), dtype=torch.uint8,
+                                device=dev)
+
+    def run(self, events=None):
+        alr, s, x, lab, o = self.alr, self.s, self.s.x, self.lab, self.out
+        wl = s.wl
+        rec = (lambda i: events[i].record()) if events is not None else (lambda i: None)
+        rec(0)
+        alr.alr_label_readout(self.params, x["Ht"], x["W"], lab, self.ws_r)
+        rec(1)
+        alr.alr_topk_loss_fwd(self.params, x["Hd"], x["W"], lab["top_idx"], lab["top_prob"],
+                              lab["tail"], o, self.ws_f, row_mask=x["row_valid"])
+        rec(2)
+        alr.alr_accept_len(o["argmax_d"], lab["argmax_t"], wl.B, s.sl.acc_len, s.sl.hist,
+                           active=x["row_valid"])
+        rec(3)
+        alr.alr_topk_logit_grad(self.params, x["Hd"], x["W"], lab["top_idx"], lab["top_prob"],
+                                lab["tail"], o["weight"], o["weight_sum"], o["lse_d"],
+                                o["tail_q"], s.G)
+        rec(4)
+        alr.alr_gemm(s.G, x["W"], s.dH, wl.N, wl.d, wl.V)
+        rec(5)
+        alr.alr_gemm(x["Hd"], s.G, s.dW, wl.d, wl.V, wl.N, a_mn=True, b_mn=True, accumulate=True)
+        rec(6)
+
+
+def time_topk(step, K, warmup):
+    import torch
+    ts = TopkStep(step)
+    for _ in range(warmup):
+        ts.run()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(K)]
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for k in range(K):
+        ts.run(ev[k])
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / K
+    wl = step.wl
+    NdV = wl.N * wl.d * wl.V
+    phase = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
+             for i, p in enumerate(TopkStep.PHASES)}
+    loss_ms = ms - phase["readout"]
+    return {"what": "compact labels (top-8 + tail bin): readout of H_t, then the loss fwd+bwd",
+            "ms_per_step": ms, "rows_per_s": wl.N / (ms / 1e3),
+            "loss_fwd_bwd_rows_per_s": wl.N / (loss_ms / 1e3),
+            "loss_executed_tflops_8NdV": 8 * NdV / (loss_ms / 1e3) / 1e12,
+            "readout_tflops_2NdV": 2 * NdV / (phase["readout"] / 1e3) / 1e12,
+            "phase_ms": phase, "gpu_launches": TopkStep.KERNELS_PER_STEP * K,
+            "loss": ts.out["loss_total"].item()}
+
+
 def run_gpu(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -375,6 +453,7 @@ def run_gpu(args, rank, world, local_rank):
     total_ms, e2e_ms = max_over_ranks([total_ms, e2e["ms"] if e2e else 0.0], device)
 
     gather = gather_bandwidth(device) if rank == 0 else None
+    topk = time_topk(step, K, args.warmup) if (rank == 0 and not args.no_topk) else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -417,6 +496,7 @@ def run_gpu(args, rank, world, local_rank):
                      "flops_per_launch": flops[dom]},
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
+        "compact_labels": topk,
         "loss": loss, "acc_hist": acc_hist,
         "clocks": clk,
         "cpu_baseline": cpu,

@@ -201,6 +201,89 @@ int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const vo
                    const float* weight, const float* weight_sum, const float* lse_d,
                    const float* lse_t, void* G, void* workspace, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------------------
+ * Compact labels: the target's top-k probabilities plus a tail bin.
+ *
+ * The paper's loss l evaluates soft cross-entropy against the target distribution restricted
+ * to its 8 most probable tokens, with the remaining mass in one tail bin (Sec. 3.1 under
+ * Eq. 1; App. A, KD loss), and each rollout step keeps exactly that label (App. A, rollout
+ * implementation: top 8 tokens and the remaining mass, greedy ties to the lower id).  These
+ * entry points compute that label from the target hidden states (the readout) and the loss
+ * against it, whose forward and backward need only the drafter's head product.
+ * ------------------------------------------------------------------------------------- */
+#define ALR_TOPK 8
+
+/* Workspace bytes alr_label_readout needs for `p` (0 on invalid params). */
+size_t alr_readout_workspace_size(const alr_params* p);
+
+/*
+ * Label readout: for each row, z_t = h_t W over the whole vocabulary (never stored), then
+ *   top_idx  [N, ALR_TOPK] int32: the most probable tokens, probability descending, equal
+ *            probabilities to the lower token id (top_idx[r*8] is the greedy token y*);
+ *   top_prob [N, ALR_TOPK]: their probabilities p_T(v);   tail [N]: 1 - sum of top_prob,
+ *            computed as the mass of the other tokens;
+ *   lse_t, argmax_t, gap_t [N] (nullable): log-sum-exp, greedy token, top-1 minus top-2;
+ *   logp_x [N] (nullable, needs corpus_tok): log p_T(corpus_tok), the erase gate's factor.
+ * Uses p->N, d, V (>= ALR_TOPK), dtype; mode, lambda, gamma and B are ignored (B must still
+ * divide N).
+ */
+int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
+                      const int32_t* corpus_tok, int32_t* top_idx, float* top_prob, float* tail,
+                      float* lse_t, int32_t* argmax_t, float* gap_t, float* logp_x,
+                      void* workspace, size_t ws_bytes, void* stream);
+
+/* Outputs of alr_topk_loss_fwd, device pointers, length N unless stated. */
+typedef struct {
+    float* loss_row;     /* l_r (required)                                                     */
+    float* lse_d;        /* log-sum-exp of z_d (required: the backward reads it)               */
+    float* tail_q;       /* drafter mass outside the row's label tokens (required: backward)   */
+    int32_t* argmax_d;   /* greedy drafter token, lowest id on ties (required)                 */
+    float* gap_d;        /* top-1 minus top-2 drafter logit (nullable)                         */
+    float* weight;       /* omega_r used (required)                                            */
+    float* loss_total;   /* [1] L of Eq. 1 times lambda                                        */
+    float* weight_sum;   /* [1] sum omega                                                      */
+} alr_topk_fwd_outputs;
+
+/* Workspace bytes alr_topk_loss_fwd needs for `p` (0 on invalid params). */
+size_t alr_topk_fwd_workspace_size(const alr_params* p);
+
+/*
+ * Forward pass of Eq. 1 with the top-k + tail soft cross-entropy:
+ *   l_r = -sum_i top_prob_i log q(top_idx_i) - tail_r log tail_q_r,
+ *   tail_q_r = 1 - sum_i q(top_idx_i) (the drafter's mass outside the label tokens; a zero
+ *   tail contributes nothing), q = softmax(h_d W) over the whole vocabulary.
+ * omega_r = weight_in[r] when weight_in is given (e.g. erase weights from alr_erase_weights),
+ * else w_k * row_mask[r] (row_mask nullable = ones).  Label tokens must lie in [0, V).
+ * tail_q is computed as (S - sum_i e^{z_i - m}) / S from the fp32 running sum S; when the
+ * drafter puts almost all its mass on the label tokens (tail_q below ~1e-5) its relative
+ * error grows accordingly.
+ */
+int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
+                      const float* top_prob, const float* tail, const float* row_mask,
+                      const float* weight_in, const alr_topk_fwd_outputs* out, void* workspace,
+                      size_t ws_bytes, void* stream);
+
+/*
+ * Gradient of that loss with respect to the drafter logits, recomputed tile by tile:
+ *   G[r, v] = c_r (q_v - top_prob_i)            for v = top_idx_i,
+ *   G[r, v] = c_r q_v (1 - tail_r / tail_q_r)   for the other tokens,
+ * c_r = lambda omega_r / sum omega.  Workspace: alr_logit_grad_workspace_size.
+ */
+int alr_topk_logit_grad(const alr_params* p, const void* Hd, const void* W,
+                        const int32_t* top_idx, const float* top_prob, const float* tail,
+                        const float* weight, const float* weight_sum, const float* lse_d,
+                        const float* tail_q, void* G, void* workspace, size_t ws_bytes,
+                        void* stream);
+
+/*
+ * Backward pass of the top-k loss: G as above, dHd = G W^T (overwritten) and, when dW is
+ * given, dW += H_d^T G.  Workspace: alr_bwd_workspace_size.
+ */
+int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
+                      const float* top_prob, const float* tail, const float* weight,
+                      const float* weight_sum, const float* lse_d, const float* tail_q,
+                      float* dHd, float* dW, void* workspace, size_t ws_bytes, void* stream);
+
 /*
  * Greedy accepted length per anchor (Sec. 3.2: slot k counts only when slots 1..k-1 were
  * accepted; MAT tau = acc + 1, Sec. 4).

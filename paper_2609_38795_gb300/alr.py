@@ -39,6 +39,15 @@ class AlrFwdOutputs(ctypes.Structure):
     _fields_ = [(f, _c_p) for f in _FWD_FIELDS]
 
 
+_TOPK_FIELDS = ("loss_row", "lse_d", "tail_q", "argmax_d", "gap_d", "weight", "loss_total",
+                "weight_sum")
+ALR_TOPK = 8
+
+
+class AlrTopkFwdOutputs(ctypes.Structure):
+    _fields_ = [(f, _c_p) for f in _TOPK_FIELDS]
+
+
 # name -> (restype, argtypes); must match include/alr.h
 SIGNATURES = {
     "alr_version": (ctypes.c_char_p, []),
@@ -59,6 +68,16 @@ SIGNATURES = {
     "alr_logit_grad_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_logit_grad": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_readout_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
+    "alr_label_readout": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                   _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_topk_fwd_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
+    "alr_topk_loss_fwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                   _c_p, ctypes.POINTER(AlrTopkFwdOutputs), _c_p, _c_sz, _c_p]),
+    "alr_topk_logit_grad": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p,
+                                     _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_topk_loss_bwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                   _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
     "alr_erase_weights": (_c_int, [_c_p, _c_p, _c_p, _c_p, _c_i32, _c_i32, _c_f, _c_i32, _c_p,
                                    _c_p]),
@@ -190,6 +209,53 @@ def alr_logit_grad(params, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, works
     _check(lib().alr_logit_grad(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W), _ptr(weight),
                                 _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t), _ptr(G),
                                 _ptr(workspace), nbytes, _stream(stream)))
+
+
+def _nbytes(ws):
+    return 0 if ws is None else ws.numel() * ws.element_size()
+
+
+def alr_readout_workspace_size(params) -> int:
+    return lib().alr_readout_workspace_size(ctypes.byref(params))
+
+
+def alr_label_readout(params, Ht, W, out: dict, workspace, corpus_tok=None, stream=None):
+    """out: top_idx [N, 8] int32, top_prob [N, 8], tail [N]; optional lse_t, argmax_t, gap_t,
+    logp_x."""
+    _check(lib().alr_label_readout(ctypes.byref(params), _ptr(Ht), _ptr(W), _ptr(corpus_tok),
+                                   _ptr(out["top_idx"]), _ptr(out["top_prob"]), _ptr(out["tail"]),
+                                   _ptr(out.get("lse_t")), _ptr(out.get("argmax_t")),
+                                   _ptr(out.get("gap_t")), _ptr(out.get("logp_x")),
+                                   _ptr(workspace), _nbytes(workspace), _stream(stream)))
+
+
+def alr_topk_fwd_workspace_size(params) -> int:
+    return lib().alr_topk_fwd_workspace_size(ctypes.byref(params))
+
+
+def alr_topk_loss_fwd(params, Hd, W, top_idx, top_prob, tail, out: dict, workspace,
+                      row_mask=None, weight_in=None, stream=None):
+    o = AlrTopkFwdOutputs(**{f: _ptr(out.get(f)) for f in _TOPK_FIELDS})
+    _check(lib().alr_topk_loss_fwd(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(top_idx),
+                                   _ptr(top_prob), _ptr(tail), _ptr(row_mask), _ptr(weight_in),
+                                   ctypes.byref(o), _ptr(workspace), _nbytes(workspace),
+                                   _stream(stream)))
+
+
+def alr_topk_logit_grad(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum, lse_d,
+                        tail_q, G, workspace=None, stream=None):
+    _check(lib().alr_topk_logit_grad(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(top_idx),
+                                     _ptr(top_prob), _ptr(tail), _ptr(weight), _ptr(weight_sum),
+                                     _ptr(lse_d), _ptr(tail_q), _ptr(G), _ptr(workspace),
+                                     _nbytes(workspace), _stream(stream)))
+
+
+def alr_topk_loss_bwd(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum, lse_d, tail_q,
+                      dHd, dW, workspace, stream=None):
+    _check(lib().alr_topk_loss_bwd(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(top_idx),
+                                   _ptr(top_prob), _ptr(tail), _ptr(weight), _ptr(weight_sum),
+                                   _ptr(lse_d), _ptr(tail_q), _ptr(dHd), _ptr(dW),
+                                   _ptr(workspace), _nbytes(workspace), _stream(stream)))
 
 
 def alr_accept_len(argmax_d, argmax_t, B, acc_len, hist=None, active=None, stream=None):

@@ -159,15 +159,17 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
 
 // fp32 inputs run tf32 products, which take K-major operands only: the head is then read from
 // a transposed copy W^T [V, d] placed in the workspace.
+// Forward-type workspace: `fields` partial statistics per row and part, one fp64 pair per
+// anchor, and W^T for fp32 inputs.
 struct FwdLayout {
   size_t part_off, anchor_off, wt_off, total;
 };
 
-FwdLayout fwd_layout(const alr_params* p, int sms) {
+FwdLayout fwd_layout(const alr_params* p, int sms, int fields = alr::kPFields) {
   const alr::LossPlan P = loss_plan(p, sms, false);
   FwdLayout L{};
   L.part_off = 0;
-  L.anchor_off = round_up(size_t(alr::kPFields) * P.n_parts * size_t(P.N) * sizeof(float), 1024);
+  L.anchor_off = round_up(size_t(fields) * P.n_parts * size_t(P.N) * sizeof(float), 1024);
   L.wt_off = L.anchor_off + round_up(2 * sizeof(double) * size_t(P.N / P.B), 1024);
   L.total = L.wt_off;
   if (p->dtype == ALR_F32) L.total += round_up(size_t(p->V) * p->d * sizeof(float), 1024);
@@ -332,7 +334,7 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
   args.withhold_first_stage = g_withhold_next.exchange(0);
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  e = alr::launch_loss_fwd(dt, m_hd, m_ht, m_w, args, s);
+  e = alr::launch_loss_kernel(alr::kModeFwd, dt, m_hd, m_ht, m_w, m_w, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "forward loss kernel launch");
   double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
   e = alr::launch_combine(args.plan, args.part, p->mode, p->gamma, row_mask, args.corpus_tok,
@@ -368,17 +370,29 @@ int check_bwd_args(const alr_params* p, const void* Hd, const void* Ht, const vo
   return require_sm103(info);
 }
 
-// G = lambda omega / sum omega (q - p), recomputing the logit tiles (the fused backward kernel).
+// Compact-label inputs of the top-k path (all NULL for the full-vocabulary loss).
+struct TopkLabels {
+  const int32_t* idx = nullptr;
+  const float* prob = nullptr;
+  const float* tail = nullptr;
+  const float* tail_q = nullptr;
+};
+
+// The fused logit-gradient kernel: G = lambda omega / sum omega (q - p) for the full
+// vocabulary (Ht given), or the top-k + tail form (labels given), recomputing the tiles.
 int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
                     const float* weight, const float* weight_sum, const float* lse_d,
-                    const float* lse_t, void* G, void* wt, const DevInfo& info, cudaStream_t s) {
+                    const float* lse_t, const TopkLabels& lab, void* G, void* wt,
+                    const DevInfo& info, cudaStream_t s) {
   const int dt = p->dtype;
   const size_t es = elem_size(dt);
   const uint32_t kke = k_per_row(dt);
+  const bool topk = lab.idx != nullptr;
   int rc;
   CUtensorMap m_hd, m_ht, m_w, m_gs;
   if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  m_ht = m_hd;
+  if (!topk && (rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
   if ((rc = head_map(&m_w, p, W, wt, s)) != ALR_OK) return rc;
   m_gs = m_w;
   if (dt == ALR_BF16 &&
@@ -392,10 +406,78 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
   args.weight = weight;
   args.weight_sum = weight_sum;
   args.lam = p->lambda;
+  args.top_idx = lab.idx;
+  args.top_prob = lab.prob;
+  args.tail = lab.tail;
+  args.tail_q = lab.tail_q;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_loss_bwd(dt, m_hd, m_ht, m_w, m_gs, args, s);
+  cudaError_t e = alr::launch_loss_kernel(topk ? alr::kModeTopkBwd : alr::kModeBwd, dt, m_hd, m_ht,
+                                          m_w, m_gs, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "logit-gradient kernel launch");
+  return ALR_OK;
+}
+
+// dH_d = G W^T and, when dW is given, dW += H_d^T G (fp32 via transposed workspace copies).
+int head_grads_impl(const alr_params* p, const void* Hd, const void* W, const void* G, float* dHd,
+                    float* dW, uint8_t* ws, const BwdLayout& lay, const DevInfo& info,
+                    cudaStream_t s) {
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  const uint32_t kke = k_per_row(dt);
+  int* status = alr::device_status_ptr();
+  int rc;
+  cudaError_t e;
+  // dH_d = G W^T: A = G [N, V] K-major, B = W [d, V] K-major.
+  CUtensorMap m_ga, m_wk;
+  if ((rc = make_map(&m_ga, G, dt, p->V, p->N, p->V * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_wk, W, dt, p->V, p->d, p->V * es, kke, 256)) != ALR_OK) return rc;
+  alr::GemmArgs gh = gemm_plan(int(p->N), p->d, p->V, dHd, p->d, info.sms);
+  gh.status = status;
+  e = alr::launch_plain_gemm(dt, false, false, false, m_ga, m_wk, gh, s);
+  if (e != cudaSuccess) return cuda_fail(e, "dH GEMM launch");
+  if (dW == nullptr) return ALR_OK;
+  alr::GemmArgs gw = gemm_plan(p->d, p->V, int(p->N), dW, p->V, info.sms);
+  gw.status = status;
+  CUtensorMap m_ha, m_gb;
+  if (dt == ALR_BF16) {
+    // dW += H_d^T G: A = H_d read as [K = N, M = d] (MN-major), B = G [K = N, V] (MN-major).
+    if ((rc = make_map(&m_ha, Hd, dt, p->d, p->N, p->d * es, kke, kke)) != ALR_OK) return rc;
+    if ((rc = make_map(&m_gb, G, dt, p->V, p->N, p->V * es, kke, kke)) != ALR_OK) return rc;
+    e = alr::launch_plain_gemm(dt, true, true, true, m_ha, m_gb, gw, s);
+  } else {
+    // K-major operands from transposed copies H_d^T [d, N'] and G^T [V, N'].
+    float* hdt = reinterpret_cast<float*>(ws + lay.hdt_off);
+    float* gt = reinterpret_cast<float*>(ws + lay.gt_off);
+    if ((e = alr::launch_transpose32(static_cast<const float*>(Hd), hdt, int(p->N), p->d,
+                                     int(lay.ld_n), s)) != cudaSuccess)
+      return cuda_fail(e, "H_d transpose launch");
+    if ((e = alr::launch_transpose32(static_cast<const float*>(G), gt, int(p->N), p->V,
+                                     int(lay.ld_n), s)) != cudaSuccess)
+      return cuda_fail(e, "G transpose launch");
+    if ((rc = make_map(&m_ha, hdt, dt, p->N, p->d, lay.ld_n * 4, kke, 128)) != ALR_OK) return rc;
+    if ((rc = make_map(&m_gb, gt, dt, p->N, p->V, lay.ld_n * 4, kke, 256)) != ALR_OK) return rc;
+    e = alr::launch_plain_gemm(dt, false, false, true, m_ha, m_gb, gw, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "dW GEMM launch");
+  return ALR_OK;
+}
+
+int check_workspace(void* workspace, size_t ws_bytes, size_t need) {
+  if (need > 0 && (workspace == nullptr || ws_bytes < need))
+    return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
+                ws_bytes, need);
+  if (need > 0 && !aligned16(workspace))
+    return fail(ALR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+  return ALR_OK;
+}
+
+int check_topk_labels(const alr_params* p, const int32_t* idx, const float* prob,
+                      const float* tail) {
+  if (p->V < alr::kTopK)
+    return fail(ALR_ERR_INVALID_ARG, "V = %d is below the %d label tokens", p->V, alr::kTopK);
+  if (idx == nullptr || prob == nullptr || tail == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "top_idx, top_prob and tail must be non-NULL");
   return ALR_OK;
 }
 
@@ -419,8 +501,8 @@ int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const vo
   if (need > 0 && (workspace == nullptr || ws_bytes < need || !aligned16(workspace)))
     return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
                 ws_bytes, need);
-  return logit_grad_impl(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, workspace, info,
-                         static_cast<cudaStream_t>(stream));
+  return logit_grad_impl(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, TopkLabels{}, G,
+                         workspace, info, static_cast<cudaStream_t>(stream));
 }
 
 int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
@@ -439,53 +521,155 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
                 ws_bytes, need);
   if (!aligned16(workspace)) return fail(ALR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
 
-  const int dt = p->dtype;
-  const size_t es = elem_size(dt);
-  const uint32_t kke = k_per_row(dt);
   const BwdLayout lay = bwd_layout(p);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   void* G = ws + lay.g_off;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e;
-  rc = logit_grad_impl(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, ws + lay.wt_off, info, s);
+  rc = logit_grad_impl(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, TopkLabels{}, G,
+                       ws + lay.wt_off, info, s);
   if (rc != ALR_OK) return rc;
-  int* status = alr::device_status_ptr();
+  return head_grads_impl(p, Hd, W, G, dHd, dW, ws, lay, info, s);
+}
 
-  // dH_d = G W^T: A = G [N, V] K-major, B = W [d, V] K-major.
-  CUtensorMap m_ga, m_wk;
-  if ((rc = make_map(&m_ga, G, dt, p->V, p->N, p->V * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_wk, W, dt, p->V, p->d, p->V * es, kke, 256)) != ALR_OK) return rc;
-  alr::GemmArgs gh = gemm_plan(int(p->N), p->d, p->V, dHd, p->d, info.sms);
-  gh.status = status;
-  e = alr::launch_plain_gemm(dt, false, false, false, m_ga, m_wk, gh, s);
-  if (e != cudaSuccess) return cuda_fail(e, "dH GEMM launch");
+size_t alr_readout_workspace_size(const alr_params* p) {
+  if (check_params(p) != ALR_OK) return 0;
+  DevInfo info;
+  if (device_info(&info) != ALR_OK) return 0;
+  return fwd_layout(p, info.sms, alr::kRFields).total;
+}
 
-  if (dW != nullptr) {
-    alr::GemmArgs gw = gemm_plan(p->d, p->V, int(p->N), dW, p->V, info.sms);
-    gw.status = status;
-    CUtensorMap m_ha, m_gb;
-    if (dt == ALR_BF16) {
-      // dW += H_d^T G: A = H_d read as [K = N, M = d] (MN-major), B = G [K = N, V] (MN-major).
-      if ((rc = make_map(&m_ha, Hd, dt, p->d, p->N, p->d * es, kke, kke)) != ALR_OK) return rc;
-      if ((rc = make_map(&m_gb, G, dt, p->V, p->N, p->V * es, kke, kke)) != ALR_OK) return rc;
-      e = alr::launch_plain_gemm(dt, true, true, true, m_ha, m_gb, gw, s);
-    } else {
-      // K-major operands from transposed copies H_d^T [d, N'] and G^T [V, N'].
-      float* hdt = reinterpret_cast<float*>(ws + lay.hdt_off);
-      float* gt = reinterpret_cast<float*>(ws + lay.gt_off);
-      if ((e = alr::launch_transpose32(static_cast<const float*>(Hd), hdt, int(p->N), p->d,
-                                       int(lay.ld_n), s)) != cudaSuccess)
-        return cuda_fail(e, "H_d transpose launch");
-      if ((e = alr::launch_transpose32(static_cast<const float*>(G), gt, int(p->N), p->V,
-                                       int(lay.ld_n), s)) != cudaSuccess)
-        return cuda_fail(e, "G transpose launch");
-      if ((rc = make_map(&m_ha, hdt, dt, p->N, p->d, lay.ld_n * 4, kke, 128)) != ALR_OK) return rc;
-      if ((rc = make_map(&m_gb, gt, dt, p->N, p->V, lay.ld_n * 4, kke, 256)) != ALR_OK) return rc;
-      e = alr::launch_plain_gemm(dt, false, false, true, m_ha, m_gb, gw, s);
-    }
-    if (e != cudaSuccess) return cuda_fail(e, "dW GEMM launch");
-  }
+int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
+                      const int32_t* corpus_tok, int32_t* top_idx, float* top_prob, float* tail,
+                      float* lse_t, int32_t* argmax_t, float* gap_t, float* logp_x,
+                      void* workspace, size_t ws_bytes, void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Ht == nullptr || W == nullptr || top_idx == nullptr || top_prob == nullptr || tail == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Ht, W, top_idx, top_prob and tail must be non-NULL");
+  if (p->V < alr::kTopK)
+    return fail(ALR_ERR_INVALID_ARG, "V = %d is below the %d label tokens", p->V, alr::kTopK);
+  if (!aligned16(Ht) || !aligned16(W))
+    return fail(ALR_ERR_INVALID_ARG, "Ht and W must be 16-byte aligned");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  const FwdLayout lay = fwd_layout(p, info.sms, alr::kRFields);
+  if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  CUtensorMap m_h, m_w;
+  if ((rc = make_map(&m_h, Ht, dt, p->d, p->N, p->d * es, k_per_row(dt), 128)) != ALR_OK) return rc;
+  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
+  alr::LossArgs args{};
+  args.plan = loss_plan(p, info.sms, false);
+  args.part = reinterpret_cast<float*>(ws + lay.part_off);
+  args.corpus_tok = corpus_tok;
+  args.status = alr::device_status_ptr();
+  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  cudaError_t e = alr::launch_loss_kernel(alr::kModeReadout, dt, m_h, m_h, m_w, m_w, args, s);
+  if (e != cudaSuccess) return cuda_fail(e, "label readout kernel launch");
+  e = alr::launch_readout_combine(args.plan, args.part, corpus_tok != nullptr, top_idx, top_prob,
+                                  tail, lse_t, argmax_t, gap_t, logp_x, s);
+  if (e != cudaSuccess) return cuda_fail(e, "readout combine launch");
   return ALR_OK;
+}
+
+size_t alr_topk_fwd_workspace_size(const alr_params* p) {
+  if (check_params(p) != ALR_OK) return 0;
+  DevInfo info;
+  if (device_info(&info) != ALR_OK) return 0;
+  return fwd_layout(p, info.sms, alr::kKFields).total;
+}
+
+int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
+                      const float* top_prob, const float* tail, const float* row_mask,
+                      const float* weight_in, const alr_topk_fwd_outputs* out, void* workspace,
+                      size_t ws_bytes, void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
+  if (Hd == nullptr || W == nullptr || out == nullptr || out->loss_row == nullptr ||
+      out->lse_d == nullptr || out->tail_q == nullptr || out->argmax_d == nullptr ||
+      out->weight == nullptr || out->loss_total == nullptr || out->weight_sum == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required top-k forward pointer is NULL");
+  if (!aligned16(Hd) || !aligned16(W))
+    return fail(ALR_ERR_INVALID_ARG, "Hd and W must be 16-byte aligned");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  const FwdLayout lay = fwd_layout(p, info.sms, alr::kKFields);
+  if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  CUtensorMap m_h, m_w;
+  if ((rc = make_map(&m_h, Hd, dt, p->d, p->N, p->d * es, k_per_row(dt), 128)) != ALR_OK) return rc;
+  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
+  alr::LossArgs args{};
+  args.plan = loss_plan(p, info.sms, false);
+  args.part = reinterpret_cast<float*>(ws + lay.part_off);
+  args.top_idx = top_idx;
+  args.status = alr::device_status_ptr();
+  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  cudaError_t e = alr::launch_loss_kernel(alr::kModeTopkFwd, dt, m_h, m_h, m_w, m_w, args, s);
+  if (e != cudaSuccess) return cuda_fail(e, "top-k forward kernel launch");
+  double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
+  e = alr::launch_topk_combine(args.plan, args.part, top_prob, tail, row_mask, weight_in, p->gamma,
+                               out->loss_row, out->lse_d, out->tail_q, out->argmax_d, out->gap_d,
+                               out->weight, anchor, s);
+  if (e != cudaSuccess) return cuda_fail(e, "top-k combine launch");
+  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
+  return ALR_OK;
+}
+
+int alr_topk_logit_grad(const alr_params* p, const void* Hd, const void* W,
+                        const int32_t* top_idx, const float* top_prob, const float* tail,
+                        const float* weight, const float* weight_sum, const float* lse_d,
+                        const float* tail_q, void* G, void* workspace, size_t ws_bytes,
+                        void* stream) {
+  DevInfo info;
+  int rc = check_bwd_args(p, Hd, Hd, W, weight, weight_sum, lse_d, lse_d, &info);
+  if (rc != ALR_OK) return rc;
+  if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
+  if (tail_q == nullptr) return fail(ALR_ERR_INVALID_ARG, "tail_q is NULL");
+  if (G == nullptr || !aligned16(G)) return fail(ALR_ERR_INVALID_ARG, "G must be non-NULL and 16-byte aligned");
+  if ((rc = check_workspace(workspace, ws_bytes, alr_logit_grad_workspace_size(p))) != ALR_OK) return rc;
+  TopkLabels lab;
+  lab.idx = top_idx;
+  lab.prob = top_prob;
+  lab.tail = tail;
+  lab.tail_q = tail_q;
+  return logit_grad_impl(p, Hd, nullptr, W, weight, weight_sum, lse_d, nullptr, lab, G, workspace,
+                         info, static_cast<cudaStream_t>(stream));
+}
+
+int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
+                      const float* top_prob, const float* tail, const float* weight,
+                      const float* weight_sum, const float* lse_d, const float* tail_q,
+                      float* dHd, float* dW, void* workspace, size_t ws_bytes, void* stream) {
+  DevInfo info;
+  int rc = check_bwd_args(p, Hd, Hd, W, weight, weight_sum, lse_d, lse_d, &info);
+  if (rc != ALR_OK) return rc;
+  if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
+  if (tail_q == nullptr || dHd == nullptr) return fail(ALR_ERR_INVALID_ARG, "tail_q and dHd must be non-NULL");
+  if (!aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
+    return fail(ALR_ERR_INVALID_ARG, "dHd and dW must be 16-byte aligned");
+  if ((rc = check_workspace(workspace, ws_bytes, alr_bwd_workspace_size(p))) != ALR_OK) return rc;
+  const BwdLayout lay = bwd_layout(p);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  void* G = ws + lay.g_off;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  TopkLabels lab;
+  lab.idx = top_idx;
+  lab.prob = top_prob;
+  lab.tail = tail;
+  lab.tail_q = tail_q;
+  rc = logit_grad_impl(p, Hd, nullptr, W, weight, weight_sum, lse_d, nullptr, lab, G,
+                       ws + lay.wt_off, info, s);
+  if (rc != ALR_OK) return rc;
+  return head_grads_impl(p, Hd, W, G, dHd, dW, ws, lay, info, s);
 }
 
 int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,

@@ -43,6 +43,26 @@ enum PartField {
   kPFields
 };
 
+// Compact labels (top-k target probabilities + tail bin): k tokens per row.
+constexpr int kTopK = 8;
+
+// Partial record of the label readout: log-sum-exp state, the k best target logits with their
+// token ids, z_t at the corpus token.
+enum ReadoutField { kRM = 0, kRS, kRTop, kRIdx = kRTop + kTopK, kRZx = kRIdx + kTopK, kRFields };
+
+// Partial record of the top-k loss forward: log-sum-exp state and greedy top-2 of z_d, and
+// z_d at the row's k label tokens (NaN where the token is outside the part's columns).
+enum TopkField { kKM = 0, kKS, kKBest, kKIdx, kKSec, kKZ, kKFields = kKZ + kTopK };
+
+// What one launch of the fused loss kernel computes.
+enum LossMode {
+  kModeFwd = 0,      // dual GEMM: full-vocabulary statistics of z_d and z_t
+  kModeBwd = 1,      // dual GEMM: G = c (q - p)
+  kModeReadout = 2,  // single GEMM on H_t: log-sum-exp, top-k, z_t at the corpus token
+  kModeTopkFwd = 3,  // single GEMM on H_d: log-sum-exp, top-2, z_d at the label tokens
+  kModeTopkBwd = 4   // single GEMM on H_d: gradient of the top-k + tail soft CE
+};
+
 struct LossArgs {
   LossPlan plan;
   float* part;                // forward: partial statistics
@@ -55,15 +75,18 @@ struct LossArgs {
   float lam;
   int* status;
   int withhold_first_stage;   // test hook: the producer never fills its first stage
+  const int32_t* top_idx;     // top-k modes: label tokens [N, kTopK]
+  const float* top_prob;      // top-k backward: label probabilities [N, kTopK]
+  const float* tail;          // top-k backward: label tail mass [N]
+  const float* tail_q;        // top-k backward: drafter mass outside the label tokens [N]
 };
 
-// Fused dual-GEMM kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
-cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s);
-// g_store: bf16 G [N, V] as 16-column x 32-row boxes without swizzle (ignored for fp32).
-cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const CUtensorMap& g_store,
-                            const LossArgs& args, cudaStream_t s);
+// Fused loss kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
+//   a0: the first hidden-state operand (H_d; H_t for the readout), a1: H_t (dual modes).
+//   g_store: bf16 G [N, V] as 16-column x 32-row boxes without swizzle (gradient modes, bf16).
+cudaError_t launch_loss_kernel(int mode, int dtype, const CUtensorMap& a0, const CUtensorMap& a1,
+                               const CUtensorMap& w, const CUtensorMap& g_store,
+                               const LossArgs& args, cudaStream_t s);
 
 // Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm.cu).
 struct GemmArgs {
@@ -94,6 +117,15 @@ cudaError_t launch_combine(const LossPlan& plan, const float* part, int mode, fl
                            float* weight, double* anchor_part, cudaStream_t s);
 cudaError_t launch_finalize(const double* anchor_part, int A, float lam, float* loss_total,
                             float* weight_sum, cudaStream_t s);
+cudaError_t launch_readout_combine(const LossPlan& plan, const float* part, bool has_corpus,
+                                   int32_t* top_idx, float* top_prob, float* tail, float* lse_t,
+                                   int32_t* argmax_t, float* gap_t, float* logp_x,
+                                   cudaStream_t s);
+cudaError_t launch_topk_combine(const LossPlan& plan, const float* part, const float* top_prob,
+                                const float* tail, const float* row_mask, const float* weight_in,
+                                float gamma, float* loss_row, float* lse_d, float* tail_q,
+                                int32_t* argmax_d, float* gap_d, float* weight,
+                                double* anchor_part, cudaStream_t s);
 cudaError_t launch_accept_len(const int32_t* am_d, const int32_t* am_t, const float* active,
                               int A, int B, int32_t* acc, int64_t* hist, cudaStream_t s);
 cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,

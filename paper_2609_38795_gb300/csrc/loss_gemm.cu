@@ -1,26 +1,29 @@
-// Fused dual-GEMM kernels of the slot loss on the sm_103a tensor cores.
+// Fused head-GEMM kernels of the slot loss on the sm_103a tensor cores.
 //
-// Both kernels compute, for a 128-row block of H_d and H_t and a kBN-column tile of the
-// vocabulary head W, the two logit tiles z_d = H_d W and z_t = H_t W with tcgen05.mma into
-// tensor memory (fp32 accumulators; the two tiles share every W stage).  The logits never
-// leave the SM:
-//   forward  - the epilogue folds each tile into running per-row statistics (online max /
-//              sum-exp for both sides, the label-weighted sums behind the soft cross-entropy
-//              of Eq. 1, greedy top-2 with lowest-index ties, z_t at the corpus token) and
-//              writes one partial record per row, vocabulary split and 64-column group;
-//   backward - the epilogue forms G = lambda omega_r / sum omega (q - p) for the tile
-//              (the gradient of Eq. 1 with respect to z_d) and streams it to global memory
-//              (bf16: through per-warp shared staging and TMA stores).
+// Every mode computes logit tiles z = H W for a 128-row block of hidden states and a
+// kBN-column tile of the vocabulary head W with tcgen05.mma into tensor memory (fp32
+// accumulators) and consumes them on chip; logits never reach global memory.
+//   kModeFwd     z_d = H_d W and z_t = H_t W (both share every W stage): running per-row
+//                statistics (online max / sum-exp of both sides, the label-weighted sums behind
+//                the soft cross-entropy of Eq. 1, greedy top-2 with lowest-index ties, z_t at
+//                the corpus token), one partial record per row, vocabulary split and 64-column
+//                group;
+//   kModeBwd     the same two tiles recomputed: G = lambda omega_r / sum omega (q - p), the
+//                gradient of Eq. 1 with respect to z_d;
+//   kModeReadout z_t only: log-sum-exp and the k most probable tokens (the label a rollout
+//                step keeps, App. A) plus z_t at the corpus token;
+//   kModeTopkFwd z_d only: log-sum-exp, greedy top-2 and z_d at the row's k label tokens (the
+//                top-k + tail-bin soft CE of Sec. 3.1);
+//   kModeTopkBwd z_d only, recomputed: the gradient of that loss.
 //
-// Tile widths: kBN = 256 (default) uses all 512 TMEM columns for one tile (z_d | z_t) and
-// 64 KB pipeline stages (1024 tensor cycles of work each); kBN = 128 double-buffers the
-// accumulators with 48 KB stages (512 cycles each).
+// Accumulators: the dual modes use 2 x kBN TMEM columns per tile (single-buffered at kBN =
+// 256), the single-operand modes kBN columns (double-buffered, so their epilogue overlaps the
+// next tile's products).
 //
 // Warp roles: warp 0 issues TMA loads, warp 1 owns tensor memory and issues the MMAs from one
 // lane, warps 2.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one row per thread)
 // and the 64 columns [64 g, 64 g + 64) of the tile, g = (w-2)/4, in 16-column sub-chunks.
-// Four epilogue warps per SM sub-partition keep the exposed epilogue short.  Every pipeline
-// wait is bounded (tc_common.cuh).
+// Every pipeline wait is bounded (tc_common.cuh).
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -46,12 +49,16 @@ struct Geo {
   static constexpr bool kTf32 = (kElem == 4);
 };
 
-template <int kBN, bool kStaged>
+constexpr bool is_dual(int mode) { return mode == kModeFwd || mode == kModeBwd; }
+constexpr bool is_grad(int mode) { return mode == kModeBwd || mode == kModeTopkBwd; }
+
+template <int kMode, int kBN, bool kStaged>
 struct Shape {
+  static constexpr int kATiles = is_dual(kMode) ? 2 : 1;
   static constexpr int kBTileBytes = kBN * 128;
-  static constexpr int kStageBytes = 2 * kATileBytes + kBTileBytes;
-  static constexpr int kAccCols = 2 * kBN;             // z_d columns, then z_t columns
-  static constexpr int kAccBufs = 512 / kAccCols;      // 2 for kBN = 128, 1 for kBN = 256
+  static constexpr int kStageBytes = kATiles * kATileBytes + kBTileBytes;
+  static constexpr int kAccCols = kATiles * kBN;       // z_d columns, then z_t columns
+  static constexpr int kAccBufs = 512 / kAccCols;
   static constexpr int kColGroups = kBN / kColsPerWarp;
   static constexpr int kEpiWarps = 4 * kColGroups;
   static constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
@@ -87,6 +94,7 @@ ALR_DEV int split_begin(const LossPlan& p, int vs) {
 }
 
 ALR_DEV float f32(uint32_t x) { return __uint_as_float(x); }
+ALR_DEV float qnan() { return __int_as_float(0x7fc00000); }
 
 // Load 16 consecutive 32-bit TMEM columns of this warp's 32 lanes (see tmem_ld32).
 ALR_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
@@ -111,19 +119,27 @@ ALR_DEV float max16(const float (&z)[16]) {
   return fmaxf(a[0], a[2]);
 }
 
-// Running statistics of one row over the columns one thread sees (forward epilogue).
-// best_x is both the greedy top-1 and the online-softmax reference of side x; s_x sums
-// exp(z_x - best_x); u and w sum exp(z_t - best_t) * z_d and * z_t.
-struct RowStats {
-  float best_d, sec_d, s_d, best_t, sec_t, s_t, u, w, zx;
-  int i_d, i_t;
-};
+// The sub-chunk's values, with columns at or past nv set to -inf.
+template <bool kFull>
+ALR_DEV void load_masked(float (&z)[16], const uint32_t (&r)[16], int nv) {
+#pragma unroll
+  for (int j = 0; j < kSub; ++j) z[j] = (kFull || j < nv) ? f32(r[j]) : -INFINITY;
+}
 
-ALR_DEV void stats_init(RowStats& st) {
-  st.best_d = st.sec_d = st.best_t = st.sec_t = -INFINITY;
-  st.s_d = st.s_t = st.u = st.w = 0.f;
-  st.i_d = st.i_t = 0x7fffffff;
-  st.zx = __int_as_float(0x7fc00000);
+// Online log-sum-exp: move the reference from m to max(m, cm) and add the sub-chunk's
+// exp(z - ref) (masked -inf columns add 0).
+ALR_DEV void lse_update(float& m, float& s, const float (&z)[16], float cm) {
+  const float nm = fmaxf(m, cm);
+  const float sc = ex2((m - nm) * kLog2e);
+  const float b = -nm * kLog2e;
+  float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+  for (int j = 0; j < kSub; j += 2) {
+    r0 += ex2(fmaf(z[j], kLog2e, b));
+    r1 += ex2(fmaf(z[j + 1], kLog2e, b));
+  }
+  s = fmaf(s, sc, r0 + r1);
+  m = nm;
 }
 
 // Greedy top-2 with lowest-index ties, given the sub-chunk maximum cm.  Columns reach a
@@ -144,16 +160,45 @@ ALR_DEV void top2_update(float& best, float& sec, int& idx, const float (&z)[16]
   }
 }
 
-// Fold one 16-column sub-chunk (nv valid columns) into the running statistics.
+// Insert (v, i) into a list sorted by value descending; an equal value stays below the
+// entries already there (they came from lower columns).
+ALR_DEV void topk_insert(float (&t)[kTopK], int (&ti)[kTopK], float v, int i) {
+  t[kTopK - 1] = v;
+  ti[kTopK - 1] = i;
+#pragma unroll
+  for (int k = kTopK - 1; k > 0; --k) {
+    const bool up = t[k] > t[k - 1];
+    const float a = t[k], b = t[k - 1];
+    const int ia = ti[k], ib = ti[k - 1];
+    t[k - 1] = up ? a : b;
+    t[k] = up ? b : a;
+    ti[k - 1] = up ? ia : ib;
+    ti[k] = up ? ib : ia;
+  }
+}
+
+// Running statistics of one row over the columns one thread sees (full-vocabulary forward).
+// best_x is both the greedy top-1 and the online-softmax reference of side x; s_x sums
+// exp(z_x - best_x); u and w sum exp(z_t - best_t) * z_d and * z_t.
+struct RowStats {
+  float best_d, sec_d, s_d, best_t, sec_t, s_t, u, w, zx;
+  int i_d, i_t;
+};
+
+ALR_DEV void stats_init(RowStats& st) {
+  st.best_d = st.sec_d = st.best_t = st.sec_t = -INFINITY;
+  st.s_d = st.s_t = st.u = st.w = 0.f;
+  st.i_d = st.i_t = 0x7fffffff;
+  st.zx = qnan();
+}
+
+// Fold one 16-column sub-chunk (nv valid columns) into the full-vocabulary statistics.
 template <bool kFull>
 ALR_DEV void stats_sub(RowStats& st, const uint32_t (&rd)[16], const uint32_t (&rt)[16], int v0,
                        int nv, int x) {
   float zd[16], zt[16];
-#pragma unroll
-  for (int j = 0; j < kSub; ++j) {
-    zd[j] = (kFull || j < nv) ? f32(rd[j]) : -INFINITY;
-    zt[j] = (kFull || j < nv) ? f32(rt[j]) : -INFINITY;
-  }
+  load_masked<kFull>(zd, rd, nv);
+  load_masked<kFull>(zt, rt, nv);
   const float cd = max16(zd), ct = max16(zt);
   // target side: rescale to the new running maximum, then add this sub-chunk
   const float nbt = fmaxf(st.best_t, ct);
@@ -179,17 +224,9 @@ ALR_DEV void stats_sub(RowStats& st, const uint32_t (&rd)[16], const uint32_t (&
   st.u = fmaf(st.u, sct, u0 + u1);
   st.w = fmaf(st.w, sct, w0 + w1);
   // drafter side
-  const float nbd = fmaxf(st.best_d, cd);
-  const float scd = ex2((st.best_d - nbd) * kLog2e);
-  const float bd = -nbd * kLog2e;
-  float r0 = 0.f, r1 = 0.f;
-#pragma unroll
-  for (int j = 0; j < kSub; j += 2) {
-    r0 += ex2(fmaf(zd[j], kLog2e, bd));      // masked columns are -inf: exp gives 0
-    r1 += ex2(fmaf(zd[j + 1], kLog2e, bd));
-  }
-  st.s_d = fmaf(st.s_d, scd, r0 + r1);
-  // greedy top-2 of both sides (moves best_d / best_t to nbd / nbt)
+  float m_d = st.best_d;
+  lse_update(m_d, st.s_d, zd, cd);
+  // greedy top-2 of both sides (moves best_d / best_t to the new maxima)
   top2_update(st.best_d, st.sec_d, st.i_d, zd, cd, v0);
   top2_update(st.best_t, st.sec_t, st.i_t, zt, ct, v0);
   const int xr = x - v0;
@@ -212,18 +249,56 @@ ALR_DEV bool warp_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
   return __shfl_sync(0xffffffffu, ok, 0) != 0;
 }
 
+// Write one warp's 32 x 16 sub-chunk of G: bf16 through its shared staging buffer and a TMA
+// store (the buffer used two stores ago must have been read first), fp32 directly.
+template <typename Elem, bool kStaged>
+ALR_DEV void store_g(const float (&g)[16], uint8_t* my_stage, uint32_t& n_stores,
+                     const CUtensorMap* tm_g, Elem* grow, int v0, int row0, bool row_ok, int V,
+                     int lane) {
+  if constexpr (kStaged) {
+    uint8_t* buf = my_stage + (n_stores & 1u) * kGStageBytes;
+    if (lane == 0) tma_store_wait_read_le1();
+    __syncwarp();
+    uint4 a, b;
+    a.x = pack_bf16x2(g[0], g[1]);
+    a.y = pack_bf16x2(g[2], g[3]);
+    a.z = pack_bf16x2(g[4], g[5]);
+    a.w = pack_bf16x2(g[6], g[7]);
+    b.x = pack_bf16x2(g[8], g[9]);
+    b.y = pack_bf16x2(g[10], g[11]);
+    b.z = pack_bf16x2(g[12], g[13]);
+    b.w = pack_bf16x2(g[14], g[15]);
+    *reinterpret_cast<uint4*>(buf + lane * 32) = a;
+    *reinterpret_cast<uint4*>(buf + lane * 32 + 16) = b;
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tm_g, buf, v0, row0);
+      tma_store_commit();
+    }
+    ++n_stores;
+  } else if (row_ok) {
+#pragma unroll
+    for (int i = 0; i < kSub / 4; ++i) {
+      if (v0 + 4 * i < V)
+        *reinterpret_cast<float4*>(grow + v0 + 4 * i) =
+            make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
+    }
+  }
+}
+
 // kWMN: the head tile is read MN-major straight from W [d, V] (bf16), or K-major from a
 // transposed copy W^T [V, d] (fp32 inputs, whose tf32 products take K-major operands only).
-// kStaged: the backward stores bf16 G through shared staging and TMA (tm_g), else directly.
-template <typename Elem, bool kBwd, bool kWMN, int kBN>
-__global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThreads, 1)
-    loss_gemm_kernel(const __grid_constant__ CUtensorMap tm_hd,
-                     const __grid_constant__ CUtensorMap tm_ht,
+template <typename Elem, int kMode, bool kWMN, int kBN>
+__global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Elem) == 2>::kThreads, 1)
+    loss_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,
+                     const __grid_constant__ CUtensorMap tm_a1,
                      const __grid_constant__ CUtensorMap tm_w,
                      const __grid_constant__ CUtensorMap tm_g, const LossArgs args) {
   using G = Geo<Elem>;
-  constexpr bool kStaged = kBwd && sizeof(Elem) == 2;
-  using S = Shape<kBN, kStaged>;
+  constexpr bool kDual = is_dual(kMode);
+  constexpr bool kStaged = is_grad(kMode) && sizeof(Elem) == 2;
+  using S = Shape<kMode, kBN, kStaged>;
   constexpr int kStages = S::kStages;
 
   extern __shared__ uint8_t smem_raw[];
@@ -257,8 +332,8 @@ __global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThread
     fence_mbar_init();
   }
   if (threadIdx.x == 32) {
-    tma_prefetch_desc(&tm_hd);
-    tma_prefetch_desc(&tm_ht);
+    tma_prefetch_desc(&tm_a0);
+    if (kDual) tma_prefetch_desc(&tm_a1);
     tma_prefetch_desc(&tm_w);
     if (kStaged) tma_prefetch_desc(&tm_g);
   }
@@ -299,16 +374,18 @@ __global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThread
               continue;
             }
             uint8_t* sb = stage_mem + stage * S::kStageBytes;
+            uint8_t* sw = sb + S::kATiles * kATileBytes;
             mbar_arrive_expect_tx(&full_bar[stage], S::kStageBytes);
-            tma_load_2d(sb, &tm_hd, &full_bar[stage], kb * G::kKE, rb * kBM);
-            tma_load_2d(sb + kATileBytes, &tm_ht, &full_bar[stage], kb * G::kKE, rb * kBM);
+            tma_load_2d(sb, &tm_a0, &full_bar[stage], kb * G::kKE, rb * kBM);
+            if constexpr (kDual)
+              tma_load_2d(sb + kATileBytes, &tm_a1, &full_bar[stage], kb * G::kKE, rb * kBM);
             if constexpr (kWMN) {
 #pragma unroll
               for (int c = 0; c < kBN / G::kChunkMN; ++c)
-                tma_load_2d(sb + 2 * kATileBytes + c * G::kChunkBytes, &tm_w, &full_bar[stage],
+                tma_load_2d(sw + c * G::kChunkBytes, &tm_w, &full_bar[stage],
                             vt * kBN + c * G::kChunkMN, kb * G::kKE);
             } else {
-              tma_load_2d(sb + 2 * kATileBytes, &tm_w, &full_bar[stage], kb * G::kKE, vt * kBN);
+              tma_load_2d(sw, &tm_w, &full_bar[stage], kb * G::kKE, vt * kBN);
             }
             armed |= 1u << stage;
             armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
@@ -349,16 +426,17 @@ __global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThread
             }
             tc_fence_after();
             const uint32_t sa = smem_u32(stage_mem + stage * S::kStageBytes);
+            const uint32_t swb = sa + S::kATiles * kATileBytes;
 #pragma unroll
             for (int kk = 0; kk < G::kKE / G::kMmaK; ++kk) {
-              const uint64_t ad = sdesc_sw128(sa + kk * 32, 16, 1024);
-              const uint64_t at = sdesc_sw128(sa + kATileBytes + kk * 32, 16, 1024);
               const uint64_t bd =
-                  kWMN ? sdesc_sw128(sa + 2 * kATileBytes + kk * G::kMmaK * 128, G::kChunkBytes, 1024)
-                       : sdesc_sw128(sa + 2 * kATileBytes + kk * 32, 16, 1024);
+                  kWMN ? sdesc_sw128(swb + kk * G::kMmaK * 128, G::kChunkBytes, 1024)
+                       : sdesc_sw128(swb + kk * 32, 16, 1024);
               const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
-              mma_issue<G::kTf32>(d_acc, ad, bd, idesc, acc);
-              mma_issue<G::kTf32>(d_acc + kBN, at, bd, idesc, acc);
+              mma_issue<G::kTf32>(d_acc, sdesc_sw128(sa + kk * 32, 16, 1024), bd, idesc, acc);
+              if constexpr (kDual)
+                mma_issue<G::kTf32>(d_acc + kBN, sdesc_sw128(sa + kATileBytes + kk * 32, 16, 1024),
+                                    bd, idesc, acc);
             }
             mma_commit(&empty_bar[stage]);
             if (++stage == kStages) {
@@ -395,44 +473,150 @@ __global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThread
       const int vt1 = split_begin(P, vs + 1);
       const int row = rb * kBM + row_in_tile;
       const bool row_ok = row < P.N;
-      if constexpr (!kBwd) {
-        RowStats st;
-        stats_init(st);
-        const int x = (args.corpus_tok != nullptr && row_ok) ? args.corpus_tok[row] : -1;
-        for (int vt = split_begin(P, vs); vt < vt1; ++vt) {
-          if (!warp_wait(&tfull_bar[abuf], aphase, ab)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
-          const int vbase = vt * kBN + cg * kColsPerWarp;
-#pragma unroll 1
-          for (int c = 0; c < kColsPerWarp / kSub; ++c) {
-            uint32_t rd[16], rt[16];
-            tmem_ld16(tb + c * kSub, rd);
-            tmem_ld16(tb + kBN + c * kSub, rt);
-            tmem_ld_wait();
-            reg_fence(rd);
-            reg_fence(rt);
-            const int v0 = vbase + c * kSub;
-            if (v0 + kSub <= P.V) {
-              stats_sub<true>(st, rd, rt, v0, kSub, x);
-            } else if (v0 < P.V) {
-              stats_sub<false>(st, rd, rt, v0, P.V - v0, x);
-            }
-          }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&tempty_bar[abuf]);
-          if (++abuf == S::kAccBufs) {
-            abuf = 0;
-            aphase ^= 1;
+      const size_t part = size_t(vs * S::kColGroups + cg);
+      const size_t fs = size_t(P.n_parts) * P.N;
+
+      // ---- per-row state for this unit ----
+      RowStats st;                       // kModeFwd
+      float m = -INFINITY, s = 0.f;      // single-operand log-sum-exp state
+      float best = -INFINITY, sec = -INFINITY, zx = qnan();
+      int bidx = 0x7fffffff, x = -1;
+      float tk[kTopK];                   // readout: k best values / top-k forward: z_d at labels
+      int ti[kTopK];                     // readout: their ids / top-k modes: label tokens
+      float tp[kTopK];                   // top-k backward: label probabilities
+      float ad = 0.f, at = 0.f, cw = 0.f, beta = 1.f;
+#pragma unroll
+      for (int i = 0; i < kTopK; ++i) {
+        tk[i] = kMode == kModeReadout ? -INFINITY : qnan();
+        ti[i] = kMode == kModeReadout ? 0x7fffffff : -1;
+        tp[i] = 0.f;
+      }
+      if constexpr (kMode == kModeFwd) stats_init(st);
+      if constexpr (kMode == kModeFwd || kMode == kModeReadout)
+        x = (args.corpus_tok != nullptr && row_ok) ? args.corpus_tok[row] : -1;
+      if constexpr (kMode == kModeTopkFwd || kMode == kModeTopkBwd) {
+        if (row_ok) {
+#pragma unroll
+          for (int i = 0; i < kTopK; ++i) ti[i] = args.top_idx[size_t(row) * kTopK + i];
+        }
+      }
+      if constexpr (is_grad(kMode)) {
+        if (row_ok) {
+          ad = -args.lse_d[row] * kLog2e;
+          const float ws = *args.weight_sum;
+          cw = ws > 0.f ? args.lam * args.weight[row] / ws : 0.f;
+          if constexpr (kMode == kModeBwd) {
+            at = -args.lse_t[row] * kLog2e;
+          } else {
+            const float tl = args.tail[row];
+            beta = tl > 0.f ? 1.f - tl / args.tail_q[row] : 1.f;
+#pragma unroll
+            for (int i = 0; i < kTopK; ++i) tp[i] = args.top_prob[size_t(row) * kTopK + i];
           }
         }
-        if (ok && row_ok) {
-          const size_t fs = size_t(P.n_parts) * P.N;
-          float* o = args.part + size_t(vs * S::kColGroups + cg) * P.N + row;
+      }
+      Elem* grow = static_cast<Elem*>(args.G) + size_t(row_ok ? row : 0) * size_t(P.V);
+
+      for (int vt = split_begin(P, vs); vt < vt1; ++vt) {
+        if (!warp_wait(&tfull_bar[abuf], aphase, ab)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
+        const int vbase = vt * kBN + cg * kColsPerWarp;
+#pragma unroll 1
+        for (int c = 0; c < kColsPerWarp / kSub; ++c) {
+          uint32_t r0[16], r1[16];
+          tmem_ld16(tb + c * kSub, r0);
+          if constexpr (kDual) tmem_ld16(tb + kBN + c * kSub, r1);
+          tmem_ld_wait();
+          reg_fence(r0);
+          if constexpr (kDual) reg_fence(r1);
+          const int v0 = vbase + c * kSub;
+          if (v0 >= P.V) continue;   // warp-uniform: the whole sub-chunk is past the vocabulary
+          const int nv = min(kSub, P.V - v0);
+
+          if constexpr (kMode == kModeFwd) {
+            if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x);
+            else stats_sub<false>(st, r0, r1, v0, nv, x);
+          } else if constexpr (kMode == kModeReadout || kMode == kModeTopkFwd) {
+            float z[16];
+            if (nv == kSub) load_masked<true>(z, r0, nv);
+            else load_masked<false>(z, r0, nv);
+            const float cm = max16(z);
+            lse_update(m, s, z, cm);
+            if constexpr (kMode == kModeReadout) {
+              if (cm > tk[kTopK - 1]) {   // some column of this sub-chunk enters the top k
+#pragma unroll
+                for (int j = 0; j < kSub; ++j)
+                  if (z[j] > tk[kTopK - 1]) topk_insert(tk, ti, z[j], v0 + j);
+              }
+              const int xr = x - v0;
+              if (xr >= 0 && xr < nv) {
+#pragma unroll
+                for (int j = 0; j < kSub; ++j)
+                  if (j == xr) zx = z[j];
+              }
+            } else {
+              top2_update(best, sec, bidx, z, cm, v0);
+              bool hit = false;
+#pragma unroll
+              for (int i = 0; i < kTopK; ++i) hit |= unsigned(ti[i] - v0) < unsigned(nv);
+              if (hit) {
+#pragma unroll
+                for (int i = 0; i < kTopK; ++i) {
+                  const int rel = ti[i] - v0;
+#pragma unroll
+                  for (int j = 0; j < kSub; ++j)
+                    if (j == rel) tk[i] = z[j];
+                }
+              }
+            }
+          } else {   // gradient modes
+            float g[16];
+            if constexpr (kMode == kModeBwd) {
+#pragma unroll
+              for (int j = 0; j < kSub; ++j)
+                g[j] = cw * (ex2(fmaf(f32(r0[j]), kLog2e, ad)) - ex2(fmaf(f32(r1[j]), kLog2e, at)));
+            } else {
+              float qv[16];
+              const float cb = cw * beta;
+#pragma unroll
+              for (int j = 0; j < kSub; ++j) {
+                qv[j] = ex2(fmaf(f32(r0[j]), kLog2e, ad));
+                g[j] = cb * qv[j];
+              }
+              bool hit = false;
+#pragma unroll
+              for (int i = 0; i < kTopK; ++i) hit |= unsigned(ti[i] - v0) < unsigned(nv);
+              if (hit) {   // the row's label tokens in this sub-chunk: c (q - prob)
+#pragma unroll
+                for (int i = 0; i < kTopK; ++i) {
+                  const int rel = ti[i] - v0;
+#pragma unroll
+                  for (int j = 0; j < kSub; ++j)
+                    if (j == rel) g[j] = cw * (qv[j] - tp[i]);
+                }
+              }
+            }
+            store_g<Elem, kStaged>(g, my_stage, n_stores, &tm_g, grow, v0, rb * kBM + q * 32,
+                                   row_ok, P.V, lane);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty_bar[abuf]);
+        if (++abuf == S::kAccBufs) {
+          abuf = 0;
+          aphase ^= 1;
+        }
+      }
+
+      // ---- per-row partial record at the end of the unit ----
+      if (ok && row_ok) {
+        float* o = args.part + part * P.N + row;
+        if constexpr (kMode == kModeFwd) {
           o[kPMd * fs] = st.best_d;
           o[kPSd * fs] = st.s_d;
           o[kPMt * fs] = st.best_t;
@@ -446,78 +630,23 @@ __global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThread
           o[kPIt * fs] = __int_as_float(st.i_t);
           o[kPSect * fs] = st.sec_t;
           o[kPZx * fs] = st.zx;
-        }
-      } else {
-        float ad = 0.f, at = 0.f, cw = 0.f;
-        if (row_ok) {
-          ad = -args.lse_d[row] * kLog2e;
-          at = -args.lse_t[row] * kLog2e;
-          const float ws = *args.weight_sum;
-          cw = ws > 0.f ? args.lam * args.weight[row] / ws : 0.f;
-        }
-        Elem* grow = static_cast<Elem*>(args.G) + size_t(row_ok ? row : 0) * size_t(P.V);
-        for (int vt = split_begin(P, vs); vt < vt1; ++vt) {
-          if (!warp_wait(&tfull_bar[abuf], aphase, ab)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
-          const int vbase = vt * kBN + cg * kColsPerWarp;
-#pragma unroll 1
-          for (int c = 0; c < kColsPerWarp / kSub; ++c) {
-            uint32_t rd[16], rt[16];
-            tmem_ld16(tb + c * kSub, rd);
-            tmem_ld16(tb + kBN + c * kSub, rt);
-            tmem_ld_wait();
-            reg_fence(rd);
-            reg_fence(rt);
-            const int v0 = vbase + c * kSub;
-            if (v0 >= P.V) continue;   // warp-uniform
-            float g[16];
+        } else if constexpr (kMode == kModeReadout) {
+          o[kRM * fs] = m;
+          o[kRS * fs] = s;
 #pragma unroll
-            for (int j = 0; j < kSub; ++j)
-              g[j] = cw * (ex2(fmaf(f32(rd[j]), kLog2e, ad)) - ex2(fmaf(f32(rt[j]), kLog2e, at)));
-            if constexpr (kStaged) {
-              // this warp's 32 x 16 sub-chunk -> shared staging -> one TMA store; the buffer
-              // used two stores ago must have been read before it is overwritten
-              uint8_t* buf = my_stage + (n_stores & 1u) * kGStageBytes;
-              if (lane == 0) tma_store_wait_read_le1();
-              __syncwarp();
-              uint4 v0v, v1v;
-              v0v.x = pack_bf16x2(g[0], g[1]);
-              v0v.y = pack_bf16x2(g[2], g[3]);
-              v0v.z = pack_bf16x2(g[4], g[5]);
-              v0v.w = pack_bf16x2(g[6], g[7]);
-              v1v.x = pack_bf16x2(g[8], g[9]);
-              v1v.y = pack_bf16x2(g[10], g[11]);
-              v1v.z = pack_bf16x2(g[12], g[13]);
-              v1v.w = pack_bf16x2(g[14], g[15]);
-              *reinterpret_cast<uint4*>(buf + lane * 32) = v0v;
-              *reinterpret_cast<uint4*>(buf + lane * 32 + 16) = v1v;
-              fence_proxy_async_smem();
-              __syncwarp();
-              if (lane == 0) {
-                tma_store_2d(&tm_g, buf, v0, rb * kBM + q * 32);
-                tma_store_commit();
-              }
-              ++n_stores;
-            } else if (row_ok) {
+          for (int i = 0; i < kTopK; ++i) {
+            o[(kRTop + i) * fs] = tk[i];
+            o[(kRIdx + i) * fs] = __int_as_float(ti[i]);
+          }
+          o[kRZx * fs] = zx;
+        } else if constexpr (kMode == kModeTopkFwd) {
+          o[kKM * fs] = m;
+          o[kKS * fs] = s;
+          o[kKBest * fs] = best;
+          o[kKIdx * fs] = __int_as_float(bidx);
+          o[kKSec * fs] = sec;
 #pragma unroll
-              for (int i = 0; i < kSub / 4; ++i) {
-                if (v0 + 4 * i < P.V)
-                  *reinterpret_cast<float4*>(grow + v0 + 4 * i) =
-                      make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
-              }
-            }
-          }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&tempty_bar[abuf]);
-          if (++abuf == S::kAccBufs) {
-            abuf = 0;
-            aphase ^= 1;
-          }
+          for (int i = 0; i < kTopK; ++i) o[(kKZ + i) * fs] = tk[i];
         }
       }
     }
@@ -534,41 +663,45 @@ __global__ void __launch_bounds__(Shape<kBN, kBwd && sizeof(Elem) == 2>::kThread
   }
 }
 
-template <typename Elem, bool kBwd, int kBN>
-cudaError_t launch_impl(const CUtensorMap& hd, const CUtensorMap& ht, const CUtensorMap& w,
+template <typename Elem, int kMode, int kBN>
+cudaError_t launch_impl(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
                         const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
-  using S = Shape<kBN, kBwd && sizeof(Elem) == 2>;
-  auto kern = loss_gemm_kernel<Elem, kBwd, sizeof(Elem) == 2, kBN>;
+  using S = Shape<kMode, kBN, is_grad(kMode) && sizeof(Elem) == 2>;
+  auto kern = loss_gemm_kernel<Elem, kMode, sizeof(Elem) == 2, kBN>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
   if (e != cudaSuccess) return e;
-  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(hd, ht, w, g, args);
+  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(a0, a1, w, g, args);
   return cudaGetLastError();
 }
 
-template <bool kBwd>
-cudaError_t dispatch(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                     const CUtensorMap& w, const CUtensorMap& g, const LossArgs& args,
-                     cudaStream_t s) {
-  if (args.plan.bn == 128) {
-    if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 128>(hd, ht, w, g, args, s);
-    return launch_impl<float, kBwd, 128>(hd, ht, w, g, args, s);
+template <typename Elem, int kMode>
+cudaError_t by_width(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
+                     const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
+  if (args.plan.bn == 128) return launch_impl<Elem, kMode, 128>(a0, a1, w, g, args, s);
+  return launch_impl<Elem, kMode, 256>(a0, a1, w, g, args, s);
+}
+
+template <typename Elem>
+cudaError_t by_mode(int mode, const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
+                    const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
+  switch (mode) {
+    case kModeFwd: return by_width<Elem, kModeFwd>(a0, a1, w, g, args, s);
+    case kModeBwd: return by_width<Elem, kModeBwd>(a0, a1, w, g, args, s);
+    case kModeReadout: return by_width<Elem, kModeReadout>(a0, a1, w, g, args, s);
+    case kModeTopkFwd: return by_width<Elem, kModeTopkFwd>(a0, a1, w, g, args, s);
+    case kModeTopkBwd: return by_width<Elem, kModeTopkBwd>(a0, a1, w, g, args, s);
+    default: return cudaErrorInvalidValue;
   }
-  if (dtype == 0) return launch_impl<__nv_bfloat16, kBwd, 256>(hd, ht, w, g, args, s);
-  return launch_impl<float, kBwd, 256>(hd, ht, w, g, args, s);
 }
 
 }  // namespace
 
-cudaError_t launch_loss_fwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const LossArgs& args, cudaStream_t s) {
-  return dispatch<false>(dtype, hd, ht, w, w, args, s);
-}
-
-cudaError_t launch_loss_bwd(int dtype, const CUtensorMap& hd, const CUtensorMap& ht,
-                            const CUtensorMap& w, const CUtensorMap& g_store,
-                            const LossArgs& args, cudaStream_t s) {
-  return dispatch<true>(dtype, hd, ht, w, g_store, args, s);
+cudaError_t launch_loss_kernel(int mode, int dtype, const CUtensorMap& a0, const CUtensorMap& a1,
+                               const CUtensorMap& w, const CUtensorMap& g_store,
+                               const LossArgs& args, cudaStream_t s) {
+  if (dtype == 0) return by_mode<__nv_bfloat16>(mode, a0, a1, w, g_store, args, s);
+  return by_mode<float>(mode, a0, a1, w, g_store, args, s);
 }
 
 }  // namespace alr

@@ -256,6 +256,154 @@ __global__ void __launch_bounds__(256) erase_weights_kernel(
   }
 }
 
+// ---------------------------------------------------------- compact labels ---
+// Insert (v, id) into a list sorted by value descending, equal values by id ascending.
+__device__ __forceinline__ void insert_ranked(float (&t)[kTopK], int (&ti)[kTopK], float v,
+                                              int id) {
+  if (!(v > t[kTopK - 1] || (v == t[kTopK - 1] && id < ti[kTopK - 1]))) return;
+  t[kTopK - 1] = v;
+  ti[kTopK - 1] = id;
+#pragma unroll
+  for (int k = kTopK - 1; k > 0; --k) {
+    const bool up = t[k] > t[k - 1] || (t[k] == t[k - 1] && ti[k] < ti[k - 1]);
+    const float a = t[k], b = t[k - 1];
+    const int ia = ti[k], ib = ti[k - 1];
+    t[k - 1] = up ? a : b;
+    t[k] = up ? b : a;
+    ti[k - 1] = up ? ia : ib;
+    ti[k] = up ? ib : ia;
+  }
+}
+
+// Label readout merge, one thread per row: log-sum-exp over all parts, the k best target
+// logits (ties to the lower id), their probabilities and the tail mass
+//   tail = (S - sum_k exp(t_k - M)) / S,
+// the greedy token with its top-1 minus top-2 gap, and log p at the corpus token.
+__global__ void __launch_bounds__(256) readout_combine_kernel(
+    LossPlan P, const float* __restrict__ part, int has_corpus, int32_t* __restrict__ top_idx,
+    float* __restrict__ top_prob, float* __restrict__ tail, float* __restrict__ lse_t,
+    int32_t* __restrict__ argmax_t, float* __restrict__ gap_t, float* __restrict__ logp_x) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= P.N) return;
+  const size_t fs = size_t(P.n_parts) * P.N;
+  float M = -INFINITY, S = 0.f, zx = quiet_nan();
+  float t[kTopK];
+  int ti[kTopK];
+#pragma unroll
+  for (int i = 0; i < kTopK; ++i) {
+    t[i] = -INFINITY;
+    ti[i] = 0x7fffffff;
+  }
+  for (int k = 0; k < P.n_parts; ++k) {
+    const float* p = part + size_t(k) * P.N + r;
+    const float m = p[kRM * fs];
+    const float nm = fmaxf(M, m);
+    S = S * ex2((M - nm) * kLog2e) + p[kRS * fs] * ex2((m - nm) * kLog2e);
+    M = nm;
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) {
+      const float v = p[(kRTop + i) * fs];
+      if (v > -INFINITY) insert_ranked(t, ti, v, __float_as_int(p[(kRIdx + i) * fs]));
+    }
+    const float z = p[kRZx * fs];
+    if (z == z) zx = z;
+  }
+  const float lse = M + logf(S);
+  double inside = 0.0;
+#pragma unroll
+  for (int i = 0; i < kTopK; ++i) {
+    top_idx[size_t(r) * kTopK + i] = ti[i];
+    top_prob[size_t(r) * kTopK + i] = expf(t[i] - lse);
+    inside += exp(double(t[i]) - double(M));
+  }
+  // with V <= k every token is in the list and the tail is empty by definition
+  tail[r] = P.V <= kTopK ? 0.f : float(fmax(0.0, (double(S) - inside) / double(S)));
+  if (lse_t) lse_t[r] = lse;
+  if (argmax_t) argmax_t[r] = ti[0];
+  if (gap_t) gap_t[r] = t[0] - t[1];
+  if (has_corpus && logp_x) logp_x[r] = zx - lse;
+}
+
+// Top-k loss merge, one warp per anchor: log-sum-exp and greedy top-2 of z_d, the label
+// tokens' z_d, the drafter's mass outside them
+//   tail_q = (S_d - sum_i exp(z_i - M_d)) / S_d,
+// the loss l = -sum_i prob_i (z_i - LSE_d) - tail log tail_q (no tail term when tail = 0),
+// the slot weight (given, or envelope times mask) and the anchor's sums for Eq. 1.
+__global__ void __launch_bounds__(256) topk_combine_kernel(
+    LossPlan P, const float* __restrict__ part, const float* __restrict__ top_prob,
+    const float* __restrict__ tail, const float* __restrict__ row_mask,
+    const float* __restrict__ weight_in, float gamma, float* __restrict__ loss_row,
+    float* __restrict__ lse_d_out, float* __restrict__ tail_q_out, int32_t* __restrict__ argmax_d,
+    float* __restrict__ gap_d, float* __restrict__ weight, double* __restrict__ anchor_part) {
+  const int A = P.N / P.B;
+  const int a = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (a >= A) return;
+  const bool active = lane < P.B;
+  const int r = a * P.B + (active ? lane : 0);
+  const size_t fs = size_t(P.n_parts) * P.N;
+  float M = -INFINITY, S = 0.f, bd = -INFINITY, secd = -INFINITY;
+  int id = 0x7fffffff;
+  float zk[kTopK];
+#pragma unroll
+  for (int i = 0; i < kTopK; ++i) zk[i] = quiet_nan();
+  if (active) {
+    for (int k = 0; k < P.n_parts; ++k) {
+      const float* p = part + size_t(k) * P.N + r;
+      const float m = p[kKM * fs];
+      const float nm = fmaxf(M, m);
+      S = S * ex2((M - nm) * kLog2e) + p[kKS * fs] * ex2((m - nm) * kLog2e);
+      M = nm;
+      const float b2 = p[kKBest * fs], s2 = p[kKSec * fs];
+      const int i2 = __float_as_int(p[kKIdx * fs]);
+      if (b2 > bd || (b2 == bd && i2 < id)) {
+        secd = fmaxf(bd, s2);
+        bd = b2;
+        id = i2;
+      } else {
+        secd = fmaxf(secd, b2);
+      }
+#pragma unroll
+      for (int i = 0; i < kTopK; ++i) {
+        const float z = p[(kKZ + i) * fs];
+        if (z == z) zk[i] = z;
+      }
+    }
+  }
+  float loss = 0.f, w = 0.f;
+  if (active) {
+    const float lse = M + logf(S);
+    double inside = 0.0, ce = 0.0;
+    for (int i = 0; i < kTopK; ++i) {
+      inside += exp(double(zk[i]) - double(M));
+      ce -= double(top_prob[size_t(r) * kTopK + i]) * (double(zk[i]) - double(lse));
+    }
+    const double tq = fmax((double(S) - inside) / double(S), 1e-30);
+    const float tl = tail[r];
+    if (tl > 0.f) ce -= double(tl) * log(tq);
+    loss = float(ce);
+    w = weight_in != nullptr ? weight_in[r]
+                             : expf(-float(lane) / gamma) * (row_mask ? row_mask[r] : 1.f);
+    loss_row[r] = loss;
+    lse_d_out[r] = lse;
+    tail_q_out[r] = float(tq);
+    argmax_d[r] = id;
+    if (gap_d) gap_d[r] = bd - secd;
+    weight[r] = w;
+  }
+  double wl = active ? double(w) * double(loss) : 0.0;
+  double ws = active ? double(w) : 0.0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    wl += __shfl_xor_sync(0xffffffffu, wl, off);
+    ws += __shfl_xor_sync(0xffffffffu, ws, off);
+  }
+  if (lane == 0) {
+    anchor_part[2 * a] = wl;
+    anchor_part[2 * a + 1] = ws;
+  }
+}
+
 // ------------------------------------------------------------------ transpose ---
 // out[c * ld_out + r] = in[r * C + c] for 32-bit elements, 32 x 32 tiles through shared memory.
 __global__ void __launch_bounds__(256) transpose32_kernel(const float* __restrict__ in,
@@ -304,6 +452,28 @@ cudaError_t launch_combine(const LossPlan& plan, const float* part, int mode, fl
   combine_kernel<<<(A + 7) / 8, 256, 0, s>>>(plan, part, mode, gamma, row_mask, corpus_tok,
                                              loss_row, ent_row, lse_d, lse_t, argmax_d, argmax_t,
                                              gap_d, gap_t, logp_x, weight, anchor_part);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_readout_combine(const LossPlan& plan, const float* part, bool has_corpus,
+                                   int32_t* top_idx, float* top_prob, float* tail, float* lse_t,
+                                   int32_t* argmax_t, float* gap_t, float* logp_x,
+                                   cudaStream_t s) {
+  readout_combine_kernel<<<(plan.N + 255) / 256, 256, 0, s>>>(plan, part, has_corpus ? 1 : 0,
+                                                              top_idx, top_prob, tail, lse_t,
+                                                              argmax_t, gap_t, logp_x);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_topk_combine(const LossPlan& plan, const float* part, const float* top_prob,
+                                const float* tail, const float* row_mask, const float* weight_in,
+                                float gamma, float* loss_row, float* lse_d, float* tail_q,
+                                int32_t* argmax_d, float* gap_d, float* weight,
+                                double* anchor_part, cudaStream_t s) {
+  const int A = plan.N / plan.B;
+  topk_combine_kernel<<<(A + 7) / 8, 256, 0, s>>>(plan, part, top_prob, tail, row_mask, weight_in,
+                                                  gamma, loss_row, lse_d, tail_q, argmax_d, gap_d,
+                                                  weight, anchor_part);
   return cudaGetLastError();
 }
 
