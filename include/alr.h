@@ -124,6 +124,28 @@ int alr_gather_ira_blocks(const void* feat, int32_t S, int32_t L, int32_t d, int
                           const int32_t* seq, const int32_t* pos, const int32_t* valid_len,
                           int32_t A, int32_t B, void* out, float* row_valid, void* stream);
 
+/*
+ * IRA block plan (Sec. 3.2, In-rollout anchors; Eq. 4; App. A).  For S samples, sample s with
+ * valid_anchors[s] = v valid anchor positions keeps m = min(v, max_blocks) blocks: the first
+ * ceil(m/2) are primary (their rollouts produce labels), the next floor(m/2) secondary, the
+ * rest unused.  Secondary block i sits in primary block i's rollout at offset
+ * j = offsets[s * (max_blocks/2) + i] (the method draws j ~ U{2..K-1}; the caller passes the
+ * draws; j outside [1, K-1] leaves the block unused).  Primary block p of sample s owns rows
+ * [s*P + p] of a label buffer [S*P, K, ...] with P = max_blocks - max_blocks/2, of which
+ * rollout_len[s*P + p] are valid (K, fewer after early termination).
+ * Outputs per block slot t = s*max_blocks + b (int32 [S*max_blocks]):
+ *   seq, pos, valid_len - the alr_gather_ira_blocks arguments that read the block's K label
+ *             rows from that buffer: a secondary block's row k reads primary row j + k - 1 and
+ *             is supervised iff j + k <= rollout_len (Eq. 4); unused blocks get seq = -1;
+ *   ctx_len   (nullable) - rollout features in the block's context: j - 1 (0 for primary);
+ *   anchor_tok (nullable) - corpus_anchor_tok[t] for a primary block, the rollout token y*_j
+ *             = rollout_tok[(s*P + p)*K + j - 1] for a secondary one, -1 when not given.
+ */
+int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* valid_anchors,
+                   const int32_t* rollout_len, const int32_t* offsets, const int32_t* rollout_tok,
+                   const int32_t* corpus_anchor_tok, int32_t* seq, int32_t* pos,
+                   int32_t* valid_len, int32_t* ctx_len, int32_t* anchor_tok, void* stream);
+
 /* Workspace bytes alr_slot_loss_fwd needs for `p` (0 on invalid params). */
 size_t alr_fwd_workspace_size(const alr_params* p);
 

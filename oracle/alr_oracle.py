@@ -335,3 +335,54 @@ def top_k_logit_grad(z_d, idx, prob, tail, weight, lam, weight_sum=None):
     G = q * beta[:, None]
     G[rows, idx] = q[rows, idx] - _f64(prob)
     return (lam * weight / wsum)[:, None] * G
+
+
+# ----------------------------------------------------------------------------------------
+# IRA block construction (Sec. 3.2, In-rollout anchors; Eq. 4; App. A)
+# ----------------------------------------------------------------------------------------
+def ira_blocks(valid_anchors, rollout_len, offsets, K, max_blocks=128, rollout_tok=None,
+               corpus_anchor_tok=None):
+    """Block plan of one batch of S samples.
+
+    Sample s has v_s valid anchor positions and keeps m_s = min(v_s, max_blocks) blocks: the
+    first ceil(m/2) are primary (they run the target rollout), the next floor(m/2) secondary;
+    slots past m are unused.  Secondary block i sits in primary block i's rollout at offset
+    j = offsets[s, i] in {2..K-1}.  Primary block p's stored rollout holds rollout_len[s, p]
+    label rows (K, or fewer after early termination).
+
+    Per block (s, b), with P = max_blocks - max_blocks // 2 primary slots per sample, the
+    gather of label rows from the primary label buffer viewed as [S * P, K, d]:
+      primary p:      seq = s*P + p, pos = 0, valid_len = rollout_len[s, p]
+      secondary i:    seq = s*P + i, pos = j, valid_len = rollout_len[s, i]
+      unused:         seq = -1 (every row invalid)
+    so row k of a secondary block reads primary row j + k - 1 and is supervised iff
+    j + k <= rollout_len (Eq. 4's 1[j + k <= K] with early termination masked, Sec. 3.2).
+    anchor_tok: the corpus token at the anchor (primary) or the rollout token y*_j (secondary);
+    ctx_len: rollout features of y*_1..y*_{j-1} in the secondary context (0 for primaries).
+    """
+    S = len(valid_anchors)
+    P = max_blocks - max_blocks // 2
+    seq = np.full((S, max_blocks), -1, dtype=np.int64)
+    pos = np.zeros((S, max_blocks), dtype=np.int64)
+    vlen = np.zeros((S, max_blocks), dtype=np.int64)
+    ctx = np.zeros((S, max_blocks), dtype=np.int64)
+    tok = np.full((S, max_blocks), -1, dtype=np.int64)
+    for s in range(S):
+        m = min(int(valid_anchors[s]), max_blocks)
+        n_prim = (m + 1) // 2
+        for b in range(m):
+            if b < n_prim:
+                p, j = b, 0
+            else:
+                p, j = b - n_prim, int(offsets[s][b - n_prim])
+                if j < 1 or j > K - 1:
+                    continue
+            seq[s, b] = s * P + p
+            pos[s, b] = j
+            vlen[s, b] = int(rollout_len[s][p])
+            ctx[s, b] = max(j - 1, 0)
+            if j == 0 and corpus_anchor_tok is not None:
+                tok[s, b] = int(corpus_anchor_tok[s][b])
+            if j > 0 and rollout_tok is not None:
+                tok[s, b] = int(rollout_tok[s][p][j - 1])      # y*_j is rollout step j
+    return dict(seq=seq, pos=pos, valid_len=vlen, ctx_len=ctx, anchor_tok=tok)

@@ -78,6 +78,8 @@ SIGNATURES = {
                                      _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_topk_loss_bwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_ira_blocks": (_c_int, [_c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                _c_p, _c_p, _c_p, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
     "alr_erase_weights": (_c_int, [_c_p, _c_p, _c_p, _c_p, _c_i32, _c_i32, _c_f, _c_i32, _c_p,
                                    _c_p]),
@@ -256,6 +258,16 @@ def alr_topk_loss_bwd(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum
                                    _ptr(top_prob), _ptr(tail), _ptr(weight), _ptr(weight_sum),
                                    _ptr(lse_d), _ptr(tail_q), _ptr(dHd), _ptr(dW),
                                    _ptr(workspace), _nbytes(workspace), _stream(stream)))
+
+
+def alr_ira_blocks(K, max_blocks, valid_anchors, rollout_len, offsets, out: dict,
+                   rollout_tok=None, corpus_anchor_tok=None, stream=None):
+    """out: seq, pos, valid_len (int32 [S*max_blocks]); optional ctx_len, anchor_tok."""
+    _check(lib().alr_ira_blocks(valid_anchors.numel(), K, max_blocks, _ptr(valid_anchors),
+                                _ptr(rollout_len), _ptr(offsets), _ptr(rollout_tok),
+                                _ptr(corpus_anchor_tok), _ptr(out["seq"]), _ptr(out["pos"]),
+                                _ptr(out["valid_len"]), _ptr(out.get("ctx_len")),
+                                _ptr(out.get("anchor_tok")), _stream(stream)))
 
 
 def alr_accept_len(argmax_d, argmax_t, B, acc_len, hist=None, active=None, stream=None):

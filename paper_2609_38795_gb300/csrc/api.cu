@@ -672,6 +672,27 @@ int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const 
   return head_grads_impl(p, Hd, W, G, dHd, dW, ws, lay, info, s);
 }
 
+int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* valid_anchors,
+                   const int32_t* rollout_len, const int32_t* offsets, const int32_t* rollout_tok,
+                   const int32_t* corpus_anchor_tok, int32_t* seq, int32_t* pos,
+                   int32_t* valid_len, int32_t* ctx_len, int32_t* anchor_tok, void* stream) {
+  if (S < 0 || K < 2 || max_blocks < 1)
+    return fail(ALR_ERR_INVALID_ARG, "bad sizes S=%d K=%d max_blocks=%d", S, K, max_blocks);
+  if (S == 0) return ALR_OK;
+  if (valid_anchors == nullptr || rollout_len == nullptr || seq == nullptr || pos == nullptr ||
+      valid_len == nullptr || (max_blocks > 1 && offsets == nullptr))
+    return fail(ALR_ERR_INVALID_ARG,
+                "valid_anchors, rollout_len, offsets, seq, pos and valid_len must be non-NULL");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  cudaError_t e = alr::launch_ira_blocks(S, K, max_blocks, valid_anchors, rollout_len, offsets,
+                                         rollout_tok, corpus_anchor_tok, seq, pos, valid_len,
+                                         ctx_len, anchor_tok, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "IRA block plan launch");
+  return ALR_OK;
+}
+
 int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,
                    int32_t A, int32_t B, int32_t* acc_len, int64_t* hist, void* stream) {
   if (A < 0 || B < 1 || B > 32) return fail(ALR_ERR_INVALID_ARG, "bad sizes A=%d B=%d", A, B);

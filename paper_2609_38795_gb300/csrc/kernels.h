@@ -132,6 +132,12 @@ cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,
                                  const int32_t* argmax_t, const float* row_mask, int A, int B,
                                  float gamma, int hard, float* weight, cudaStream_t s);
 
+cudaError_t launch_ira_blocks(int S, int K, int max_blocks, const int32_t* valid_anchors,
+                              const int32_t* rollout_len, const int32_t* offsets,
+                              const int32_t* rollout_tok, const int32_t* corpus_anchor_tok,
+                              int32_t* seq, int32_t* pos, int32_t* vlen, int32_t* ctx_len,
+                              int32_t* anchor_tok, cudaStream_t s);
+
 // out[c, r] = in[r, c] for an fp32 [R, C] matrix; out rows are ld_out elements apart.
 cudaError_t launch_transpose32(const float* in, float* out, int R, int C, int ld_out,
                                cudaStream_t s);

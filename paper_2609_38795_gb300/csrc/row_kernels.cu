@@ -404,6 +404,52 @@ __global__ void __launch_bounds__(256) topk_combine_kernel(
   }
 }
 
+// ------------------------------------------------------------- IRA block plan ---
+// One thread per block slot (s, b): sample s keeps m = min(v_s, max_blocks) blocks, the
+// first ceil(m/2) primary, the next floor(m/2) secondary (Sec. 3.2); secondary i sits in
+// primary i's rollout at offset j.  Emits the label-row gather (seq, pos, valid_len) over
+// the primary label buffer [S * P, K, d], the anchor token and the rollout context length.
+__global__ void __launch_bounds__(256) ira_blocks_kernel(
+    int S, int K, int max_blocks, const int32_t* __restrict__ valid_anchors,
+    const int32_t* __restrict__ rollout_len, const int32_t* __restrict__ offsets,
+    const int32_t* __restrict__ rollout_tok, const int32_t* __restrict__ corpus_anchor_tok,
+    int32_t* __restrict__ seq, int32_t* __restrict__ pos, int32_t* __restrict__ vlen,
+    int32_t* __restrict__ ctx_len, int32_t* __restrict__ anchor_tok) {
+  const long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= (long long)S * max_blocks) return;
+  const int s = int(t / max_blocks), b = int(t - (long long)s * max_blocks);
+  const int P = max_blocks - max_blocks / 2, Q = max_blocks / 2;
+  const int m = max(0, min(valid_anchors[s], max_blocks));
+  const int n_prim = (m + 1) / 2;
+  int p = -1, j = 0;
+  if (b < n_prim) {
+    p = b;
+  } else if (b < m) {
+    p = b - n_prim;
+    j = offsets[size_t(s) * Q + p];
+    if (j < 1 || j > K - 1) p = -1;   // an offset outside the rollout leaves the block unused
+  }
+  if (p < 0) {
+    seq[t] = -1;
+    pos[t] = 0;
+    vlen[t] = 0;
+    if (ctx_len) ctx_len[t] = 0;
+    if (anchor_tok) anchor_tok[t] = -1;
+    return;
+  }
+  const size_t prim = size_t(s) * P + p;
+  seq[t] = int(prim);
+  pos[t] = j;
+  vlen[t] = rollout_len[prim];
+  if (ctx_len) ctx_len[t] = j > 0 ? j - 1 : 0;
+  if (anchor_tok) {
+    int tok = -1;
+    if (j == 0 && corpus_anchor_tok) tok = corpus_anchor_tok[t];
+    if (j > 0 && rollout_tok) tok = rollout_tok[prim * K + (j - 1)];   // y*_j
+    anchor_tok[t] = tok;
+  }
+}
+
 // ------------------------------------------------------------------ transpose ---
 // out[c * ld_out + r] = in[r * C + c] for 32-bit elements, 32 x 32 tiles through shared memory.
 __global__ void __launch_bounds__(256) transpose32_kernel(const float* __restrict__ in,
@@ -423,6 +469,18 @@ __global__ void __launch_bounds__(256) transpose32_kernel(const float* __restric
 }
 
 }  // namespace
+
+cudaError_t launch_ira_blocks(int S, int K, int max_blocks, const int32_t* valid_anchors,
+                              const int32_t* rollout_len, const int32_t* offsets,
+                              const int32_t* rollout_tok, const int32_t* corpus_anchor_tok,
+                              int32_t* seq, int32_t* pos, int32_t* vlen, int32_t* ctx_len,
+                              int32_t* anchor_tok, cudaStream_t s) {
+  const long long n = (long long)S * max_blocks;
+  ira_blocks_kernel<<<unsigned((n + 255) / 256), 256, 0, s>>>(
+      S, K, max_blocks, valid_anchors, rollout_len, offsets, rollout_tok, corpus_anchor_tok, seq,
+      pos, vlen, ctx_len, anchor_tok);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_transpose32(const float* in, float* out, int R, int C, int ld_out,
                                cudaStream_t s) {

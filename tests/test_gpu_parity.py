@@ -233,3 +233,41 @@ def test_erase_weights_kernel(hard):
                           argmax_t=am_t.numpy(), hard=bool(hard))
     ref = np.tile(orc.slot_envelope(B, gamma), A) * mask.double().numpy() * gate
     np.testing.assert_allclose(P.np64(w), ref, rtol=1e-5, atol=1e-7)
+
+
+# ------------------------------------------------------------- IRA block plan (f3) ---
+def test_ira_block_plan_bit_exact_and_gather():
+    """The device block plan equals the oracle's (integers, bit for bit), including m odd /
+    even, v = 0, v > 128, an early-terminated rollout and out-of-range offsets; the plan then
+    drives the gather of secondary-block label rows from the primary label buffer."""
+    K, max_b, d = 15, 128, 64
+    P_ = max_b - max_b // 2
+    g = torch.Generator().manual_seed(12)
+    valid = torch.tensor([0, 1, 2, 7, 128, 300, 65], dtype=torch.int32)
+    S = len(valid)
+    offsets = torch.randint(2, K, (S, max_b // 2), generator=g, dtype=torch.int32)
+    offsets[6, 3] = 0                                     # outside the rollout: unused block
+    offsets[6, 4] = K
+    rlen = torch.full((S, P_), K, dtype=torch.int32)
+    rlen[3, 1] = 9
+    roll_tok = torch.randint(0, 1000, (S, P_, K), generator=g, dtype=torch.int32)
+    corp_tok = torch.randint(0, 1000, (S, max_b), generator=g, dtype=torch.int32)
+    out = {k: torch.full((S * max_b,), -9, dtype=torch.int32, device="cuda")
+           for k in ("seq", "pos", "valid_len", "ctx_len", "anchor_tok")}
+    alr.alr_ira_blocks(K, max_b, valid.cuda(), rlen.cuda(), offsets.cuda(), out,
+                       rollout_tok=roll_tok.cuda(), corpus_anchor_tok=corp_tok.cuda())
+    ref = orc.ira_blocks(valid.numpy(), rlen.numpy(), offsets.numpy(), K, max_b,
+                         rollout_tok=roll_tok.numpy(), corpus_anchor_tok=corp_tok.numpy())
+    for k in out:
+        assert np.array_equal(P.npi(out[k]), ref[k].reshape(-1)), k
+    # gather the K label rows of every block from a primary label buffer [S*P, K, d]
+    lab = torch.randn(S * P_, K, d, generator=g).to(torch.bfloat16)
+    rows = torch.empty(S * max_b * K, d, dtype=torch.bfloat16, device="cuda")
+    valid_rows = torch.empty(S * max_b * K, device="cuda")
+    alr.alr_gather_ira_blocks(lab.cuda(), out["seq"], out["pos"], K, rows, valid_rows,
+                              valid_len=out["valid_len"])
+    g_ref, v_ref = orc.gather_ira_blocks(lab.float().numpy(), ref["seq"].reshape(-1),
+                                         ref["pos"].reshape(-1), K,
+                                         valid_len=ref["valid_len"].reshape(-1))
+    assert np.array_equal(rows.float().cpu().numpy(), g_ref)
+    assert np.array_equal(valid_rows.cpu().numpy(), v_ref)

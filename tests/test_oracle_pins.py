@@ -300,3 +300,41 @@ def test_gather_index_by_index_and_secondary_block_mask():
                                      valid_len=np.array([K]))
         assert v.tolist() == [1.0 if j + k <= K else 0.0 for k in range(1, K + 1)]
         np.testing.assert_array_equal(o[: K - j], prim[1, j:K])
+
+
+# ------------------------------------------------------------- IRA block plan (Eq. 4) ---
+def test_ira_block_split_and_inheritance():
+    """ceil(m/2) primary and floor(m/2) secondary blocks with m = min(v, 128); a secondary at
+    offset j supervises exactly the slots k with j + k <= K (Eq. 4), reading primary row
+    j + k - 1; its anchor token is y*_j and its context holds j - 1 rollout features."""
+    K, max_b = 15, 128
+    P = max_b // 2
+    rng = np.random.default_rng(5)
+    valid = np.array([0, 1, 2, 7, 128, 300])
+    offsets = rng.integers(2, K, size=(len(valid), P))
+    rlen = np.full((len(valid), P), K)
+    rlen[3, 1] = 9                                        # an early-terminated rollout
+    roll_tok = rng.integers(0, 1000, size=(len(valid), P, K))
+    corp_tok = rng.integers(0, 1000, size=(len(valid), max_b))
+    out = orc.ira_blocks(valid, rlen, offsets, K, max_b, rollout_tok=roll_tok,
+                         corpus_anchor_tok=corp_tok)
+    for s, v in enumerate(valid):
+        m = min(v, max_b)
+        kinds = ["P" if b < (m + 1) // 2 else ("S" if b < m else "-") for b in range(max_b)]
+        assert kinds.count("P") == -(-m // 2) and kinds.count("S") == m // 2
+        for b, kind in enumerate(kinds):
+            if kind == "-":
+                assert out["seq"][s, b] == -1
+                continue
+            p = b if kind == "P" else b - (m + 1) // 2
+            assert out["seq"][s, b] == s * P + p
+            j = 0 if kind == "P" else offsets[s, p]
+            assert out["pos"][s, b] == j and out["valid_len"][s, b] == rlen[s, p]
+            assert out["ctx_len"][s, b] == max(j - 1, 0)
+            assert out["anchor_tok"][s, b] == (corp_tok[s, b] if kind == "P" else roll_tok[s, p, j - 1])
+            # supervised slots through the gather's validity rule
+            lab = np.arange(len(valid) * P * K, dtype=np.float32).reshape(len(valid) * P, K, 1)
+            _, rv = orc.gather_ira_blocks(lab, out["seq"][s, b:b + 1],
+                                          out["pos"][s, b:b + 1], K,
+                                          valid_len=out["valid_len"][s, b:b + 1])
+            assert rv.tolist() == [1.0 if j + k <= rlen[s, p] else 0.0 for k in range(1, K + 1)]
