@@ -5,8 +5,10 @@ One step = the whole path over one batch of the 8B-text workload (d=4096, V=1519
 2048 anchors = 32768 slot rows; seeded synthetic inputs, rollout feature buffer of 16
 sequences x 4096 positions):
     IRA gather of the target hidden rows  ->  fused forward (logits, online LSE, soft CE,
-    greedy argmaxes, slot weights, Eq. 1)  ->  accepted length  ->  logit gradient G
-    (recomputed tiles)  ->  dH_d = G W^T  ->  dW += H_d^T G.
+    greedy argmaxes, slot weights, Eq. 1; both logit matrices kept in fp16)  ->  accepted
+    length  ->  logit gradient G from the kept logits  ->  dH_d = G W^T  ->  dW += H_d^T G.
+The step that recomputes the logits in the backward instead of keeping them is timed beside
+it (`recompute`).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
 
@@ -46,6 +48,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-anchors", type=int, default=1)
+    ap.add_argument("--no-recompute", action="store_true",
+                    help="skip the measurement of the step that recomputes the logits")
     ap.add_argument("--no-topk", action="store_true",
                     help="skip the compact-label (top-8 + tail) step measurement")
     ap.add_argument("--anchors", type=int, default=0,
@@ -256,17 +260,21 @@ def make_inputs(wl, sigma, device, seed):
 
 
 class Step:
-    """Buffers and the sequence of C-ABI calls of one step."""
+    """Buffers and the sequence of C-ABI calls of one step.  keep: the forward keeps both
+    logit matrices (fp16) and G is computed from them in place of z_d; otherwise G is
+    computed by recomputing both head products."""
     N_PHASES = 6
     PHASES = ["gather", "fwd", "accept_len", "logit_grad", "dH_gemm", "dW_gemm"]
     KERNELS_PER_STEP = 8   # gather, fwd (loss, combine, finalize), accept, logit grad, dH, dW
 
-    def __init__(self, wl, inputs, device):
+    def __init__(self, wl, inputs, device, keep=True):
         import torch
         from paper_2609_38795_gb300 import alr
-        self.alr, self.wl, self.x = alr, wl, inputs
-        self.sl = alr.SlotLoss(wl.N, wl.d, wl.V, wl.B, dtype=torch.bfloat16, device=device)
-        self.G = torch.empty(wl.N, wl.V, dtype=torch.bfloat16, device=device)
+        self.alr, self.wl, self.x, self.keep = alr, wl, inputs, keep
+        self.sl = alr.SlotLoss(wl.N, wl.d, wl.V, wl.B, dtype=torch.bfloat16, device=device,
+                               keep_logits=keep)
+        self.G = (self.sl.G if keep else
+                  torch.empty(wl.N, wl.V, dtype=torch.bfloat16, device=device))
         self.dH = torch.empty(wl.N, wl.d, dtype=torch.float32, device=device)
         self.dW = torch.zeros(wl.d, wl.V, dtype=torch.float32, device=device)
 
@@ -281,8 +289,12 @@ class Step:
         sl.accept(active=x["row_valid"])
         rec(3)
         o = sl.out
-        alr.alr_logit_grad(sl.params, x["Hd"], x["Ht"], x["W"], o["weight"], o["weight_sum"],
-                           o["lse_d"], o["lse_t"], self.G)
+        if self.keep:
+            alr.alr_logit_grad_from_logits(sl.params, sl.Zd, sl.Zt, o["weight"], o["weight_sum"],
+                                           o["lse_d"], o["lse_t"], self.G)
+        else:
+            alr.alr_logit_grad(sl.params, x["Hd"], x["Ht"], x["W"], o["weight"],
+                               o["weight_sum"], o["lse_d"], o["lse_t"], self.G)
         rec(4)
         alr.alr_gemm(self.G, x["W"], self.dH, wl.N, wl.d, wl.V)                    # G W^T
         rec(5)
@@ -337,6 +349,34 @@ class TopkStep:
         rec(5)
         alr.alr_gemm(x["Hd"], s.G, s.dW, wl.d, wl.V, wl.N, a_mn=True, b_mn=True, accumulate=True)
         rec(6)
+
+
+def time_recompute(wl, x, device, K, warmup):
+    """The step whose backward recomputes both head products instead of reading kept logits
+    (12 NdV tensor flops, no logit storage)."""
+    import torch
+    st = Step(wl, x, device, keep=False)
+    for _ in range(warmup):
+        st.run()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(K)]
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for k in range(K):
+        st.run(ev[k])
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / K
+    NdV = wl.N * wl.d * wl.V
+    phase = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
+             for i, p in enumerate(Step.PHASES)}
+    out = {"what": "same step, logits recomputed by the backward (nothing kept)",
+           "ms_per_step": ms, "rows_per_s": wl.N / (ms / 1e3),
+           "executed_tflops_12NdV": 12 * NdV / (ms / 1e3) / 1e12, "phase_ms": phase,
+           "gpu_launches": Step.KERNELS_PER_STEP * K, "loss": st.sl.out["loss_total"].item()}
+    del st
+    torch.cuda.empty_cache()
+    return out
 
 
 def time_topk(step, K, warmup):
@@ -454,6 +494,8 @@ def run_gpu(args, rank, world, local_rank):
 
     gather = gather_bandwidth(device) if rank == 0 else None
     topk = time_topk(step, K, args.warmup) if (rank == 0 and not args.no_topk) else None
+    recompute = (time_recompute(wl, x, device, K, args.warmup)
+                 if (rank == 0 and not args.no_recompute) else None)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -469,10 +511,11 @@ def run_gpu(args, rank, world, local_rank):
     NdV = wl.N * wl.d * wl.V
     ms_step = total_ms / K
     rows_per_s = job_rows_per_s(world, wl.N, K, total_ms)
-    exec_tf = 12 * NdV / (ms_step / 1e3) / 1e12
     algo_tf = 8 * NdV / (ms_step / 1e3) / 1e12
-    # dominant kernel by measured time; its algorithmic flops per launch
-    flops = {"fwd": 4 * NdV, "logit_grad": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
+    # dominant kernel by measured time (the tensor-core phases); its flops per launch
+    flops = {"fwd": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
+    # the logit gradient from kept logits streams z_d, z_t (fp16) in and G (bf16) out
+    g_bytes = 6 * wl.N * wl.V
     dom = max(flops, key=lambda p: phase_ms[p])
     achieved = flops[dom] / (phase_ms[dom] / 1e3) / 1e12
     out = {
@@ -482,9 +525,9 @@ def run_gpu(args, rank, world, local_rank):
         "config": {"workload": f"{WORKLOAD}{' PROFILING SUBSET' if args.anchors else ''}: d={wl.d} V={wl.V} B={wl.B} A={wl.A} rows={wl.N} "
                                f"sigma={args.sigma} feature buffer {wl.S}x{wl.L}",
                    "global_batch_rows": world * wl.N, "l2": "inputs larger than L2 "
-                   "(W 1.24 GB, H 268 MB each, G 10 GB)", "parallelism": f"replicas{world}"},
-        "tensor_tflops": {"executed_12NdV": exec_tf, "algorithmic_8NdV": algo_tf,
-                          "pct_peak_executed": exec_tf / pk["bf16"],
+                   "(W 1.24 GB, H 268 MB each, kept logits 2 x 10 GB)", "parallelism": f"replicas{world}"},
+        "tensor_tflops": {"executed_8NdV": algo_tf, "algorithmic_8NdV": algo_tf,
+                          "pct_peak_executed": algo_tf / pk["bf16"],
                           "pct_peak_algorithmic": algo_tf / pk["bf16"],
                           "peak_tflops": pk["bf16"], "peak_source": pk["source"]},
         "phase_ms": phase_ms,
@@ -494,6 +537,9 @@ def run_gpu(args, rank, world, local_rank):
                      "frac_of_burst_peak": achieved / pk["bf16"], "traffic": kernel_traffic(dom),
                      "peak_note": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
                      "flops_per_launch": flops[dom]},
+        "logit_grad_hbm": {"bytes": g_bytes, "GB/s": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9,
+                           "frac_of_hbm": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9 / pk["hbm"]},
+        "recompute": recompute,
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
         "compact_labels": topk,

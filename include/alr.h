@@ -224,6 +224,52 @@ int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const vo
                    const float* lse_t, void* G, void* workspace, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------------------
+ * Kept logits: the same loss with the logits stored by the forward instead of recomputed by
+ * the backward.  The forward's two head products are the path's dominant cost; keeping their
+ * results costs 2 * N * V logit elements of device memory (fp16 for bf16 inputs: 2 x 9.96 GB
+ * at N = 32768, V = 151936) and spares the backward those two products.  The gradient is the
+ * one of Eq. 1 with respect to z_d, as in alr_slot_loss_bwd.
+ * ------------------------------------------------------------------------------------- */
+
+/*
+ * alr_slot_loss_fwd, which also writes the logits z_d = H_d W and z_t = H_t W:
+ *   Zd, Zt  [N, V] row-major, fp16 for ALR_BF16 inputs (rounded to nearest from the fp32
+ *           accumulators; |z| must stay below 65504, the fp16 range), fp32 for ALR_F32 inputs;
+ *           caller-owned, 16-byte aligned, not overlapping any input or output.
+ * Every other argument, output and error is that of alr_slot_loss_fwd (same workspace size),
+ * and the forward outputs are bit-identical to it.
+ */
+int alr_slot_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* Ht,
+                                  const void* W, const float* row_mask, const int32_t* corpus_tok,
+                                  void* Zd, void* Zt, const alr_fwd_outputs* out, void* workspace,
+                                  size_t ws_bytes, void* stream);
+
+/*
+ * G[r, v] = lambda * omega_r / sum omega * (exp(Zd[r, v] - lse_d[r]) - exp(Zt[r, v] - lse_t[r]))
+ * from kept logits (element types as in alr_slot_loss_fwd_keep_logits) and the forward's
+ * weight, weight_sum, lse_d, lse_t; G [N, V] has the element type of p->dtype (bf16 / fp32).
+ * G may be Zd itself (the gradient then overwrites z_d in place); it must not otherwise
+ * overlap Zd or Zt.  Rows with omega_r = 0 (or sum omega = 0) get G = 0.  No workspace.
+ */
+int alr_logit_grad_from_logits(const alr_params* p, const void* Zd, const void* Zt,
+                               const float* weight, const float* weight_sum, const float* lse_d,
+                               const float* lse_t, void* G, void* stream);
+
+/* Workspace bytes alr_slot_loss_bwd_from_logits needs (0 for bf16; G^T and H_d^T for fp32). */
+size_t alr_bwd_from_logits_workspace_size(const alr_params* p);
+
+/*
+ * Backward pass from kept logits: alr_logit_grad_from_logits into G (caller-owned [N, V],
+ * may be Zd), then dH_d = G W^T (overwrites dHd [N, d] fp32) and, when dW is given,
+ * dW += H_d^T G (dW [d, V] fp32).  Errors as in alr_slot_loss_bwd.
+ */
+int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
+                                  const void* Zd, const void* Zt, const float* weight,
+                                  const float* weight_sum, const float* lse_d, const float* lse_t,
+                                  void* G, float* dHd, float* dW, void* workspace,
+                                  size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------------
  * Compact labels: the target's top-k probabilities plus a tail bin.
  *
  * The paper's loss l evaluates soft cross-entropy against the target distribution restricted

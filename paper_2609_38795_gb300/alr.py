@@ -68,6 +68,15 @@ SIGNATURES = {
     "alr_logit_grad_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_logit_grad": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_slot_loss_fwd_keep_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_p, _c_p,
+                                               ctypes.POINTER(AlrFwdOutputs), _c_p, _c_sz, _c_p]),
+    "alr_logit_grad_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
+                                            _c_p, _c_p, _c_p, _c_p]),
+    "alr_bwd_from_logits_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
+    "alr_slot_loss_bwd_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                               _c_sz, _c_p]),
     "alr_readout_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_label_readout": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
@@ -217,6 +226,39 @@ def _nbytes(ws):
     return 0 if ws is None else ws.numel() * ws.element_size()
 
 
+def logits_dtype(t_dtype):
+    """Element type of the kept logits for inputs of type t_dtype."""
+    return torch.float16 if t_dtype == torch.bfloat16 else torch.float32
+
+
+def alr_slot_loss_fwd_keep_logits(params, Hd, Ht, W, Zd, Zt, out: dict, workspace, row_mask=None,
+                                  corpus_tok=None, stream=None):
+    o = AlrFwdOutputs(**{f: _ptr(out.get(f)) for f in _FWD_FIELDS})
+    _check(lib().alr_slot_loss_fwd_keep_logits(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W),
+                                               _ptr(row_mask), _ptr(corpus_tok), _ptr(Zd),
+                                               _ptr(Zt), ctypes.byref(o), _ptr(workspace),
+                                               _nbytes(workspace), _stream(stream)))
+
+
+def alr_logit_grad_from_logits(params, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, stream=None):
+    _check(lib().alr_logit_grad_from_logits(ctypes.byref(params), _ptr(Zd), _ptr(Zt), _ptr(weight),
+                                            _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t), _ptr(G),
+                                            _stream(stream)))
+
+
+def alr_bwd_from_logits_workspace_size(params) -> int:
+    return lib().alr_bwd_from_logits_workspace_size(ctypes.byref(params))
+
+
+def alr_slot_loss_bwd_from_logits(params, Hd, W, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, dHd,
+                                  dW, workspace=None, stream=None):
+    _check(lib().alr_slot_loss_bwd_from_logits(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(Zd),
+                                               _ptr(Zt), _ptr(weight), _ptr(weight_sum),
+                                               _ptr(lse_d), _ptr(lse_t), _ptr(G), _ptr(dHd),
+                                               _ptr(dW), _ptr(workspace), _nbytes(workspace),
+                                               _stream(stream)))
+
+
 def alr_readout_workspace_size(params) -> int:
     return lib().alr_readout_workspace_size(ctypes.byref(params))
 
@@ -291,7 +333,11 @@ def alr_gemm(A, B, C, M, Nc, K, a_mn=False, b_mn=False, accumulate=False, stream
 # ------------------------------------------------------------------ convenience ---
 @dataclass
 class SlotLoss:
-    """Owns the outputs and workspaces of the slot-loss calls for one problem size."""
+    """Owns the outputs and workspaces of the slot-loss calls for one problem size.
+
+    keep_logits: the forward also writes z_d and z_t (``self.Zd``, ``self.Zt``) and the
+    backward computes G from them in place of z_d instead of recomputing the head products;
+    each forward then allows one backward."""
     N: int
     d: int
     V: int
@@ -301,6 +347,7 @@ class SlotLoss:
     lam: float = 1.0
     gamma: float = 2.0
     device: str = "cuda"
+    keep_logits: bool = False
 
     def __post_init__(self):
         self.params = make_params(self.N, self.d, self.V, self.B, self.dtype, self.mode,
@@ -315,6 +362,11 @@ class SlotLoss:
         self.ws_fwd = torch.empty(max(alr_fwd_workspace_size(self.params), 16), dtype=torch.uint8,
                                   device=dev)
         self._ws_bwd = None
+        self.Zd = self.Zt = None
+        if self.keep_logits:
+            lt = logits_dtype(self.dtype)
+            self.Zd = torch.empty(N, self.V, dtype=lt, device=dev)
+            self.Zt = torch.empty(N, self.V, dtype=lt, device=dev)
         self.acc_len = torch.empty(N // self.B, dtype=torch.int32, device=dev)
         self.hist = torch.empty(self.B + 1, dtype=torch.int64, device=dev)
 
@@ -326,8 +378,13 @@ class SlotLoss:
         return self._ws_bwd
 
     def forward(self, Hd, Ht, W, row_mask=None, corpus_tok=None, stream=None):
-        alr_slot_loss_fwd(self.params, Hd, Ht, W, self.out, self.ws_fwd, row_mask=row_mask,
-                          corpus_tok=corpus_tok, stream=stream)
+        if self.keep_logits:
+            alr_slot_loss_fwd_keep_logits(self.params, Hd, Ht, W, self.Zd, self.Zt, self.out,
+                                          self.ws_fwd, row_mask=row_mask, corpus_tok=corpus_tok,
+                                          stream=stream)
+        else:
+            alr_slot_loss_fwd(self.params, Hd, Ht, W, self.out, self.ws_fwd, row_mask=row_mask,
+                              corpus_tok=corpus_tok, stream=stream)
         return self.out
 
     def accept(self, active=None, stream=None):
@@ -337,5 +394,19 @@ class SlotLoss:
 
     def backward(self, Hd, Ht, W, dHd, dW=None, stream=None):
         o = self.out
+        if self.keep_logits:
+            if self._ws_bwd is None:
+                n = alr_bwd_from_logits_workspace_size(self.params)
+                self._ws_bwd = torch.empty(max(n, 16), dtype=torch.uint8, device=self.device)
+            alr_slot_loss_bwd_from_logits(self.params, Hd, W, self.Zd, self.Zt, o["weight"],
+                                          o["weight_sum"], o["lse_d"], o["lse_t"], self.G, dHd,
+                                          dW, self._ws_bwd, stream=stream)
+            return
         alr_slot_loss_bwd(self.params, Hd, Ht, W, o["weight"], o["weight_sum"], o["lse_d"],
                           o["lse_t"], dHd, dW, self.ws_bwd, stream=stream)
+
+    @property
+    def G(self):
+        """With keep_logits, the logit gradient's storage: z_d's buffer, viewed as the input
+        element type."""
+        return None if self.Zd is None else self.Zd.view(self.dtype)

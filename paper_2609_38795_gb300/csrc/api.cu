@@ -87,8 +87,12 @@ size_t elem_size(int dtype) { return dtype == ALR_BF16 ? 2 : 4; }
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Element type of the kept logits for bf16 inputs (tensor maps only; not an ALR_* dtype).
+constexpr int kMapF16 = 2;
+
 // 2-D tiled tensor map (128-byte swizzle unless stated): `inner` contiguous elements per row,
-// `outer` rows `row_bytes` apart; boxes of box_inner x box_outer elements.
+// `outer` rows `row_bytes` apart; boxes of box_inner x box_outer elements.  dtype: ALR_BF16,
+// ALR_F32 or kMapF16.
 int make_map(CUtensorMap* m, const void* ptr, int dtype, uint64_t inner, uint64_t outer,
              uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer,
              CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
@@ -98,7 +102,10 @@ int make_map(CUtensorMap* m, const void* ptr, int dtype, uint64_t inner, uint64_
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = enc(m, dtype == ALR_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+  const CUtensorMapDataType ty = dtype == ALR_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16
+                                 : dtype == kMapF16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                                    : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+  CUresult r = enc(m, ty,
                    2, const_cast<void*>(ptr), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -183,15 +190,17 @@ struct BwdLayout {
   int64_t ld_n;
 };
 
-BwdLayout bwd_layout(const alr_params* p) {
+// with_g = false: the layout of the backward from kept logits, whose G is the caller's and
+// which needs no W^T (G^T and H_d^T only, for fp32).
+BwdLayout bwd_layout(const alr_params* p, bool with_g = true) {
   BwdLayout L{};
   const size_t es = p->dtype == ALR_BF16 ? 2 : 4;
   L.g_off = 0;
-  L.total = round_up(size_t(p->N) * size_t(p->V) * es, 1024);
+  L.total = with_g ? round_up(size_t(p->N) * size_t(p->V) * es, 1024) : 0;
   L.ld_n = (p->N + 3) / 4 * 4;
   if (p->dtype == ALR_F32) {
     L.wt_off = L.total;
-    L.gt_off = L.wt_off + round_up(size_t(p->V) * p->d * 4, 1024);
+    L.gt_off = L.wt_off + (with_g ? round_up(size_t(p->V) * p->d * 4, 1024) : 0);
     L.hdt_off = L.gt_off + round_up(size_t(p->V) * L.ld_n * 4, 1024);
     L.total = L.hdt_off + round_up(size_t(p->d) * L.ld_n * 4, 1024);
   }
@@ -222,6 +231,76 @@ int head_map(CUtensorMap* m, const alr_params* p, const void* W, void* wt, cudaS
                                           p->d, p->V, p->d, s);
   if (e != cudaSuccess) return cuda_fail(e, "head transpose launch");
   return make_map(m, wt, ALR_F32, p->d, p->V, uint64_t(p->d) * 4, kke, ALR_LOSS_BN);
+}
+
+// The full-vocabulary forward; with Zd / Zt given, the fused kernel also writes both logit
+// matrices (kModeFwdKeep).
+int fwd_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
+             const float* row_mask, const int32_t* corpus_tok, void* Zd, void* Zt,
+             const alr_fwd_outputs* out, void* workspace, size_t ws_bytes, void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || Ht == nullptr || W == nullptr || out == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht, W and out must be non-NULL");
+  if (!aligned16(Hd) || !aligned16(Ht) || !aligned16(W))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht and W must be 16-byte aligned");
+  if (out->loss_row == nullptr || out->lse_d == nullptr || out->lse_t == nullptr ||
+      out->argmax_d == nullptr || out->argmax_t == nullptr || out->weight == nullptr ||
+      out->loss_total == nullptr || out->weight_sum == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required forward output pointer is NULL");
+  if (p->mode != ALR_MODE_ALR && corpus_tok == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "the erase modes need corpus_tok");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  const FwdLayout lay = fwd_layout(p, info.sms);
+  if (workspace == nullptr || ws_bytes < lay.total)
+    return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
+                ws_bytes, lay.total);
+  if (!aligned16(workspace)) return fail(ALR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+
+  const int dt = p->dtype;
+  const size_t es = elem_size(dt);
+  const uint32_t kke = k_per_row(dt);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  CUtensorMap m_hd, m_ht, m_w;
+  if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
+  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
+
+  alr::LossArgs args{};
+  args.plan = loss_plan(p, info.sms, false);
+  args.part = reinterpret_cast<float*>(ws + lay.part_off);
+  args.corpus_tok = p->mode != ALR_MODE_ALR ? corpus_tok : nullptr;
+  args.lam = p->lambda;
+  args.withhold_first_stage = g_withhold_next.exchange(0);
+  args.status = alr::device_status_ptr();
+  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+  args.zd_out = Zd;
+  args.zt_out = Zt;
+  // bf16 inputs keep fp16 logits through TMA stores of 16-column x 32-row boxes
+  CUtensorMap m_zd = m_w, m_zt = m_w;
+  if (Zd != nullptr && dt == ALR_BF16) {
+    if ((rc = make_map(&m_zd, Zd, kMapF16, p->V, p->N, p->V * 2, 16, 32,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
+      return rc;
+    if ((rc = make_map(&m_zt, Zt, kMapF16, p->V, p->N, p->V * 2, 16, 32,
+                       CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
+      return rc;
+  }
+  e = alr::launch_loss_kernel(Zd != nullptr ? alr::kModeFwdKeep : alr::kModeFwd, dt, m_hd, m_ht,
+                              m_w, m_zd, m_zt, args, s);
+  if (e != cudaSuccess) return cuda_fail(e, "forward loss kernel launch");
+  double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
+  e = alr::launch_combine(args.plan, args.part, p->mode, p->gamma, row_mask, args.corpus_tok,
+                          out->loss_row, out->ent_row, out->lse_d, out->lse_t, out->argmax_d,
+                          out->argmax_t, out->gap_d, out->gap_t, out->logp_x, out->weight, anchor,
+                          s);
+  if (e != cudaSuccess) return cuda_fail(e, "combine launch");
+  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
+  return ALR_OK;
 }
 
 }  // namespace
@@ -295,56 +374,19 @@ size_t alr_fwd_workspace_size(const alr_params* p) {
 int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
                       const float* row_mask, const int32_t* corpus_tok, const alr_fwd_outputs* out,
                       void* workspace, size_t ws_bytes, void* stream) {
-  int rc = check_params(p);
-  if (rc != ALR_OK) return rc;
-  if (Hd == nullptr || Ht == nullptr || W == nullptr || out == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht, W and out must be non-NULL");
-  if (!aligned16(Hd) || !aligned16(Ht) || !aligned16(W))
-    return fail(ALR_ERR_INVALID_ARG, "Hd, Ht and W must be 16-byte aligned");
-  if (out->loss_row == nullptr || out->lse_d == nullptr || out->lse_t == nullptr ||
-      out->argmax_d == nullptr || out->argmax_t == nullptr || out->weight == nullptr ||
-      out->loss_total == nullptr || out->weight_sum == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "a required forward output pointer is NULL");
-  if (p->mode != ALR_MODE_ALR && corpus_tok == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "the erase modes need corpus_tok");
-  DevInfo info;
-  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  const FwdLayout lay = fwd_layout(p, info.sms);
-  if (workspace == nullptr || ws_bytes < lay.total)
-    return fail(ALR_ERR_INVALID_ARG, "workspace of %zu bytes is smaller than the %zu needed",
-                ws_bytes, lay.total);
-  if (!aligned16(workspace)) return fail(ALR_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+  return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, nullptr, nullptr, out, workspace, ws_bytes,
+                  stream);
+}
 
-  const int dt = p->dtype;
-  const size_t es = elem_size(dt);
-  const uint32_t kke = k_per_row(dt);
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e;
-  CUtensorMap m_hd, m_ht, m_w;
-  if ((rc = make_map(&m_hd, Hd, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_ht, Ht, dt, p->d, p->N, p->d * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
-
-  alr::LossArgs args{};
-  args.plan = loss_plan(p, info.sms, false);
-  args.part = reinterpret_cast<float*>(ws + lay.part_off);
-  args.corpus_tok = p->mode != ALR_MODE_ALR ? corpus_tok : nullptr;
-  args.lam = p->lambda;
-  args.withhold_first_stage = g_withhold_next.exchange(0);
-  args.status = alr::device_status_ptr();
-  if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  e = alr::launch_loss_kernel(alr::kModeFwd, dt, m_hd, m_ht, m_w, m_w, args, s);
-  if (e != cudaSuccess) return cuda_fail(e, "forward loss kernel launch");
-  double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
-  e = alr::launch_combine(args.plan, args.part, p->mode, p->gamma, row_mask, args.corpus_tok,
-                          out->loss_row, out->ent_row, out->lse_d, out->lse_t, out->argmax_d,
-                          out->argmax_t, out->gap_d, out->gap_t, out->logp_x, out->weight, anchor,
-                          s);
-  if (e != cudaSuccess) return cuda_fail(e, "combine launch");
-  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
-  if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
-  return ALR_OK;
+int alr_slot_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* Ht,
+                                  const void* W, const float* row_mask, const int32_t* corpus_tok,
+                                  void* Zd, void* Zt, const alr_fwd_outputs* out, void* workspace,
+                                  size_t ws_bytes, void* stream) {
+  if (Zd == nullptr || Zt == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Zd and Zt must be non-NULL");
+  if (!aligned16(Zd) || !aligned16(Zt))
+    return fail(ALR_ERR_INVALID_ARG, "Zd and Zt must be 16-byte aligned");
+  return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, Zd, Zt, out, workspace, ws_bytes, stream);
 }
 
 size_t alr_bwd_workspace_size(const alr_params* p) {
@@ -413,7 +455,7 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
   cudaError_t e = alr::launch_loss_kernel(topk ? alr::kModeTopkBwd : alr::kModeBwd, dt, m_hd, m_ht,
-                                          m_w, m_gs, args, s);
+                                          m_w, m_gs, m_gs, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "logit-gradient kernel launch");
   return ALR_OK;
 }
@@ -531,6 +573,49 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
   return head_grads_impl(p, Hd, W, G, dHd, dW, ws, lay, info, s);
 }
 
+int alr_logit_grad_from_logits(const alr_params* p, const void* Zd, const void* Zt,
+                               const float* weight, const float* weight_sum, const float* lse_d,
+                               const float* lse_t, void* G, void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Zd == nullptr || Zt == nullptr || G == nullptr || weight == nullptr ||
+      weight_sum == nullptr || lse_d == nullptr || lse_t == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (!aligned16(Zd) || !aligned16(Zt) || !aligned16(G))
+    return fail(ALR_ERR_INVALID_ARG, "Zd, Zt and G must be 16-byte aligned");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  cudaError_t e = alr::launch_logits_grad(p->dtype, Zd, Zt, lse_d, lse_t, weight, weight_sum,
+                                          p->lambda, int(p->N), p->V, G,
+                                          static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "logit-gradient launch");
+  return ALR_OK;
+}
+
+size_t alr_bwd_from_logits_workspace_size(const alr_params* p) {
+  if (check_params(p) != ALR_OK) return 0;
+  return bwd_layout(p, false).total;
+}
+
+int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
+                                  const void* Zd, const void* Zt, const float* weight,
+                                  const float* weight_sum, const float* lse_d, const float* lse_t,
+                                  void* G, float* dHd, float* dW, void* workspace,
+                                  size_t ws_bytes, void* stream) {
+  int rc = alr_logit_grad_from_logits(p, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, stream);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || W == nullptr || dHd == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Hd, W and dHd must be non-NULL");
+  if (!aligned16(Hd) || !aligned16(W) || !aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, W, dHd and dW must be 16-byte aligned");
+  const BwdLayout lay = bwd_layout(p, false);
+  if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  return head_grads_impl(p, Hd, W, G, dHd, dW, static_cast<uint8_t*>(workspace), lay, info,
+                         static_cast<cudaStream_t>(stream));
+}
+
 size_t alr_readout_workspace_size(const alr_params* p) {
   if (check_params(p) != ALR_OK) return 0;
   DevInfo info;
@@ -567,7 +652,7 @@ int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
   args.corpus_tok = corpus_tok;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_loss_kernel(alr::kModeReadout, dt, m_h, m_h, m_w, m_w, args, s);
+  cudaError_t e = alr::launch_loss_kernel(alr::kModeReadout, dt, m_h, m_h, m_w, m_w, m_w, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "label readout kernel launch");
   e = alr::launch_readout_combine(args.plan, args.part, corpus_tok != nullptr, top_idx, top_prob,
                                   tail, lse_t, argmax_t, gap_t, logp_x, s);
@@ -612,7 +697,7 @@ int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const 
   args.top_idx = top_idx;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_loss_kernel(alr::kModeTopkFwd, dt, m_h, m_h, m_w, m_w, args, s);
+  cudaError_t e = alr::launch_loss_kernel(alr::kModeTopkFwd, dt, m_h, m_h, m_w, m_w, m_w, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "top-k forward kernel launch");
   double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
   e = alr::launch_topk_combine(args.plan, args.part, top_prob, tail, row_mask, weight_in, p->gamma,

@@ -60,7 +60,8 @@ enum LossMode {
   kModeBwd = 1,      // dual GEMM: G = c (q - p)
   kModeReadout = 2,  // single GEMM on H_t: log-sum-exp, top-k, z_t at the corpus token
   kModeTopkFwd = 3,  // single GEMM on H_d: log-sum-exp, top-2, z_d at the label tokens
-  kModeTopkBwd = 4   // single GEMM on H_d: gradient of the top-k + tail soft CE
+  kModeTopkBwd = 4,  // single GEMM on H_d: gradient of the top-k + tail soft CE
+  kModeFwdKeep = 5   // kModeFwd that also writes z_d and z_t to global memory
 };
 
 struct LossArgs {
@@ -79,14 +80,18 @@ struct LossArgs {
   const float* top_prob;      // top-k backward: label probabilities [N, kTopK]
   const float* tail;          // top-k backward: label tail mass [N]
   const float* tail_q;        // top-k backward: drafter mass outside the label tokens [N]
+  void* zd_out;               // kModeFwdKeep: z_d, z_t [N, V] (fp16 for bf16 inputs, else fp32)
+  void* zt_out;
 };
 
 // Fused loss kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
 //   a0: the first hidden-state operand (H_d; H_t for the readout), a1: H_t (dual modes).
-//   g_store: bf16 G [N, V] as 16-column x 32-row boxes without swizzle (gradient modes, bf16).
+//   g_store: bf16 G [N, V] as 16-column x 32-row boxes without swizzle (gradient modes, bf16),
+//            or fp16 z_d [N, V] in the same boxes (kModeFwdKeep, bf16);
+//   g_store2: fp16 z_t [N, V] (kModeFwdKeep, bf16).  Unused maps may be any valid map.
 cudaError_t launch_loss_kernel(int mode, int dtype, const CUtensorMap& a0, const CUtensorMap& a1,
                                const CUtensorMap& w, const CUtensorMap& g_store,
-                               const LossArgs& args, cudaStream_t s);
+                               const CUtensorMap& g_store2, const LossArgs& args, cudaStream_t s);
 
 // Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm.cu).
 struct GemmArgs {
@@ -126,6 +131,11 @@ cudaError_t launch_topk_combine(const LossPlan& plan, const float* part, const f
                                 float gamma, float* loss_row, float* lse_d, float* tail_q,
                                 int32_t* argmax_d, float* gap_d, float* weight,
                                 double* anchor_part, cudaStream_t s);
+// G = lambda omega_r / sum omega (exp(z_d - lse_d) - exp(z_t - lse_t)) from kept logits
+// (fp16 for dtype 0, fp32 for dtype 1) into G [N, V] (bf16 / fp32); G may be zd itself.
+cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const float* lse_d,
+                               const float* lse_t, const float* weight, const float* weight_sum,
+                               float lam, int N, int V, void* G, cudaStream_t s);
 cudaError_t launch_accept_len(const int32_t* am_d, const int32_t* am_t, const float* active,
                               int A, int B, int32_t* acc, int64_t* hist, cudaStream_t s);
 cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,

@@ -2,12 +2,15 @@
 //
 // Every mode computes logit tiles z = H W for a 128-row block of hidden states and a
 // kBN-column tile of the vocabulary head W with tcgen05.mma into tensor memory (fp32
-// accumulators) and consumes them on chip; logits never reach global memory.
+// accumulators) and consumes them on chip; only kModeFwdKeep writes logits to global memory.
 //   kModeFwd     z_d = H_d W and z_t = H_t W (both share every W stage): running per-row
 //                statistics (online max / sum-exp of both sides, the label-weighted sums behind
 //                the soft cross-entropy of Eq. 1, greedy top-2 with lowest-index ties, z_t at
 //                the corpus token), one partial record per row, vocabulary split and 64-column
 //                group;
+//   kModeFwdKeep the same, and both logit tiles are also written to global memory (fp16 for
+//                bf16 inputs, fp32 for fp32 inputs) so that the backward need not recompute
+//                them;
 //   kModeBwd     the same two tiles recomputed: G = lambda omega_r / sum omega (q - p), the
 //                gradient of Eq. 1 with respect to z_d;
 //   kModeReadout z_t only: log-sum-exp and the k most probable tokens (the label a rollout
@@ -24,6 +27,8 @@
 // lane, warps 2.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one row per thread)
 // and the 64 columns [64 g, 64 g + 64) of the tile, g = (w-2)/4, in 16-column sub-chunks.
 // Every pipeline wait is bounded (tc_common.cuh).
+#include <cuda_fp16.h>
+
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -49,8 +54,15 @@ struct Geo {
   static constexpr bool kTf32 = (kElem == 4);
 };
 
-constexpr bool is_dual(int mode) { return mode == kModeFwd || mode == kModeBwd; }
+constexpr bool is_fwd(int mode) { return mode == kModeFwd || mode == kModeFwdKeep; }
+constexpr bool is_dual(int mode) { return is_fwd(mode) || mode == kModeBwd; }
 constexpr bool is_grad(int mode) { return mode == kModeBwd || mode == kModeTopkBwd; }
+// Modes whose epilogue writes 16-bit [N, V] tiles through shared staging and TMA stores: the
+// bf16 gradient (two buffers per warp, double-buffered) and the kept fp16 logits (one buffer
+// per logit matrix).  fp32 outputs are written directly.
+constexpr bool is_staged(int mode, int elem_bytes) {
+  return elem_bytes == 2 && (is_grad(mode) || mode == kModeFwdKeep);
+}
 
 template <int kMode, int kBN, bool kStaged>
 struct Shape {
@@ -242,6 +254,49 @@ ALR_DEV uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
+ALR_DEV uint32_t pack_f16x2(uint32_t a, uint32_t b) {
+  __half2 h = __floats2half2_rn(f32(a), f32(b));
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Keep one warp's 32 x 16 sub-chunk of z_d and z_t, fp16 (bf16 inputs): each lane packs its
+// row into the warp's two staging buffers, then one lane issues a TMA store per matrix (rows
+// past N and columns past V are clipped by the tensor maps).  The stores of the previous
+// sub-chunk must have finished reading the buffers first.
+ALR_DEV void keep_logits_staged(const uint32_t (&rd)[16], const uint32_t (&rt)[16],
+                                uint8_t* my_stage, const CUtensorMap* tm_zd,
+                                const CUtensorMap* tm_zt, int v0, int row0, int lane) {
+  if (lane == 0) tma_store_wait_read_all();
+  __syncwarp();
+  uint4* bd = reinterpret_cast<uint4*>(my_stage + lane * 32);
+  uint4* bt = reinterpret_cast<uint4*>(my_stage + kGStageBytes + lane * 32);
+  bd[0] = make_uint4(pack_f16x2(rd[0], rd[1]), pack_f16x2(rd[2], rd[3]), pack_f16x2(rd[4], rd[5]),
+                     pack_f16x2(rd[6], rd[7]));
+  bd[1] = make_uint4(pack_f16x2(rd[8], rd[9]), pack_f16x2(rd[10], rd[11]),
+                     pack_f16x2(rd[12], rd[13]), pack_f16x2(rd[14], rd[15]));
+  bt[0] = make_uint4(pack_f16x2(rt[0], rt[1]), pack_f16x2(rt[2], rt[3]), pack_f16x2(rt[4], rt[5]),
+                     pack_f16x2(rt[6], rt[7]));
+  bt[1] = make_uint4(pack_f16x2(rt[8], rt[9]), pack_f16x2(rt[10], rt[11]),
+                     pack_f16x2(rt[12], rt[13]), pack_f16x2(rt[14], rt[15]));
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    tma_store_2d(tm_zd, my_stage, v0, row0);
+    tma_store_2d(tm_zt, my_stage + kGStageBytes, v0, row0);
+    tma_store_commit();
+  }
+}
+
+// Keep one thread's 16 fp32 logits (fp32 inputs) with direct streaming stores: columns v0..
+// of its row, nv of them valid (8 or 16, as V is a multiple of 8); row * V + v0 is a multiple
+// of 8, so every vector store is aligned.
+ALR_DEV void keep_logits_f32(const uint32_t (&r)[16], void* base, size_t off, int nv) {
+  uint4* p = reinterpret_cast<uint4*>(static_cast<float*>(base) + off);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    if (4 * i < nv) __stcs(p + i, make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]));
+}
+
 // Warp-uniform bounded wait: lane 0 waits, the verdict is broadcast.
 ALR_DEV bool warp_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
   int ok = 1;
@@ -289,15 +344,18 @@ ALR_DEV void store_g(const float (&g)[16], uint8_t* my_stage, uint32_t& n_stores
 
 // kWMN: the head tile is read MN-major straight from W [d, V] (bf16), or K-major from a
 // transposed copy W^T [V, d] (fp32 inputs, whose tf32 products take K-major operands only).
+// tm_g: the bf16 G store map (gradient modes) or the z_d store map (kModeFwdKeep, bf16);
+// tm_g2: the z_t store map (kModeFwdKeep, bf16).
 template <typename Elem, int kMode, bool kWMN, int kBN>
-__global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Elem) == 2>::kThreads, 1)
+__global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem))>::kThreads, 1)
     loss_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,
                      const __grid_constant__ CUtensorMap tm_a1,
                      const __grid_constant__ CUtensorMap tm_w,
-                     const __grid_constant__ CUtensorMap tm_g, const LossArgs args) {
+                     const __grid_constant__ CUtensorMap tm_g,
+                     const __grid_constant__ CUtensorMap tm_g2, const LossArgs args) {
   using G = Geo<Elem>;
   constexpr bool kDual = is_dual(kMode);
-  constexpr bool kStaged = is_grad(kMode) && sizeof(Elem) == 2;
+  constexpr bool kStaged = is_staged(kMode, sizeof(Elem));
   using S = Shape<kMode, kBN, kStaged>;
   constexpr int kStages = S::kStages;
 
@@ -336,6 +394,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Ele
     if (kDual) tma_prefetch_desc(&tm_a1);
     tma_prefetch_desc(&tm_w);
     if (kStaged) tma_prefetch_desc(&tm_g);
+    if (kStaged && kMode == kModeFwdKeep) tma_prefetch_desc(&tm_g2);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
@@ -477,7 +536,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Ele
       const size_t fs = size_t(P.n_parts) * P.N;
 
       // ---- per-row state for this unit ----
-      RowStats st;                       // kModeFwd
+      RowStats st;                       // forward modes
       float m = -INFINITY, s = 0.f;      // single-operand log-sum-exp state
       float best = -INFINITY, sec = -INFINITY, zx = qnan();
       int bidx = 0x7fffffff, x = -1;
@@ -491,8 +550,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Ele
         ti[i] = kMode == kModeReadout ? 0x7fffffff : -1;
         tp[i] = 0.f;
       }
-      if constexpr (kMode == kModeFwd) stats_init(st);
-      if constexpr (kMode == kModeFwd || kMode == kModeReadout)
+      if constexpr (is_fwd(kMode)) stats_init(st);
+      if constexpr (is_fwd(kMode) || kMode == kModeReadout)
         x = (args.corpus_tok != nullptr && row_ok) ? args.corpus_tok[row] : -1;
       if constexpr (kMode == kModeTopkFwd || kMode == kModeTopkBwd) {
         if (row_ok) {
@@ -537,9 +596,18 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Ele
           if (v0 >= P.V) continue;   // warp-uniform: the whole sub-chunk is past the vocabulary
           const int nv = min(kSub, P.V - v0);
 
-          if constexpr (kMode == kModeFwd) {
+          if constexpr (is_fwd(kMode)) {
             if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x);
             else stats_sub<false>(st, r0, r1, v0, nv, x);
+            if constexpr (kMode == kModeFwdKeep) {
+              if constexpr (kStaged) {
+                keep_logits_staged(r0, r1, my_stage, &tm_g, &tm_g2, v0, rb * kBM + q * 32, lane);
+              } else if (row_ok) {
+                const size_t off = size_t(row) * size_t(P.V) + size_t(v0);
+                keep_logits_f32(r0, args.zd_out, off, nv);
+                keep_logits_f32(r1, args.zt_out, off, nv);
+              }
+            }
           } else if constexpr (kMode == kModeReadout || kMode == kModeTopkFwd) {
             float z[16];
             if (nv == kSub) load_masked<true>(z, r0, nv);
@@ -616,7 +684,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Ele
       // ---- per-row partial record at the end of the unit ----
       if (ok && row_ok) {
         float* o = args.part + part * P.N + row;
-        if constexpr (kMode == kModeFwd) {
+        if constexpr (is_fwd(kMode)) {
           o[kPMd * fs] = st.best_d;
           o[kPSd * fs] = st.s_d;
           o[kPMt * fs] = st.best_t;
@@ -665,32 +733,36 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_grad(kMode) && sizeof(Ele
 
 template <typename Elem, int kMode, int kBN>
 cudaError_t launch_impl(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
-                        const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
-  using S = Shape<kMode, kBN, is_grad(kMode) && sizeof(Elem) == 2>;
+                        const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
+                        cudaStream_t s) {
+  using S = Shape<kMode, kBN, is_staged(kMode, sizeof(Elem))>;
   auto kern = loss_gemm_kernel<Elem, kMode, sizeof(Elem) == 2, kBN>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
   if (e != cudaSuccess) return e;
-  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(a0, a1, w, g, args);
+  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(a0, a1, w, g, g2, args);
   return cudaGetLastError();
 }
 
 template <typename Elem, int kMode>
 cudaError_t by_width(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
-                     const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
-  if (args.plan.bn == 128) return launch_impl<Elem, kMode, 128>(a0, a1, w, g, args, s);
-  return launch_impl<Elem, kMode, 256>(a0, a1, w, g, args, s);
+                     const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
+                     cudaStream_t s) {
+  if (args.plan.bn == 128) return launch_impl<Elem, kMode, 128>(a0, a1, w, g, g2, args, s);
+  return launch_impl<Elem, kMode, 256>(a0, a1, w, g, g2, args, s);
 }
 
 template <typename Elem>
 cudaError_t by_mode(int mode, const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
-                    const CUtensorMap& g, const LossArgs& args, cudaStream_t s) {
+                    const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
+                    cudaStream_t s) {
   switch (mode) {
-    case kModeFwd: return by_width<Elem, kModeFwd>(a0, a1, w, g, args, s);
-    case kModeBwd: return by_width<Elem, kModeBwd>(a0, a1, w, g, args, s);
-    case kModeReadout: return by_width<Elem, kModeReadout>(a0, a1, w, g, args, s);
-    case kModeTopkFwd: return by_width<Elem, kModeTopkFwd>(a0, a1, w, g, args, s);
-    case kModeTopkBwd: return by_width<Elem, kModeTopkBwd>(a0, a1, w, g, args, s);
+    case kModeFwd: return by_width<Elem, kModeFwd>(a0, a1, w, g, g2, args, s);
+    case kModeFwdKeep: return by_width<Elem, kModeFwdKeep>(a0, a1, w, g, g2, args, s);
+    case kModeBwd: return by_width<Elem, kModeBwd>(a0, a1, w, g, g2, args, s);
+    case kModeReadout: return by_width<Elem, kModeReadout>(a0, a1, w, g, g2, args, s);
+    case kModeTopkFwd: return by_width<Elem, kModeTopkFwd>(a0, a1, w, g, g2, args, s);
+    case kModeTopkBwd: return by_width<Elem, kModeTopkBwd>(a0, a1, w, g, g2, args, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -699,9 +771,9 @@ cudaError_t by_mode(int mode, const CUtensorMap& a0, const CUtensorMap& a1, cons
 
 cudaError_t launch_loss_kernel(int mode, int dtype, const CUtensorMap& a0, const CUtensorMap& a1,
                                const CUtensorMap& w, const CUtensorMap& g_store,
-                               const LossArgs& args, cudaStream_t s) {
-  if (dtype == 0) return by_mode<__nv_bfloat16>(mode, a0, a1, w, g_store, args, s);
-  return by_mode<float>(mode, a0, a1, w, g_store, args, s);
+                               const CUtensorMap& g_store2, const LossArgs& args, cudaStream_t s) {
+  if (dtype == 0) return by_mode<__nv_bfloat16>(mode, a0, a1, w, g_store, g_store2, args, s);
+  return by_mode<float>(mode, a0, a1, w, g_store, g_store2, args, s);
 }
 
 }  // namespace alr

@@ -1,7 +1,9 @@
 // Row-level kernels of the slot-loss path: the IRA gather, the merge of per-split forward
 // statistics into the per-row loss terms and slot weights, the batch reduction of Eq. 1,
-// the accepted-length statistic and the erase-gate weights.
+// the accepted-length statistic, the erase-gate weights and the logit gradient from logits the
+// forward kept.
 #include <cfloat>
+#include <cuda_fp16.h>
 
 #include "kernels.h"
 #include "tc_common.cuh"
@@ -468,7 +470,123 @@ __global__ void __launch_bounds__(256) transpose32_kernel(const float* __restric
   }
 }
 
+// ------------------------------------------------ logit gradient from kept logits ---
+// G[r, v] = c_r (exp(z_d - lse_d) - exp(z_t - lse_t)) with c_r = lambda omega_r / sum omega:
+// the gradient of Eq. 1 with respect to z_d, from the logits the forward wrote.  One block per
+// row, 8 columns per vector (V is a multiple of 8), kLogitsUnroll vectors of each matrix in
+// flight per thread, held raw until all of them have arrived.  G may be the z_d buffer itself:
+// each element is read before the thread that read it overwrites it, and no other thread
+// touches it.  Masked rows (c_r = 0) read nothing.
+constexpr int kLogitsUnroll = 4;
+
+// 8 kept logits as loaded: fp16 (bf16 inputs) or fp32 (fp32 inputs).
+template <typename Z>
+struct Raw8;
+
+template <>
+struct Raw8<__half> {
+  uint4 u;
+  __device__ __forceinline__ void load(const __half* p) {
+    u = __ldcs(reinterpret_cast<const uint4*>(p));
+  }
+  __device__ __forceinline__ void to_float(float (&v)[8]) const {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[i]));
+      v[2 * i] = f.x;
+      v[2 * i + 1] = f.y;
+    }
+  }
+};
+
+template <>
+struct Raw8<float> {
+  float4 a, b;
+  __device__ __forceinline__ void load(const float* p) {
+    a = __ldcs(reinterpret_cast<const float4*>(p));
+    b = __ldcs(reinterpret_cast<const float4*>(p) + 1);
+  }
+  __device__ __forceinline__ void to_float(float (&v)[8]) const {
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+};
+
+__device__ __forceinline__ uint32_t bf16x2_bits(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ void store8(__nv_bfloat16* p, const float (&g)[8]) {
+  *reinterpret_cast<uint4*>(p) = make_uint4(bf16x2_bits(g[0], g[1]), bf16x2_bits(g[2], g[3]),
+                                            bf16x2_bits(g[4], g[5]), bf16x2_bits(g[6], g[7]));
+}
+
+__device__ __forceinline__ void store8(float* p, const float (&g)[8]) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(g[0], g[1], g[2], g[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(g[4], g[5], g[6], g[7]);
+}
+
+template <typename Z, typename Gt>
+__global__ void __launch_bounds__(256, sizeof(Z) == 2 ? 4 : 2) logits_grad_kernel(const Z* zd, const Z* zt,
+                                                             const float* __restrict__ lse_d,
+                                                             const float* __restrict__ lse_t,
+                                                             const float* __restrict__ weight,
+                                                             const float* __restrict__ weight_sum,
+                                                             float lam, int V, Gt* G) {
+  const int row = blockIdx.x;
+  const float ws = *weight_sum;
+  const float c = ws > 0.f ? lam * weight[row] / ws : 0.f;
+  const size_t base = size_t(row) * size_t(V);
+  const int n8 = V / 8;
+  if (c == 0.f) {
+    const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int i = threadIdx.x; i < n8; i += blockDim.x) store8(G + base + 8 * size_t(i), z);
+    return;
+  }
+  const float ad = -lse_d[row] * kLog2e, at = -lse_t[row] * kLog2e;
+  for (int i0 = threadIdx.x; i0 < n8; i0 += kLogitsUnroll * blockDim.x) {
+    Raw8<Z> a[kLogitsUnroll], b[kLogitsUnroll];
+#pragma unroll
+    for (int u = 0; u < kLogitsUnroll; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n8) {
+        a[u].load(zd + base + 8 * size_t(i));
+        b[u].load(zt + base + 8 * size_t(i));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kLogitsUnroll; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n8) {
+        float x[8], y[8], g[8];
+        a[u].to_float(x);
+        b[u].to_float(y);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          g[j] = c * (ex2(fmaf(x[j], kLog2e, ad)) - ex2(fmaf(y[j], kLog2e, at)));
+        store8(G + base + 8 * size_t(i), g);
+      }
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const float* lse_d,
+                               const float* lse_t, const float* weight, const float* weight_sum,
+                               float lam, int N, int V, void* G, cudaStream_t s) {
+  if (dtype == 0)
+    logits_grad_kernel<__half, __nv_bfloat16><<<N, 256, 0, s>>>(
+        static_cast<const __half*>(zd), static_cast<const __half*>(zt), lse_d, lse_t, weight,
+        weight_sum, lam, V, static_cast<__nv_bfloat16*>(G));
+  else
+    logits_grad_kernel<float, float><<<N, 256, 0, s>>>(
+        static_cast<const float*>(zd), static_cast<const float*>(zt), lse_d, lse_t, weight,
+        weight_sum, lam, V, static_cast<float*>(G));
+  return cudaGetLastError();
+}
 
 cudaError_t launch_ira_blocks(int S, int K, int max_blocks, const int32_t* valid_anchors,
                               const int32_t* rollout_len, const int32_t* offsets,

@@ -42,22 +42,35 @@ def _rows(anchors, B):
 
 
 class Run:
-    """The step bench.py times: gather -> forward -> accepted length -> logit gradient ->
-    dH = G W^T -> dW += H_d^T G, all through the C ABI on the current stream."""
+    """The step bench.py times: gather -> forward keeping the logits -> accepted length ->
+    logit gradient from the kept logits (in place of z_d) -> dH = G W^T -> dW += H_d^T G, all
+    through the C ABI on the current stream.  keep=False: the forward keeps nothing and the
+    logit gradient recomputes the head products instead.  The kept logits of `sample_rows`
+    are copied out before the gradient overwrites z_d."""
 
-    def __init__(self, wl, x, mode=alr.ALR_MODE_ALR, lam=1.0, corpus_tok=None):
+    def __init__(self, wl, x, mode=alr.ALR_MODE_ALR, lam=1.0, corpus_tok=None, keep=True,
+                 sample_rows=None):
         self.wl, self.x = wl, x
         N, d, V, B = wl.N, wl.d, wl.V, wl.B
         x["Ht"] = torch.empty(N, d, dtype=torch.bfloat16, device="cuda")
         x["row_valid"] = torch.empty(N, device="cuda")
         alr.alr_gather_ira_blocks(x["F"], x["seq"], x["pos"], B, x["Ht"], x["row_valid"])
-        self.sl = alr.SlotLoss(N, d, V, B, mode=mode, lam=lam)
+        self.sl = alr.SlotLoss(N, d, V, B, mode=mode, lam=lam, keep_logits=keep)
         self.sl.forward(x["Hd"], x["Ht"], x["W"], row_mask=x["row_valid"], corpus_tok=corpus_tok)
         self.acc, self.hist = self.sl.accept(active=x["row_valid"])
         o = self.sl.out
-        self.G = torch.empty(N, V, dtype=torch.bfloat16, device="cuda")
-        alr.alr_logit_grad(self.sl.params, x["Hd"], x["Ht"], x["W"], o["weight"], o["weight_sum"],
-                           o["lse_d"], o["lse_t"], self.G)
+        self.z_sample = None
+        if keep:
+            if sample_rows is not None:
+                idx = torch.from_numpy(sample_rows).cuda()
+                self.z_sample = (P.np64(self.sl.Zd[idx]), P.np64(self.sl.Zt[idx]))
+            self.G = self.sl.G
+            alr.alr_logit_grad_from_logits(self.sl.params, self.sl.Zd, self.sl.Zt, o["weight"],
+                                           o["weight_sum"], o["lse_d"], o["lse_t"], self.G)
+        else:
+            self.G = torch.empty(N, V, dtype=torch.bfloat16, device="cuda")
+            alr.alr_logit_grad(self.sl.params, x["Hd"], x["Ht"], x["W"], o["weight"],
+                               o["weight_sum"], o["lse_d"], o["lse_t"], self.G)
         self.dH = torch.empty(N, d, device="cuda")
         alr.alr_gemm(self.G, x["W"], self.dH, N, d, V)
         self.dW = torch.zeros(d, V, device="cuda")
@@ -86,6 +99,10 @@ def _check_step(wl, x, run, Ht_ref, valid_ref, Hd64, W64, mode=alr.ALR_MODE_ALR,
     r = orc.slot_loss_forward(Hd64[rows], Ht_ref[rows], W64, B, mode=mode, lam=lam,
                               row_mask=valid_ref[rows], corpus_tok=tok)
     g = P.fwd_to_numpy(run.sl, rows)
+    if run.z_sample is not None:
+        # kept logits: fp16 rounding of the fp32 accumulators (2^-11 relative)
+        for z_g, z_r in zip(run.z_sample, (r["z_d"], r["z_t"])):
+            assert np.all(np.abs(z_g - z_r) <= 2.0 ** -11 * np.abs(z_r) + 1e-4)
     if mode == alr.ALR_MODE_ERASE_HARD:
         # a near-tie target row may flip its greedy token and with it the hard gate of the
         # anchor's later rows: compare the weights of anchors without near-ties only
@@ -125,16 +142,17 @@ def _check_step(wl, x, run, Ht_ref, valid_ref, Hd64, W64, mode=alr.ALR_MODE_ALR,
     return near
 
 
-@pytest.mark.parametrize("sigma", [0.25, 0.5, 1.0])
-def test_text8b_full_batch(sigma):
-    """d=4096, V=151936, B=16, 2048 anchors (32768 rows), feature buffer 16 x 4096."""
+@pytest.mark.parametrize("sigma,keep", [(0.25, True), (0.5, True), (1.0, True), (0.5, False)])
+def test_text8b_full_batch(sigma, keep):
+    """d=4096, V=151936, B=16, 2048 anchors (32768 rows), feature buffer 16 x 4096; the
+    kept-logits step at three noise levels and the recomputing step at one."""
     wl = synthetic.WORKLOADS["text8b"]
     x = synthetic.rollout_batch(wl.d, wl.V, wl.A, wl.B, wl.S, wl.L, sigma, device="cuda", seed=0)
-    run = Run(wl, x)
+    run = Run(wl, x, keep=keep, sample_rows=_rows(_sample_anchors(wl.A), wl.B))
     Ht_ref, valid_ref, Hd64, W64 = _oracle_inputs(wl, x)
     near = _check_step(wl, x, run, Ht_ref, valid_ref, Hd64, W64)
     hist = P.npi(run.hist).tolist()
-    print(f"text8b sigma={sigma}: acc-len histogram {hist}, {near} near-tie sampled rows")
+    print(f"text8b sigma={sigma} keep={keep}: acc-len histogram {hist}, {near} near-tie sampled rows")
 
 
 @pytest.mark.parametrize("mode", [alr.ALR_MODE_ERASE_SOFT, alr.ALR_MODE_ERASE_HARD])
@@ -150,7 +168,7 @@ def test_erase_full_batch(mode):
     tok = rnd.numpy().astype(np.int64)
     tok[rows] = np.where(mask.numpy()[rows], tok[rows], greedy)
     tok_dev = torch.from_numpy(tok.astype(np.int32)).cuda()
-    run = Run(wl, x, mode=mode, corpus_tok=tok_dev)
+    run = Run(wl, x, mode=mode, corpus_tok=tok_dev, sample_rows=rows)
     _check_step(wl, x, run, Ht_ref, valid_ref, Hd64, W64, mode=mode, corpus_tok=tok)
 
 
@@ -159,7 +177,7 @@ def test_vl7b_full_batch_and_gradient_sub_batch():
     full backward (every dH and dW entry) on an 8-anchor sub-batch at full d and V."""
     wl = synthetic.WORKLOADS["vl7b"]
     x = synthetic.rollout_batch(wl.d, wl.V, wl.A, wl.B, wl.S, wl.L, wl.sigma, device="cuda", seed=2)
-    run = Run(wl, x, lam=1.013441)
+    run = Run(wl, x, lam=1.013441, sample_rows=_rows(_sample_anchors(wl.A), wl.B))
     Ht_ref, valid_ref, Hd64, W64 = _oracle_inputs(wl, x)
     _check_step(wl, x, run, Ht_ref, valid_ref, Hd64, W64, lam=1.013441)
     # sub-batch gradient in full, through the composite backward entry point
