@@ -70,6 +70,7 @@ def peaks():
 # ------------------------------------------------------------------ DRAM traffic ---
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "loss_gemm_traffic.json")
 KERNEL_SOURCES = ["paper_2609_38795_gb300/csrc/loss_gemm.cu",
+                  "paper_2609_38795_gb300/csrc/row_kernels.cu",
                   "paper_2609_38795_gb300/csrc/tc_common.cuh",
                   "paper_2609_38795_gb300/csrc/kernels.h"]
 
@@ -84,7 +85,8 @@ def kernel_sources_sha256():
 
 
 def kernel_traffic(phase):
-    """DRAM bytes per full-size launch of a fused loss kernel, from the committed ncu summary,
+    """DRAM bytes per full-size launch of the kernel of a step phase ("fwd": the fused forward
+    keeping the logits; "logit_grad": G from the kept logits), from the committed ncu summary,
     or None when that summary is missing or was taken from other kernel sources."""
     try:
         with open(TRAFFIC_FILE) as f:
@@ -538,7 +540,8 @@ def run_gpu(args, rank, world, local_rank):
                      "peak_note": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
                      "flops_per_launch": flops[dom]},
         "logit_grad_hbm": {"bytes": g_bytes, "GB/s": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9,
-                           "frac_of_hbm": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9 / pk["hbm"]},
+                           "frac_of_hbm": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9 / pk["hbm"],
+                           "traffic": kernel_traffic("logit_grad")},
         "recompute": recompute,
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
