@@ -353,6 +353,14 @@ class TopkStep:
         rec(6)
 
 
+def check_device_status(what):
+    """Raise if a bounded pipeline wait of the library timed out (its kernels then return
+    early and their outputs and timings are void)."""
+    from paper_2609_38795_gb300 import alr
+    if alr.alr_device_status() != alr.ALR_OK:
+        raise RuntimeError(f"{what}: device status: {alr.alr_last_error()}")
+
+
 def time_recompute(wl, x, device, K, warmup):
     """The step whose backward recomputes both head products instead of reading kept logits
     (12 NdV tensor flops, no logit storage)."""
@@ -369,6 +377,7 @@ def time_recompute(wl, x, device, K, warmup):
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / K
+    check_device_status("recomputing step")
     NdV = wl.N * wl.d * wl.V
     phase = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
              for i, p in enumerate(Step.PHASES)}
@@ -395,6 +404,7 @@ def time_topk(step, K, warmup):
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / K
+    check_device_status("compact-label step")
     wl = step.wl
     NdV = wl.N * wl.d * wl.V
     phase = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
@@ -429,8 +439,7 @@ def run_gpu(args, rank, world, local_rank):
     for _ in range(args.warmup):
         step.run()
     torch.cuda.synchronize()
-    if alr.alr_device_status() != alr.ALR_OK:
-        raise RuntimeError("device status: " + alr.alr_last_error())
+    check_device_status("warm-up")
 
     K = args.steps
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(K)]
@@ -452,8 +461,7 @@ def run_gpu(args, rank, world, local_rank):
     total_ms = t_start.elapsed_time(t_stop)
     phase_ms = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
                 for i, p in enumerate(Step.PHASES)}
-    if alr.alr_device_status() != alr.ALR_OK:
-        raise RuntimeError("device status: " + alr.alr_last_error())
+    check_device_status("timed steps")
     acc_hist = step.sl.hist.cpu().tolist()
     loss = step.sl.out["loss_total"].item()
 
@@ -487,6 +495,7 @@ def run_gpu(args, rank, world, local_rank):
         b.record()
         torch.cuda.synchronize()
         e2e_ms = a.elapsed_time(b)
+        check_device_status("end-to-end steps")
         if world > 1:
             dist.barrier()
         e2e = {"ms": e2e_ms, "h2d": h2d, "d2h": d2h}
@@ -501,7 +510,7 @@ def run_gpu(args, rank, world, local_rank):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rps, ts = time_oracle(wl, x, args.cpu_sample_anchors, reps=3)
+        rps, ts = time_oracle(wl, x, args.cpu_sample_anchors, reps=10)
         cpu = {"value": rps, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                "sample": f"{args.cpu_sample_anchors} anchor(s) x {wl.B} rows of the {WORKLOAD} "
                          f"workload, full d={wl.d} and V={wl.V}, fwd+bwd in fp64, "

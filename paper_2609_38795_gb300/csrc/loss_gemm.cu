@@ -78,6 +78,9 @@ struct Shape {
   static constexpr int kFit = (kSmemBudget - 1024 - kCtrlBytes - kStaging) / kStageBytes;
   static constexpr int kStages = kFit < 4 ? kFit : 4;
   static constexpr size_t kSmem = 1024 + size_t(kStages) * kStageBytes + kStaging + kCtrlBytes;
+  // control block: full / empty barrier per stage, full / empty per accumulator buffer, the
+  // drain barrier, the TMEM address and the abort word
+  static_assert((2 * kStages + 2 * kAccBufs + 1) * 8 + 8 <= kCtrlBytes, "control block");
 };
 
 // Unit u -> (row block, vocabulary split).  Units go group by group (group_rows row blocks);
@@ -366,8 +369,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(gstage + S::kStaging);
   uint64_t* empty_bar = full_bar + kStages;
   uint64_t* tfull_bar = empty_bar + kStages;
-  uint64_t* tempty_bar = tfull_bar + 2;
-  uint64_t* drain_bar = tempty_bar + 2;
+  uint64_t* tempty_bar = tfull_bar + S::kAccBufs;
+  uint64_t* drain_bar = tempty_bar + S::kAccBufs;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile int* abort_word = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
