@@ -5,6 +5,7 @@
 #include <atomic>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
@@ -207,6 +208,29 @@ BwdLayout bwd_layout(const alr_params* p, bool with_g = true) {
   return L;
 }
 
+// Form of the bf16 products, chosen by the environment variable ALR_GEMM_FORM:
+//   "mcast"   clusters of two CTAs, each on a 128 x 256 tile, sharing every B tile by TMA
+//             multicast (plain_gemm.cu), the default;
+//   "single"  one CTA per 128 x 256 tile, each loading its own B tiles;
+//   "pair"    CTA pairs with M = 256 products (pair_gemm.cu).
+// The step runs at the GB300's power cap, so the form that moves fewest bytes per product
+// wins: multicast halves the B traffic out of L2 and runs 6 % faster than single CTAs at the
+// same clock and power.  The pair form issues more products per clock but draws more power
+// per product and settles at a clock ~20 % lower.  tf32 products always run on single CTAs.
+enum GemmForm { kGemmSingle = 0, kGemmMcast = 1, kGemmPair = 2 };
+
+GemmForm gemm_form(int dtype) {
+  if (dtype != ALR_BF16) return kGemmSingle;
+  const char* v = getenv("ALR_GEMM_FORM");
+  if (v == nullptr) return kGemmMcast;
+  if (strcmp(v, "single") == 0) return kGemmSingle;
+  if (strcmp(v, "pair") == 0) return kGemmPair;
+  return kGemmMcast;
+}
+
+// Rows of a K-major B box (B columns loaded by one copy).
+uint32_t gemm_b_rows(int dtype) { return gemm_form(dtype) == kGemmSingle ? 256 : 128; }
+
 alr::GemmArgs gemm_plan(int M, int Nc, int K, float* C, int64_t ldc, int sms) {
   alr::GemmArgs g{};
   g.M = M;
@@ -220,6 +244,57 @@ alr::GemmArgs gemm_plan(int M, int Nc, int K, float* C, int64_t ldc, int sms) {
   g.n_tiles = g.n_mb * g.n_nb;
   g.grid = sms < g.n_tiles ? sms : g.n_tiles;
   return g;
+}
+
+// Plan of the pair GEMM: 256 x 256 tiles over `pairs` resident CTA pairs.
+alr::GemmArgs pair_gemm_plan(int M, int Nc, int K, float* C, int64_t ldc, int pairs) {
+  alr::GemmArgs g{};
+  g.M = M;
+  g.Nc = Nc;
+  g.K = K;
+  g.C = C;
+  g.ldc = ldc;
+  g.n_mb = (M + 255) / 256;
+  g.n_nb = (Nc + 255) / 256;
+  g.group_m = g.n_mb < 8 ? g.n_mb : 8;
+  g.n_tiles = g.n_mb * g.n_nb;
+  g.grid = 2 * (pairs < g.n_tiles ? pairs : g.n_tiles);
+  return g;
+}
+
+// C (+)= A B with the operand maps already encoded (B boxes of gemm_b_rows(dt) rows).
+int launch_gemm(int dt, bool a_mn, bool b_mn, bool acc, const CUtensorMap& ma,
+                const CUtensorMap& mb, int M, int Nc, int K, float* C, int64_t ldc, int sms,
+                cudaStream_t s, const char* what) {
+  cudaError_t e;
+  const GemmForm form = gemm_form(dt);
+  if (form == kGemmPair) {
+    const int pairs = alr::pair_gemm_max_pairs();
+    if (pairs < 1) return fail(ALR_ERR_CUDA, "%s: no CTA pair of the GEMM fits on this device", what);
+    alr::GemmArgs g = pair_gemm_plan(M, Nc, K, C, ldc, pairs);
+    g.status = alr::device_status_ptr();
+    if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+    e = alr::launch_pair_gemm(a_mn, b_mn, acc, ma, mb, g, s);
+  } else if (form == kGemmMcast) {
+    const int pairs = alr::plain_gemm_mc_max_pairs();
+    if (pairs < 1) return fail(ALR_ERR_CUDA, "%s: no CTA cluster of the GEMM fits on this device", what);
+    // 128-row blocks in pairs: n_mb counts pairs, raster groups of 8 pairs
+    alr::GemmArgs g = gemm_plan(M, Nc, K, C, ldc, sms);
+    g.n_mb = ((M + 127) / 128 + 1) / 2;
+    g.group_m = g.n_mb < 8 ? g.n_mb : 8;
+    g.n_tiles = g.n_mb * g.n_nb;
+    g.grid = 2 * (pairs < g.n_tiles ? pairs : g.n_tiles);
+    g.status = alr::device_status_ptr();
+    if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+    e = alr::launch_plain_gemm_mc(a_mn, b_mn, acc, ma, mb, g, s);
+  } else {
+    alr::GemmArgs g = gemm_plan(M, Nc, K, C, ldc, sms);
+    g.status = alr::device_status_ptr();
+    if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+    e = alr::launch_plain_gemm(dt, a_mn, b_mn, acc, ma, mb, g, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, what);
+  return ALR_OK;
 }
 
 // Tensor map of the head operand of the fused loss kernels: MN-major tiles straight from
@@ -467,26 +542,24 @@ int head_grads_impl(const alr_params* p, const void* Hd, const void* W, const vo
   const int dt = p->dtype;
   const size_t es = elem_size(dt);
   const uint32_t kke = k_per_row(dt);
-  int* status = alr::device_status_ptr();
   int rc;
   cudaError_t e;
   // dH_d = G W^T: A = G [N, V] K-major, B = W [d, V] K-major.
   CUtensorMap m_ga, m_wk;
   if ((rc = make_map(&m_ga, G, dt, p->V, p->N, p->V * es, kke, 128)) != ALR_OK) return rc;
-  if ((rc = make_map(&m_wk, W, dt, p->V, p->d, p->V * es, kke, 256)) != ALR_OK) return rc;
-  alr::GemmArgs gh = gemm_plan(int(p->N), p->d, p->V, dHd, p->d, info.sms);
-  gh.status = status;
-  e = alr::launch_plain_gemm(dt, false, false, false, m_ga, m_wk, gh, s);
-  if (e != cudaSuccess) return cuda_fail(e, "dH GEMM launch");
+  if ((rc = make_map(&m_wk, W, dt, p->V, p->d, p->V * es, kke, gemm_b_rows(dt))) != ALR_OK)
+    return rc;
+  if ((rc = launch_gemm(dt, false, false, false, m_ga, m_wk, int(p->N), p->d, p->V, dHd, p->d,
+                        info.sms, s, "dH GEMM launch")) != ALR_OK)
+    return rc;
   if (dW == nullptr) return ALR_OK;
-  alr::GemmArgs gw = gemm_plan(p->d, p->V, int(p->N), dW, p->V, info.sms);
-  gw.status = status;
   CUtensorMap m_ha, m_gb;
   if (dt == ALR_BF16) {
     // dW += H_d^T G: A = H_d read as [K = N, M = d] (MN-major), B = G [K = N, V] (MN-major).
     if ((rc = make_map(&m_ha, Hd, dt, p->d, p->N, p->d * es, kke, kke)) != ALR_OK) return rc;
     if ((rc = make_map(&m_gb, G, dt, p->V, p->N, p->V * es, kke, kke)) != ALR_OK) return rc;
-    e = alr::launch_plain_gemm(dt, true, true, true, m_ha, m_gb, gw, s);
+    return launch_gemm(dt, true, true, true, m_ha, m_gb, p->d, p->V, int(p->N), dW, p->V,
+                       info.sms, s, "dW GEMM launch");
   } else {
     // K-major operands from transposed copies H_d^T [d, N'] and G^T [V, N'].
     float* hdt = reinterpret_cast<float*>(ws + lay.hdt_off);
@@ -498,11 +571,11 @@ int head_grads_impl(const alr_params* p, const void* Hd, const void* W, const vo
                                      int(lay.ld_n), s)) != cudaSuccess)
       return cuda_fail(e, "G transpose launch");
     if ((rc = make_map(&m_ha, hdt, dt, p->N, p->d, lay.ld_n * 4, kke, 128)) != ALR_OK) return rc;
-    if ((rc = make_map(&m_gb, gt, dt, p->N, p->V, lay.ld_n * 4, kke, 256)) != ALR_OK) return rc;
-    e = alr::launch_plain_gemm(dt, false, false, true, m_ha, m_gb, gw, s);
+    if ((rc = make_map(&m_gb, gt, dt, p->N, p->V, lay.ld_n * 4, kke, gemm_b_rows(dt))) != ALR_OK)
+      return rc;
+    return launch_gemm(dt, false, false, true, m_ha, m_gb, p->d, p->V, int(p->N), dW, p->V,
+                       info.sms, s, "dW GEMM launch");
   }
-  if (e != cudaSuccess) return cuda_fail(e, "dW GEMM launch");
-  return ALR_OK;
 }
 
 int check_workspace(void* workspace, size_t ws_bytes, size_t need) {
@@ -835,15 +908,10 @@ int alr_gemm(int32_t dtype, int32_t a_mn, int32_t b_mn, int32_t accumulate, cons
   else rc = make_map(&ma, A, dtype, K, M, K * es, kke, 128);
   if (rc != ALR_OK) return rc;
   if (b_mn) rc = make_map(&mb, B, dtype, Nc, K, Nc * es, kke, kke);
-  else rc = make_map(&mb, B, dtype, K, Nc, K * es, kke, 256);
+  else rc = make_map(&mb, B, dtype, K, Nc, K * es, kke, gemm_b_rows(dtype));
   if (rc != ALR_OK) return rc;
-  alr::GemmArgs g = gemm_plan(M, Nc, K, C, Nc, info.sms);
-  g.status = alr::device_status_ptr();
-  if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_plain_gemm(dtype, a_mn != 0, b_mn != 0, accumulate != 0, ma, mb, g,
-                                         static_cast<cudaStream_t>(stream));
-  if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
-  return ALR_OK;
+  return launch_gemm(dtype, a_mn != 0, b_mn != 0, accumulate != 0, ma, mb, M, Nc, K, C, Nc,
+                     info.sms, static_cast<cudaStream_t>(stream), "gemm launch");
 }
 
 }  // extern "C"

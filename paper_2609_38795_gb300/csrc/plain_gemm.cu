@@ -5,6 +5,12 @@
 // 128 x 256 output tiles, tcgen05.mma (M=128, N=256) into two 256-column TMEM buffers,
 // a 4-stage TMA pipeline with 128-byte swizzle, persistent CTAs over raster groups of
 // `group_m` row blocks.  Warp roles as in loss_gemm.cu.
+//
+// Multicast form (kMc, bf16): clusters of two CTAs compute the two 128-row tiles 2i, 2i + 1
+// against the same 256 columns of B.  Each CTA loads its own A rows and one 128-column half of
+// the B tile, multicast into both CTAs' stage, so every B byte leaves L2 once per pair; a stage
+// is refilled only after both CTAs' products have read it (both MMA issuers' commits arrive on
+// both CTAs' empty barriers).
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -68,7 +74,26 @@ ALR_DEV void load_operand(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, i
   }
 }
 
-template <typename Elem, bool kAMN, bool kBMN, bool kAcc>
+// B half of the multicast form: `kExtent` / 2 MN rows starting at half `r`, into the same
+// offsets of both CTAs.
+template <typename Elem, bool kMN, int kExtent>
+ALR_DEV void load_operand_half_mc(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int mn0,
+                                  int kb, int r) {
+  using G = Geo<Elem>;
+  constexpr int kHalfExt = kExtent / 2;
+  if constexpr (kMN) {
+#pragma unroll
+    for (int c = 0; c < kHalfExt / G::kChunkMN; ++c) {
+      const int cc = r * (kHalfExt / G::kChunkMN) + c;
+      tma_load_2d_mc(dst + cc * G::kChunkBytes, map, bar, mn0 + cc * G::kChunkMN, kb * G::kKE,
+                     0x3);
+    }
+  } else {
+    tma_load_2d_mc(dst + r * kHalfExt * 128, map, bar, kb * G::kKE, mn0 + r * kHalfExt, 0x3);
+  }
+}
+
+template <typename Elem, bool kAMN, bool kBMN, bool kAcc, bool kMc>
 __global__ void __launch_bounds__(kThreads, 1)
     plain_gemm_kernel(const __grid_constant__ CUtensorMap tm_a,
                       const __grid_constant__ CUtensorMap tm_b, const GemmArgs args) {
@@ -86,11 +111,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const AbortFlag ab{abort_word, args.status};
+  // kMc: tiles are handed out per cluster, and CTA `rank` takes row block 2 mb + rank
+  const int rank = kMc ? int(cluster_ctarank()) : 0;
+  const int t0 = kMc ? int(cluster_id_x()) : int(blockIdx.x);
+  const int t_step = kMc ? int(n_clusters_x()) : int(gridDim.x);
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&full_bar[i], 1);
-      mbar_init(&empty_bar[i], 1);
+      mbar_init(&empty_bar[i], kMc ? 2 : 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);
@@ -110,6 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (kMc) cluster_sync();   // the peer's copies and commits find initialised barriers
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int n_kb = (args.K + G::kKE - 1) / G::kKE;
@@ -119,9 +149,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0, armed = 0, armed_par = 0;
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < args.n_tiles; t += gridDim.x) {
+      for (int t = t0; ok && t < args.n_tiles; t += t_step) {
         int mb, nb;
         decode_tile(args, t, mb, nb);
+        if (kMc) mb = 2 * mb + rank;
         for (int kb = 0; kb < n_kb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1, ab)) {
             ok = false;
@@ -130,7 +161,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* sb = smem + stage * kStageBytes;
           mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
           load_operand<Elem, kAMN, kBM>(sb, &tm_a, &full_bar[stage], mb * kBM, kb);
-          load_operand<Elem, kBMN, kBN>(sb + kABytes, &tm_b, &full_bar[stage], nb * kBN, kb);
+          if constexpr (kMc)
+            load_operand_half_mc<Elem, kBMN, kBN>(sb + kABytes, &tm_b, &full_bar[stage], nb * kBN,
+                                                  kb, rank);
+          else
+            load_operand<Elem, kBMN, kBN>(sb + kABytes, &tm_b, &full_bar[stage], nb * kBN, kb);
           armed |= 1u << stage;
           armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
           if (++stage == kStages) {
@@ -150,7 +185,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0, abuf = 0;
       uint32_t phase = 0, aphase = 0;
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < args.n_tiles; t += gridDim.x) {
+      for (int t = t0; ok && t < args.n_tiles; t += t_step) {
         if (!mbar_wait(&tempty_bar[abuf], aphase ^ 1, ab)) break;
         tc_fence_after();
         const uint32_t d_acc = tmem_base + uint32_t(abuf * kBN);
@@ -167,7 +202,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 operand_desc<Elem, kBMN>(sa + kABytes, kk), idesc,
                                 (kb > 0 || kk > 0) ? 1u : 0u);
           }
-          mma_commit(&empty_bar[stage]);
+          if constexpr (kMc) mma_commit_mc(&empty_bar[stage], 0x3);
+          else mma_commit(&empty_bar[stage]);
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1;
@@ -188,9 +224,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16);
     int abuf = 0;
     uint32_t aphase = 0;
-    for (int t = blockIdx.x; t < args.n_tiles; t += gridDim.x) {
+    for (int t = t0; t < args.n_tiles; t += t_step) {
       int mb, nb;
       decode_tile(args, t, mb, nb);
+      if (kMc) mb = 2 * mb + rank;
       if (!warp_wait(&tfull_bar[abuf], aphase, ab)) break;
       tc_fence_after();
       const int m = mb * kBM + q * 32 + lane;
@@ -236,21 +273,38 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (kMc) cluster_sync();   // no CTA leaves while its peer may still write into it
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, 512);
   }
 }
 
-template <typename Elem, bool kAMN, bool kBMN, bool kAcc>
+template <typename Elem, bool kAMN, bool kBMN, bool kAcc, bool kMc = false>
 cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,
                      cudaStream_t s) {
-  auto kern = plain_gemm_kernel<Elem, kAMN, kBMN, kAcc>;
+  auto kern = plain_gemm_kernel<Elem, kAMN, kBMN, kAcc, kMc>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes));
   if (e != cudaSuccess) return e;
-  kern<<<args.grid, kThreads, kSmemBytes, s>>>(a, b, args);
-  return cudaGetLastError();
+  if constexpr (!kMc) {
+    kern<<<args.grid, kThreads, kSmemBytes, s>>>(a, b, args);
+    return cudaGetLastError();
+  } else {
+    cudaLaunchConfig_t cfg{};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(unsigned(args.grid));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a, b, args);
+  }
 }
 
 template <typename Elem>
@@ -279,6 +333,48 @@ cudaError_t dispatch(bool a_mn, bool b_mn, bool acc, const CUtensorMap& a, const
 }  // namespace
 
 size_t plain_gemm_smem_bytes(int) { return kSmemBytes; }
+
+int plain_gemm_mc_max_pairs() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] > 0) return cached[dev];
+  auto kern = plain_gemm_kernel<__nv_bfloat16, false, false, false, true>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           int(kSmemBytes)) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) return 0;
+  cached[dev] = n;
+  return n;
+}
+
+cudaError_t launch_plain_gemm_mc(bool a_mn, bool b_mn, bool acc, const CUtensorMap& a,
+                                 const CUtensorMap& b, const GemmArgs& args, cudaStream_t s) {
+  using E = __nv_bfloat16;
+  const int key = (a_mn ? 4 : 0) | (b_mn ? 2 : 0) | (acc ? 1 : 0);
+  switch (key) {
+    case 0: return launch_t<E, false, false, false, true>(a, b, args, s);
+    case 1: return launch_t<E, false, false, true, true>(a, b, args, s);
+    case 2: return launch_t<E, false, true, false, true>(a, b, args, s);
+    case 3: return launch_t<E, false, true, true, true>(a, b, args, s);
+    case 4: return launch_t<E, true, false, false, true>(a, b, args, s);
+    case 5: return launch_t<E, true, false, true, true>(a, b, args, s);
+    case 6: return launch_t<E, true, true, false, true>(a, b, args, s);
+    default: return launch_t<E, true, true, true, true>(a, b, args, s);
+  }
+}
 
 cudaError_t launch_plain_gemm(int dtype, bool a_mn, bool b_mn, bool accumulate,
                               const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,

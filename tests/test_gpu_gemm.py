@@ -1,5 +1,7 @@
 """The tensor-core GEMM of the backward (alr_gemm) against an fp64 product, for every operand
-layout, both element types, with ragged M, N and K tails and with accumulation."""
+layout, both element types, with ragged M, N and K tails and with accumulation.  The largest
+shape has more 256 x 256 tiles (81) than a GB300 holds CTA pairs, so pairs run several tiles
+and cycle through both accumulator buffers."""
 
 import itertools
 
@@ -30,10 +32,18 @@ def _operands(M, Nc, K, dtype, a_mn, b_mn, seed):
     return A_st, B_st, ref
 
 
+@pytest.mark.parametrize("form", ["single", "mcast", "pair"])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("a_mn,b_mn", list(itertools.product([False, True], repeat=2)))
-@pytest.mark.parametrize("shape", [(200, 264, 200), (256, 512, 1024), (8, 8, 8)])
-def test_gemm_layouts(dtype, a_mn, b_mn, shape):
+@pytest.mark.parametrize("shape", [(200, 264, 200), (256, 512, 1024), (8, 8, 8),
+                                   (2200, 2056, 520)])
+def test_gemm_layouts(form, dtype, a_mn, b_mn, shape, monkeypatch):
+    """Every form of the bf16 product (ALR_GEMM_FORM): single CTAs, clusters sharing B by
+    multicast, CTA pairs with M = 256 products; fp32 (tf32) runs on single CTAs whatever the
+    setting."""
+    if dtype == torch.float32 and form != "single":
+        pytest.skip("tf32 products have one form")
+    monkeypatch.setenv("ALR_GEMM_FORM", form)
     M, Nc, K = shape
     if dtype == torch.float32 and (a_mn or b_mn):
         A_st, B_st, _ = _operands(M, Nc, K, dtype, a_mn, b_mn, seed=1)
