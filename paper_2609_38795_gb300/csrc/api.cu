@@ -142,6 +142,17 @@ int check_params(const alr_params* p) {
 #define ALR_LOSS_BN 256
 #endif
 
+// The fused loss kernels run on single CTAs unless the environment variable ALR_LOSS_FORM is
+// "mcast" (bf16 inputs): clusters of two CTAs sharing every head tile by TMA multicast.  The
+// dual-product modes already share each head tile between z_d and z_t, and at the power cap
+// the multicast form settles ~4 % lower in clock for ~1 % fewer L2 bytes per product: it is
+// not faster, so it is not the default.  Both forms give bit-identical results.
+bool loss_multicast(const alr_params* p) {
+  if (p->dtype != ALR_BF16 || ALR_LOSS_BN != 256) return false;
+  const char* v = getenv("ALR_LOSS_FORM");
+  return v != nullptr && strcmp(v, "mcast") == 0;
+}
+
 alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
   alr::LossPlan P{};
   P.N = int(p->N);
@@ -149,13 +160,18 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
   P.V = p->V;
   P.B = p->B;
   P.bn = ALR_LOSS_BN;
-  P.n_rb = int((p->N + 127) / 128);
+  P.mc = loss_multicast(p) ? 1 : 0;
+  // row blocks, or row-block pairs for the multicast form (which places sms / 2 clusters)
+  const int rb = int((p->N + 127) / 128);
+  P.n_rb = P.mc ? (rb + 1) / 2 : rb;
+  const int slots = P.mc ? sms / 2 : sms;
+  const int group = P.mc ? 4 : 8;
   P.n_vt = (p->V + P.bn - 1) / P.bn;
-  P.group_rows = P.n_rb < 8 ? P.n_rb : 8;
+  P.group_rows = P.n_rb < group ? P.n_rb : group;
   if (bwd) {
     P.n_vs = P.n_vt;  // one tile per unit
   } else {
-    int vs = sms / P.group_rows;
+    int vs = slots / P.group_rows;
     if (vs < 1) vs = 1;
     P.n_vs = vs < P.n_vt ? vs : P.n_vt;
   }

@@ -22,6 +22,9 @@ struct LossPlan {
   int group_rows;  // row blocks per group
   int n_units;     // n_rb * n_vs
   int grid;        // persistent CTAs
+  int mc;          // 1: clusters of two CTAs share each head tile by TMA multicast (bf16,
+                   // 256-column tiles); n_rb and group_rows then count row-block pairs and
+                   // the grid is sized from the clusters that fit
 };
 
 // Partial statistics of one row over the columns of one vocabulary split seen by one

@@ -27,6 +27,12 @@
 // lane, warps 2.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one row per thread)
 // and the 64 columns [64 g, 64 g + 64) of the tile, g = (w-2)/4, in 16-column sub-chunks.
 // Every pipeline wait is bounded (tc_common.cuh).
+//
+// Multicast form (kMc, bf16 inputs, 256-column tiles): clusters of two CTAs take row blocks
+// 2i and 2i + 1 of the same vocabulary split and walk its tiles in lockstep.  Each CTA loads its
+// own hidden-state tiles and one 128-column half of every head tile, multicast into both CTAs'
+// stage, so each W byte leaves L2 once per pair; a stage is refilled only after both CTAs'
+// products have read it.  Under the power cap the saved L2 traffic is saved energy.
 #include <cuda_fp16.h>
 
 #include "kernels.h"
@@ -349,7 +355,9 @@ ALR_DEV void store_g(const float (&g)[16], uint8_t* my_stage, uint32_t& n_stores
 // transposed copy W^T [V, d] (fp32 inputs, whose tf32 products take K-major operands only).
 // tm_g: the bf16 G store map (gradient modes) or the z_d store map (kModeFwdKeep, bf16);
 // tm_g2: the z_t store map (kModeFwdKeep, bf16).
-template <typename Elem, int kMode, bool kWMN, int kBN>
+// One block per SM.  With 18 warps (256-column tiles) two of the four SM sub-partitions hold
+// five warps in their 16K-register files, which caps a thread at 96 registers.
+template <typename Elem, int kMode, bool kWMN, int kBN, bool kMc>
 __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem))>::kThreads, 1)
     loss_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,
                      const __grid_constant__ CUtensorMap tm_a1,
@@ -378,11 +386,17 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
   const int lane = threadIdx.x & 31;
   const LossPlan& P = args.plan;
   const AbortFlag ab{abort_word, args.status};
+  // kMc: units are handed out per cluster (P.n_rb counts row-block pairs) and CTA `rank`
+  // takes row block 2 rb + rank
+  static_assert(!kMc || (kWMN && kBN == 256), "multicast form: bf16 head, 256-column tiles");
+  const int rank = kMc ? int(cluster_ctarank()) : 0;
+  const int u0 = kMc ? int(cluster_id_x()) : int(blockIdx.x);
+  const int u_step = kMc ? int(n_clusters_x()) : int(gridDim.x);
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&full_bar[i], 1);
-      mbar_init(&empty_bar[i], 1);
+      mbar_init(&empty_bar[i], kMc ? 2 : 1);
     }
     for (int i = 0; i < S::kAccBufs; ++i) {
       mbar_init(&tfull_bar[i], 1);
@@ -405,6 +419,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (kMc) cluster_sync();   // the peer's copies and commits find initialised barriers
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int n_kb = (P.d + G::kKE - 1) / G::kKE;
@@ -415,9 +430,10 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
       int stage = 0;
       uint32_t phase = 0, armed = 0, armed_par = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < P.n_units; u += gridDim.x) {
+      for (int u = u0; ok && u < P.n_units; u += u_step) {
         int rb, vs;
         decode_unit(P, u, rb, vs);
+        if (kMc) rb = 2 * rb + rank;
         const int vt1 = split_begin(P, vs + 1);
         for (int vt = split_begin(P, vs); ok && vt < vt1; ++vt) {
           for (int kb = 0; kb < n_kb; ++kb) {
@@ -425,7 +441,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
               ok = false;
               break;
             }
-            if (args.withhold_first_stage && u == int(blockIdx.x) && vt == split_begin(P, vs) &&
+            if (args.withhold_first_stage && u == u0 && vt == split_begin(P, vs) &&
                 kb == 0) {
               // test hook: leave this stage empty, so the MMA issuer's bounded wait on it runs
               // out and the whole CTA takes the timeout path
@@ -441,7 +457,16 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
             tma_load_2d(sb, &tm_a0, &full_bar[stage], kb * G::kKE, rb * kBM);
             if constexpr (kDual)
               tma_load_2d(sb + kATileBytes, &tm_a1, &full_bar[stage], kb * G::kKE, rb * kBM);
-            if constexpr (kWMN) {
+            if constexpr (kMc) {
+              // this CTA's half of the head tile, into both CTAs' stage
+              constexpr int kHalfChunks = kBN / G::kChunkMN / 2;
+#pragma unroll
+              for (int c = 0; c < kHalfChunks; ++c) {
+                const int cc = rank * kHalfChunks + c;
+                tma_load_2d_mc(sw + cc * G::kChunkBytes, &tm_w, &full_bar[stage],
+                               vt * kBN + cc * G::kChunkMN, kb * G::kKE, 0x3);
+              }
+            } else if constexpr (kWMN) {
 #pragma unroll
               for (int c = 0; c < kBN / G::kChunkMN; ++c)
                 tma_load_2d(sw + c * G::kChunkBytes, &tm_w, &full_bar[stage],
@@ -470,9 +495,10 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
       int stage = 0, abuf = 0;
       uint32_t phase = 0, aphase = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < P.n_units; u += gridDim.x) {
+      for (int u = u0; ok && u < P.n_units; u += u_step) {
         int rb, vs;
         decode_unit(P, u, rb, vs);
+        if (kMc) rb = 2 * rb + rank;
         const int vt1 = split_begin(P, vs + 1);
         for (int vt = split_begin(P, vs); ok && vt < vt1; ++vt) {
           if (!mbar_wait(&tempty_bar[abuf], aphase ^ 1, ab)) {
@@ -500,7 +526,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
                 mma_issue<G::kTf32>(d_acc + kBN, sdesc_sw128(sa + kATileBytes + kk * 32, 16, 1024),
                                     bd, idesc, acc);
             }
-            mma_commit(&empty_bar[stage]);
+            if constexpr (kMc) mma_commit_mc(&empty_bar[stage], 0x3);
+            else mma_commit(&empty_bar[stage]);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1;
@@ -529,9 +556,10 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
     int abuf = 0;
     uint32_t aphase = 0;
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < P.n_units; u += gridDim.x) {
+    for (int u = u0; ok && u < P.n_units; u += u_step) {
       int rb, vs;
       decode_unit(P, u, rb, vs);
+      if (kMc) rb = 2 * rb + rank;
       const int vt1 = split_begin(P, vs + 1);
       const int row = rb * kBM + row_in_tile;
       const bool row_ok = row < P.N;
@@ -728,31 +756,71 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (kMc) cluster_sync();   // no CTA leaves while its peer may still write into it
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, 512);
   }
 }
 
-template <typename Elem, int kMode, int kBN>
+cudaLaunchConfig_t cluster2_config(cudaLaunchAttribute* attr, unsigned grid, unsigned threads,
+                                   size_t smem, cudaStream_t s) {
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+template <typename Elem, int kMode, int kBN, bool kMc>
 cudaError_t launch_impl(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
                         const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
                         cudaStream_t s) {
   using S = Shape<kMode, kBN, is_staged(kMode, sizeof(Elem))>;
-  auto kern = loss_gemm_kernel<Elem, kMode, sizeof(Elem) == 2, kBN>;
+  auto kern = loss_gemm_kernel<Elem, kMode, sizeof(Elem) == 2, kBN, kMc>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(S::kSmem));
   if (e != cudaSuccess) return e;
-  kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(a0, a1, w, g, g2, args);
-  return cudaGetLastError();
+  if constexpr (!kMc) {
+    kern<<<args.plan.grid, S::kThreads, S::kSmem, s>>>(a0, a1, w, g, g2, args);
+    return cudaGetLastError();
+  } else {
+    // as many clusters as fit at once (one CTA per SM), at most one per unit
+    static int max_clusters[64] = {0};
+    int dev = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    cudaLaunchAttribute attr[1];
+    if (max_clusters[dev] == 0) {
+      cudaLaunchConfig_t q = cluster2_config(attr, 2, S::kThreads, S::kSmem, s);
+      int n = 0;
+      if ((e = cudaOccupancyMaxActiveClusters(&n, kern, &q)) != cudaSuccess) return e;
+      if (n < 1) return cudaErrorInvalidConfiguration;
+      max_clusters[dev] = n;
+    }
+    const int clusters = max_clusters[dev] < args.plan.n_units ? max_clusters[dev]
+                                                               : args.plan.n_units;
+    cudaLaunchConfig_t cfg = cluster2_config(attr, unsigned(2 * clusters), S::kThreads, S::kSmem, s);
+    return cudaLaunchKernelEx(&cfg, kern, a0, a1, w, g, g2, args);
+  }
 }
 
 template <typename Elem, int kMode>
 cudaError_t by_width(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
                      const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
                      cudaStream_t s) {
-  if (args.plan.bn == 128) return launch_impl<Elem, kMode, 128>(a0, a1, w, g, g2, args, s);
-  return launch_impl<Elem, kMode, 256>(a0, a1, w, g, g2, args, s);
+  if (args.plan.bn == 128) return launch_impl<Elem, kMode, 128, false>(a0, a1, w, g, g2, args, s);
+  if constexpr (sizeof(Elem) == 2) {
+    if (args.plan.mc) return launch_impl<Elem, kMode, 256, true>(a0, a1, w, g, g2, args, s);
+  }
+  return launch_impl<Elem, kMode, 256, false>(a0, a1, w, g, g2, args, s);
 }
 
 template <typename Elem>

@@ -238,25 +238,27 @@ ALR_DEV void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: 
 ALR_DEV bool elect_one_lane() { return (threadIdx.x & 31u) == 0; }
 
 // ------------------------------------------------- CTA pairs (2-SM tensor-core products) ---
+// (The cluster coordinates are constant for a kernel's lifetime: their reads are not volatile,
+// so the compiler may re-read them instead of holding them in registers.)
 // A cluster of two CTAs on neighbouring SMs computes one M = 256 product: each CTA holds 128
 // rows of A and half of the columns of B in its own shared memory, and receives its 128 rows
 // of D in its own tensor memory.  The even CTA issues the MMAs for both; all tcgen05
 // allocation, MMA and commit instructions of such a kernel use .cta_group::2.
 ALR_DEV uint32_t cluster_ctarank() {
   uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  asm("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
 }
 
 ALR_DEV uint32_t cluster_id_x() {
   uint32_t r;
-  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  asm("mov.u32 %0, %%clusterid.x;" : "=r"(r));
   return r;
 }
 
 ALR_DEV uint32_t n_clusters_x() {
   uint32_t r;
-  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  asm("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
   return r;
 }
 

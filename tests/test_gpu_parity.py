@@ -271,3 +271,61 @@ def test_ira_block_plan_bit_exact_and_gather():
                                          valid_len=ref["valid_len"].reshape(-1))
     assert np.array_equal(rows.float().cpu().numpy(), g_ref)
     assert np.array_equal(valid_rows.cpu().numpy(), v_ref)
+
+
+# ------------------------------------------------------ loss kernel forms (multicast) ---
+def _all_outputs(Hd, Ht, W, B, mode, tok):
+    """Every fused-kernel output of one problem: forward, kept logits, logit gradient
+    (recomputed), label readout, top-8 forward and gradient."""
+    N, d = Hd.shape
+    V = W.shape[1]
+    out = {}
+    sl = P.gpu_forward(Hd, Ht, W, B, mode=mode, corpus_tok=tok)
+    out.update({f"fwd.{k}": v.clone() for k, v in sl.out.items() if k != "logp_x" or tok is not None})
+    keep = alr.SlotLoss(N, d, V, B, mode=mode, keep_logits=True)
+    keep.forward(Hd, Ht, W, corpus_tok=tok)
+    out["Zd"], out["Zt"] = keep.Zd.clone(), keep.Zt.clone()
+    G = torch.empty(N, V, dtype=Hd.dtype, device="cuda")
+    o = sl.out
+    alr.alr_logit_grad(sl.params, Hd, Ht, W, o["weight"], o["weight_sum"], o["lse_d"], o["lse_t"], G)
+    out["G"] = G
+    f = lambda *sh: torch.empty(*sh, device="cuda")  # noqa: E731
+    lab = dict(top_idx=torch.empty(N, 8, dtype=torch.int32, device="cuda"), top_prob=f(N, 8),
+               tail=f(N), lse_t=f(N), argmax_t=torch.empty(N, dtype=torch.int32, device="cuda"),
+               gap_t=f(N))
+    ws = torch.empty(alr.alr_readout_workspace_size(sl.params), dtype=torch.uint8, device="cuda")
+    alr.alr_label_readout(sl.params, Ht, W, lab, ws)
+    out.update({f"readout.{k}": v for k, v in lab.items()})
+    tk = dict(loss_row=f(N), lse_d=f(N), tail_q=f(N), argmax_d=torch.empty(N, dtype=torch.int32, device="cuda"),
+              gap_d=f(N), weight=f(N), loss_total=f(1), weight_sum=f(1))
+    ws = torch.empty(alr.alr_topk_fwd_workspace_size(sl.params), dtype=torch.uint8, device="cuda")
+    alr.alr_topk_loss_fwd(sl.params, Hd, W, lab["top_idx"], lab["top_prob"], lab["tail"], tk, ws)
+    out.update({f"topk.{k}": v for k, v in tk.items()})
+    Gk = torch.empty(N, V, dtype=Hd.dtype, device="cuda")
+    alr.alr_topk_logit_grad(sl.params, Hd, W, lab["top_idx"], lab["top_prob"], lab["tail"],
+                            tk["weight"], tk["weight_sum"], tk["lse_d"], tk["tail_q"], Gk)
+    out["topk.G"] = Gk
+    torch.cuda.synchronize()
+    assert alr.alr_device_status() == alr.ALR_OK
+    return out
+
+
+@pytest.mark.parametrize("N", [272, 2048])
+def test_loss_kernel_forms_agree_bit_for_bit(N, monkeypatch):
+    """The multicast form of the fused kernels (clusters of two row blocks sharing each head
+    tile, ALR_LOSS_FORM=mcast) and the single-CTA default compute every unit identically, so all
+    outputs agree bit for bit: N = 272 has an odd number of row blocks (the last cluster's
+    second CTA has no rows), N = 2048 several raster groups of pairs."""
+    B, d, V = 16, 520, 3000
+    Hd, Ht, W = _inputs(d, V, N // B, B, 0.5, torch.bfloat16, seed=N)
+    tok = torch.randint(0, V, (N,), dtype=torch.int32, device="cuda")
+    monkeypatch.setenv("ALR_LOSS_FORM", "single")
+    single = _all_outputs(Hd, Ht, W, B, alr.ALR_MODE_ERASE_SOFT, tok)
+    monkeypatch.setenv("ALR_LOSS_FORM", "mcast")
+    mcast = _all_outputs(Hd, Ht, W, B, alr.ALR_MODE_ERASE_SOFT, tok)
+    for k in single:
+        a, b = single[k].cpu(), mcast[k].cpu()
+        if a.dtype.is_floating_point:
+            a, b = a.view(torch.int16 if a.element_size() == 2 else torch.int32), \
+                b.view(torch.int16 if b.element_size() == 2 else torch.int32)
+        assert torch.equal(a, b), k
