@@ -128,16 +128,13 @@ ALR_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "r"(taddr));
 }
 
-// Maximum of 16 values by a balanced tree (depth 4).
+// Maximum of 16 values: seven three-input maxima, depth 3 (max is exact, so any order gives
+// the same value).
 ALR_DEV float max16(const float (&z)[16]) {
-  float a[8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) a[i] = fmaxf(z[2 * i], z[2 * i + 1]);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) a[i] = fmaxf(a[2 * i], a[2 * i + 1]);
-  a[0] = fmaxf(a[0], a[1]);
-  a[2] = fmaxf(a[2], a[3]);
-  return fmaxf(a[0], a[2]);
+  const float a = max3(z[0], z[1], z[2]), b = max3(z[3], z[4], z[5]);
+  const float c = max3(z[6], z[7], z[8]), d = max3(z[9], z[10], z[11]);
+  const float e = max3(z[12], z[13], z[14]);
+  return max3(max3(a, b, c), max3(d, e, z[15]), -INFINITY);
 }
 
 // The sub-chunk's values, with columns at or past nv set to -inf.
@@ -148,17 +145,19 @@ ALR_DEV void load_masked(float (&z)[16], const uint32_t (&r)[16], int nv) {
 }
 
 // Online log-sum-exp: move the reference from m to max(m, cm) and add the sub-chunk's
-// exp(z - ref) (masked -inf columns add 0).
+// exp(z - ref) (masked -inf columns add 0).  Even and odd columns are summed in the two lanes
+// of packed registers.
 ALR_DEV void lse_update(float& m, float& s, const float (&z)[16], float cm) {
   const float nm = fmaxf(m, cm);
   const float sc = ex2((m - nm) * kLog2e);
   const float b = -nm * kLog2e;
-  float r0 = 0.f, r1 = 0.f;
+  const uint64_t l2e = f2_pack(kLog2e, kLog2e), b2 = f2_pack(b, b);
+  uint64_t r = f2_pack(0.f, 0.f);
 #pragma unroll
-  for (int j = 0; j < kSub; j += 2) {
-    r0 += ex2(fmaf(z[j], kLog2e, b));
-    r1 += ex2(fmaf(z[j + 1], kLog2e, b));
-  }
+  for (int j = 0; j < kSub; j += 2)
+    r = f2_add(r, f2_ex2(f2_fma(f2_pack(z[j], z[j + 1]), l2e, b2)));
+  float r0, r1;
+  f2_unpack(r, r0, r1);
   s = fmaf(s, sc, r0 + r1);
   m = nm;
 }
@@ -226,19 +225,36 @@ ALR_DEV void stats_sub(RowStats& st, const uint32_t (&rd)[16], const uint32_t (&
   const float sct = ex2((st.best_t - nbt) * kLog2e);
   const float bt = -nbt * kLog2e;
   float s0 = 0.f, s1 = 0.f, u0 = 0.f, u1 = 0.f, w0 = 0.f, w1 = 0.f;
+  if constexpr (kFull) {
+    // even / odd columns in the two lanes of packed registers (same sums as the scalar loop)
+    const uint64_t l2e = f2_pack(kLog2e, kLog2e), b2 = f2_pack(bt, bt);
+    uint64_t S = f2_pack(0.f, 0.f), U = S, Wt = S;
 #pragma unroll
-  for (int j = 0; j < kSub; j += 2) {
-    if (kFull || j < nv) {
-      const float e = ex2(fmaf(zt[j], kLog2e, bt));
-      s0 += e;
-      u0 = fmaf(e, zd[j], u0);
-      w0 = fmaf(e, zt[j], w0);
+    for (int j = 0; j < kSub; j += 2) {
+      const uint64_t ZT = f2_pack(zt[j], zt[j + 1]), ZD = f2_pack(zd[j], zd[j + 1]);
+      const uint64_t E = f2_ex2(f2_fma(ZT, l2e, b2));
+      S = f2_add(S, E);
+      U = f2_fma(E, ZD, U);
+      Wt = f2_fma(E, ZT, Wt);
     }
-    if (kFull || j + 1 < nv) {
-      const float e = ex2(fmaf(zt[j + 1], kLog2e, bt));
-      s1 += e;
-      u1 = fmaf(e, zd[j + 1], u1);
-      w1 = fmaf(e, zt[j + 1], w1);
+    f2_unpack(S, s0, s1);
+    f2_unpack(U, u0, u1);
+    f2_unpack(Wt, w0, w1);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kSub; j += 2) {
+      if (j < nv) {
+        const float e = ex2(fmaf(zt[j], kLog2e, bt));
+        s0 += e;
+        u0 = fmaf(e, zd[j], u0);
+        w0 = fmaf(e, zt[j], w0);
+      }
+      if (j + 1 < nv) {
+        const float e = ex2(fmaf(zt[j + 1], kLog2e, bt));
+        s1 += e;
+        u1 = fmaf(e, zd[j + 1], u1);
+        w1 = fmaf(e, zt[j + 1], w1);
+      }
     }
   }
   st.s_t = fmaf(st.s_t, sct, s0 + s1);
@@ -628,8 +644,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
           const int nv = min(kSub, P.V - v0);
 
           if constexpr (is_fwd(kMode)) {
-            if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x);
-            else stats_sub<false>(st, r0, r1, v0, nv, x);
+            // kept logits first: their packed copies die before the statistics need registers
             if constexpr (kMode == kModeFwdKeep) {
               if constexpr (kStaged) {
                 keep_logits_staged(r0, r1, my_stage, &tm_g, &tm_g2, v0, rb * kBM + q * 32, lane);
@@ -639,6 +654,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
                 keep_logits_f32(r1, args.zt_out, off, nv);
               }
             }
+            if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x);
+            else stats_sub<false>(st, r0, r1, v0, nv, x);
           } else if constexpr (kMode == kModeReadout || kMode == kModeTopkFwd) {
             float z[16];
             if (nv == kSub) load_masked<true>(z, r0, nv);
@@ -674,17 +691,24 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
             }
           } else {   // gradient modes
             float g[16];
+            const uint64_t l2e = f2_pack(kLog2e, kLog2e), ad2 = f2_pack(ad, ad);
             if constexpr (kMode == kModeBwd) {
+              const uint64_t at2 = f2_pack(at, at), cw2 = f2_pack(cw, cw);
 #pragma unroll
-              for (int j = 0; j < kSub; ++j)
-                g[j] = cw * (ex2(fmaf(f32(r0[j]), kLog2e, ad)) - ex2(fmaf(f32(r1[j]), kLog2e, at)));
+              for (int j = 0; j < kSub; j += 2) {
+                const uint64_t q2 = f2_ex2(f2_fma(f2_pack(f32(r0[j]), f32(r0[j + 1])), l2e, ad2));
+                const uint64_t p2 = f2_ex2(f2_fma(f2_pack(f32(r1[j]), f32(r1[j + 1])), l2e, at2));
+                f2_unpack(f2_mul(cw2, f2_sub(q2, p2)), g[j], g[j + 1]);
+              }
             } else {
               float qv[16];
               const float cb = cw * beta;
+              const uint64_t cb2 = f2_pack(cb, cb);
 #pragma unroll
-              for (int j = 0; j < kSub; ++j) {
-                qv[j] = ex2(fmaf(f32(r0[j]), kLog2e, ad));
-                g[j] = cb * qv[j];
+              for (int j = 0; j < kSub; j += 2) {
+                const uint64_t q2 = f2_ex2(f2_fma(f2_pack(f32(r0[j]), f32(r0[j + 1])), l2e, ad2));
+                f2_unpack(q2, qv[j], qv[j + 1]);
+                f2_unpack(f2_mul(cb2, q2), g[j], g[j + 1]);
               }
               bool hit = false;
 #pragma unroll
