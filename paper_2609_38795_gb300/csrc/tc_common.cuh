@@ -38,6 +38,50 @@ ALR_DEV float ex2(float x) {
   return y;
 }
 
+// ------------------------------------------------------ paired fp32 arithmetic ---
+// Two fp32 lanes in one 64-bit register, combined by the sm_100-family packed instructions:
+// each lane is computed exactly as the scalar instruction would, in one issue slot for both.
+ALR_DEV uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+ALR_DEV void f2_unpack(uint64_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+ALR_DEV uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+ALR_DEV uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+ALR_DEV uint64_t f2_sub(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+ALR_DEV uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+// 2^a and 2^b of a packed pair (two special-function operations).
+ALR_DEV uint64_t f2_ex2(uint64_t v) {
+  float a, b;
+  f2_unpack(v, a, b);
+  return f2_pack(ex2(a), ex2(b));
+}
+// Three-input maximum (one instruction); no NaN inputs occur where it is used.
+ALR_DEV float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 // ---------------------------------------------------------------- mbarrier ---
 ALR_DEV void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
@@ -82,18 +126,25 @@ struct AbortFlag {
   int* status;   // per-device status word in global memory
 };
 
+// A suspended waiter wakes whenever its barrier (or its CTA's barriers) change state, which
+// during a tile happens every few hundred cycles; the clock and the abort word are checked
+// only on every kWaitCheckEvery-th wake-up, so a wake-up costs a handful of instructions.
+constexpr uint32_t kWaitCheckEvery = 16;
+
 // Wait until the phase with the given parity has completed.  Returns false (after recording
 // the timeout) if the limit elapses or another role of the CTA already gave up.
 ALR_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
-  for (;;) {
+  for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (*ab.smem) return false;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
-      *ab.smem = 1;
-      atomicExch(ab.status, kStatusTimeout);
-      return false;
+    if (i % kWaitCheckEvery == 0) {
+      if (*ab.smem) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *ab.smem = 1;
+        atomicExch(ab.status, kStatusTimeout);
+        return false;
+      }
     }
   }
 }
@@ -297,13 +348,15 @@ ALR_DEV bool mbar_try_wait_cl(uint64_t* bar, uint32_t parity) {
 ALR_DEV bool mbar_wait_cl(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
   if (mbar_try_wait_cl(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
-  for (;;) {
+  for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait_cl(bar, parity)) return true;
-    if (*ab.smem) return false;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
-      *ab.smem = 1;
-      atomicExch(ab.status, kStatusTimeout);
-      return false;
+    if (i % kWaitCheckEvery == 0) {
+      if (*ab.smem) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *ab.smem = 1;
+        atomicExch(ab.status, kStatusTimeout);
+        return false;
+      }
     }
   }
 }
