@@ -353,6 +353,44 @@ int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const 
                       float* dHd, float* dW, void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * Kept logits for the top-k loss (as for the full-vocabulary loss above): the forward also
+ * writes z_d = H_d W, and the gradient is then formed from it instead of recomputing the head
+ * product.
+ *
+ * alr_topk_loss_fwd_keep_logits: alr_topk_loss_fwd (same arguments, outputs, workspace and
+ * errors, bit-identical outputs) that also writes Zd [N, V] row-major, fp16 for ALR_BF16 inputs
+ * (|z| < 65504), fp32 for ALR_F32; caller-owned, 16-byte aligned, overlapping nothing else.
+ */
+int alr_topk_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* W,
+                                  const int32_t* top_idx, const float* top_prob, const float* tail,
+                                  const float* row_mask, const float* weight_in, void* Zd,
+                                  const alr_topk_fwd_outputs* out, void* workspace,
+                                  size_t ws_bytes, void* stream);
+
+/*
+ * G of the top-k + tail loss from kept z_d (types as above) and the forward's weight,
+ * weight_sum, lse_d, tail_q: G = c_r beta_r q outside the row's label tokens and
+ * c_r (q - top_prob) at them, q = exp(z_d - lse_d), c_r = lambda omega_r / sum omega,
+ * beta_r = 1 - tail_r / tail_q_r.  G [N, V] (bf16 / fp32) may be Zd itself (in place); it must
+ * not otherwise overlap Zd.  A row's label tokens must be distinct.  No workspace.
+ */
+int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const int32_t* top_idx,
+                                    const float* top_prob, const float* tail, const float* weight,
+                                    const float* weight_sum, const float* lse_d,
+                                    const float* tail_q, void* G, void* stream);
+
+/*
+ * Backward of the top-k loss from kept z_d: alr_topk_logit_grad_from_logits into G (may be Zd),
+ * dHd = G W^T (overwritten) and, when dW is given, dW += H_d^T G.
+ * Workspace: alr_bwd_from_logits_workspace_size.
+ */
+int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
+                                  const void* Zd, const int32_t* top_idx, const float* top_prob,
+                                  const float* tail, const float* weight, const float* weight_sum,
+                                  const float* lse_d, const float* tail_q, void* G, float* dHd,
+                                  float* dW, void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * Greedy accepted length per anchor (Sec. 3.2: slot k counts only when slots 1..k-1 were
  * accepted; MAT tau = acc + 1, Sec. 4).
  *   argmax_d, argmax_t [A*B] int32; active [A*B] float or NULL (rows with active <= 0 stop

@@ -87,6 +87,15 @@ SIGNATURES = {
                                      _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_topk_loss_bwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_topk_loss_fwd_keep_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_p, _c_p,
+                                               ctypes.POINTER(AlrTopkFwdOutputs), _c_p, _c_sz,
+                                               _c_p]),
+    "alr_topk_logit_grad_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
+                                                 _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]),
+    "alr_topk_loss_bwd_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_sz, _c_p]),
     "alr_ira_blocks": (_c_int, [_c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
@@ -300,6 +309,34 @@ def alr_topk_loss_bwd(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum
                                    _ptr(top_prob), _ptr(tail), _ptr(weight), _ptr(weight_sum),
                                    _ptr(lse_d), _ptr(tail_q), _ptr(dHd), _ptr(dW),
                                    _ptr(workspace), _nbytes(workspace), _stream(stream)))
+
+
+def alr_topk_loss_fwd_keep_logits(params, Hd, W, top_idx, top_prob, tail, Zd, out: dict,
+                                  workspace, row_mask=None, weight_in=None, stream=None):
+    o = AlrTopkFwdOutputs(**{f: _ptr(out.get(f)) for f in _TOPK_FIELDS})
+    _check(lib().alr_topk_loss_fwd_keep_logits(ctypes.byref(params), _ptr(Hd), _ptr(W),
+                                               _ptr(top_idx), _ptr(top_prob), _ptr(tail),
+                                               _ptr(row_mask), _ptr(weight_in), _ptr(Zd),
+                                               ctypes.byref(o), _ptr(workspace),
+                                               _nbytes(workspace), _stream(stream)))
+
+
+def alr_topk_logit_grad_from_logits(params, Zd, top_idx, top_prob, tail, weight, weight_sum,
+                                    lse_d, tail_q, G, stream=None):
+    _check(lib().alr_topk_logit_grad_from_logits(ctypes.byref(params), _ptr(Zd), _ptr(top_idx),
+                                                 _ptr(top_prob), _ptr(tail), _ptr(weight),
+                                                 _ptr(weight_sum), _ptr(lse_d), _ptr(tail_q),
+                                                 _ptr(G), _stream(stream)))
+
+
+def alr_topk_loss_bwd_from_logits(params, Hd, W, Zd, top_idx, top_prob, tail, weight, weight_sum,
+                                  lse_d, tail_q, G, dHd, dW, workspace=None, stream=None):
+    _check(lib().alr_topk_loss_bwd_from_logits(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(Zd),
+                                               _ptr(top_idx), _ptr(top_prob), _ptr(tail),
+                                               _ptr(weight), _ptr(weight_sum), _ptr(lse_d),
+                                               _ptr(tail_q), _ptr(G), _ptr(dHd), _ptr(dW),
+                                               _ptr(workspace), _nbytes(workspace),
+                                               _stream(stream)))
 
 
 def alr_ira_blocks(K, max_blocks, valid_anchors, rollout_len, offsets, out: dict,

@@ -756,10 +756,15 @@ size_t alr_topk_fwd_workspace_size(const alr_params* p) {
   return fwd_layout(p, info.sms, alr::kKFields).total;
 }
 
-int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
-                      const float* top_prob, const float* tail, const float* row_mask,
-                      const float* weight_in, const alr_topk_fwd_outputs* out, void* workspace,
-                      size_t ws_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The top-k + tail forward; with Zd given the fused kernel also writes z_d (kModeTopkFwdKeep).
+int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
+                  const float* top_prob, const float* tail, const float* row_mask,
+                  const float* weight_in, void* Zd, const alr_topk_fwd_outputs* out,
+                  void* workspace, size_t ws_bytes, void* stream) {
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
@@ -784,9 +789,16 @@ int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const 
   args.plan = loss_plan(p, info.sms, false);
   args.part = reinterpret_cast<float*>(ws + lay.part_off);
   args.top_idx = top_idx;
+  args.zd_out = Zd;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-  cudaError_t e = alr::launch_loss_kernel(alr::kModeTopkFwd, dt, m_h, m_h, m_w, m_w, m_w, args, s);
+  CUtensorMap m_zd = m_w;
+  if (Zd != nullptr && dt == ALR_BF16 &&
+      (rc = make_map(&m_zd, Zd, kMapF16, p->V, p->N, p->V * 2, 16, 32,
+                     CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
+    return rc;
+  cudaError_t e = alr::launch_loss_kernel(Zd != nullptr ? alr::kModeTopkFwdKeep : alr::kModeTopkFwd,
+                                          dt, m_h, m_h, m_w, m_zd, m_zd, args, s);
   if (e != cudaSuccess) return cuda_fail(e, "top-k forward kernel launch");
   double* anchor = reinterpret_cast<double*>(ws + lay.anchor_off);
   e = alr::launch_topk_combine(args.plan, args.part, top_prob, tail, row_mask, weight_in, p->gamma,
@@ -796,6 +808,70 @@ int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const 
   e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
   if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
   return ALR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
+                      const float* top_prob, const float* tail, const float* row_mask,
+                      const float* weight_in, const alr_topk_fwd_outputs* out, void* workspace,
+                      size_t ws_bytes, void* stream) {
+  return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, nullptr, out,
+                       workspace, ws_bytes, stream);
+}
+
+int alr_topk_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* W,
+                                  const int32_t* top_idx, const float* top_prob, const float* tail,
+                                  const float* row_mask, const float* weight_in, void* Zd,
+                                  const alr_topk_fwd_outputs* out, void* workspace,
+                                  size_t ws_bytes, void* stream) {
+  if (Zd == nullptr || !aligned16(Zd))
+    return fail(ALR_ERR_INVALID_ARG, "Zd must be non-NULL and 16-byte aligned");
+  return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, Zd, out,
+                       workspace, ws_bytes, stream);
+}
+
+int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const int32_t* top_idx,
+                                    const float* top_prob, const float* tail, const float* weight,
+                                    const float* weight_sum, const float* lse_d,
+                                    const float* tail_q, void* G, void* stream) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
+  if (Zd == nullptr || G == nullptr || weight == nullptr || weight_sum == nullptr ||
+      lse_d == nullptr || tail_q == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (!aligned16(Zd) || !aligned16(G))
+    return fail(ALR_ERR_INVALID_ARG, "Zd and G must be 16-byte aligned");
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  cudaError_t e = alr::launch_topk_logits_grad(p->dtype, Zd, top_idx, top_prob, tail, tail_q,
+                                               lse_d, weight, weight_sum, p->lambda, int(p->N),
+                                               p->V, G, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "top-k logit-gradient launch");
+  return ALR_OK;
+}
+
+int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
+                                  const void* Zd, const int32_t* top_idx, const float* top_prob,
+                                  const float* tail, const float* weight, const float* weight_sum,
+                                  const float* lse_d, const float* tail_q, void* G, float* dHd,
+                                  float* dW, void* workspace, size_t ws_bytes, void* stream) {
+  int rc = alr_topk_logit_grad_from_logits(p, Zd, top_idx, top_prob, tail, weight, weight_sum,
+                                           lse_d, tail_q, G, stream);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || W == nullptr || dHd == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Hd, W and dHd must be non-NULL");
+  if (!aligned16(Hd) || !aligned16(W) || !aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, W, dHd and dW must be 16-byte aligned");
+  const BwdLayout lay = bwd_layout(p, false);
+  if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
+  DevInfo info;
+  if ((rc = require_sm103(&info)) != ALR_OK) return rc;
+  return head_grads_impl(p, Hd, W, G, dHd, dW, static_cast<uint8_t*>(workspace), lay, info,
+                         static_cast<cudaStream_t>(stream));
 }
 
 int alr_topk_logit_grad(const alr_params* p, const void* Hd, const void* W,

@@ -64,7 +64,8 @@ enum LossMode {
   kModeReadout = 2,  // single GEMM on H_t: log-sum-exp, top-k, z_t at the corpus token
   kModeTopkFwd = 3,  // single GEMM on H_d: log-sum-exp, top-2, z_d at the label tokens
   kModeTopkBwd = 4,  // single GEMM on H_d: gradient of the top-k + tail soft CE
-  kModeFwdKeep = 5   // kModeFwd that also writes z_d and z_t to global memory
+  kModeFwdKeep = 5,  // kModeFwd that also writes z_d and z_t to global memory
+  kModeTopkFwdKeep = 6  // kModeTopkFwd that also writes z_d to global memory
 };
 
 struct LossArgs {
@@ -83,7 +84,7 @@ struct LossArgs {
   const float* top_prob;      // top-k backward: label probabilities [N, kTopK]
   const float* tail;          // top-k backward: label tail mass [N]
   const float* tail_q;        // top-k backward: drafter mass outside the label tokens [N]
-  void* zd_out;               // kModeFwdKeep: z_d, z_t [N, V] (fp16 for bf16 inputs, else fp32)
+  void* zd_out;               // keep modes: z_d (and z_t) [N, V] (fp16 for bf16 inputs, else fp32)
   void* zt_out;
 };
 
@@ -154,6 +155,15 @@ cudaError_t launch_topk_combine(const LossPlan& plan, const float* part, const f
 cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const float* lse_d,
                                const float* lse_t, const float* weight, const float* weight_sum,
                                float lam, int N, int V, void* G, cudaStream_t s);
+// Gradient of the top-k + tail soft CE from kept z_d (fp16 for dtype 0, fp32 for dtype 1):
+// G = c_r beta_r q outside the row's label tokens, c_r (q - prob_i) at label token i, with
+// q = exp(z_d - lse_d), c_r = lambda omega_r / sum omega, beta_r = 1 - tail_r / tail_q_r (1 when
+// tail_r = 0).  G (bf16 / fp32) may be zd itself.
+cudaError_t launch_topk_logits_grad(int dtype, const void* zd, const int32_t* top_idx,
+                                    const float* top_prob, const float* tail, const float* tail_q,
+                                    const float* lse_d, const float* weight,
+                                    const float* weight_sum, float lam, int N, int V, void* G,
+                                    cudaStream_t s);
 cudaError_t launch_accept_len(const int32_t* am_d, const int32_t* am_t, const float* active,
                               int A, int B, int32_t* acc, int64_t* hist, cudaStream_t s);
 cudaError_t launch_erase_weights(const float* logp_x, const int32_t* corpus_tok,

@@ -17,7 +17,8 @@
 //                step keeps, App. A) plus z_t at the corpus token;
 //   kModeTopkFwd z_d only: log-sum-exp, greedy top-2 and z_d at the row's k label tokens (the
 //                top-k + tail-bin soft CE of Sec. 3.1);
-//   kModeTopkBwd z_d only, recomputed: the gradient of that loss.
+//   kModeTopkBwd z_d only, recomputed: the gradient of that loss;
+//   kModeTopkFwdKeep  kModeTopkFwd that also writes z_d (fp16 for bf16 inputs, fp32 else).
 //
 // Accumulators: the dual modes use 2 x kBN TMEM columns per tile (single-buffered at kBN =
 // 256), the single-operand modes kBN columns (double-buffered, so their epilogue overlaps the
@@ -63,11 +64,12 @@ struct Geo {
 constexpr bool is_fwd(int mode) { return mode == kModeFwd || mode == kModeFwdKeep; }
 constexpr bool is_dual(int mode) { return is_fwd(mode) || mode == kModeBwd; }
 constexpr bool is_grad(int mode) { return mode == kModeBwd || mode == kModeTopkBwd; }
+constexpr bool is_topk_fwd(int mode) { return mode == kModeTopkFwd || mode == kModeTopkFwdKeep; }
 // Modes whose epilogue writes 16-bit [N, V] tiles through shared staging and TMA stores: the
 // bf16 gradient (two buffers per warp, double-buffered) and the kept fp16 logits (one buffer
 // per logit matrix).  fp32 outputs are written directly.
 constexpr bool is_staged(int mode, int elem_bytes) {
-  return elem_bytes == 2 && (is_grad(mode) || mode == kModeFwdKeep);
+  return elem_bytes == 2 && (is_grad(mode) || mode == kModeFwdKeep || mode == kModeTopkFwdKeep);
 }
 
 template <int kMode, int kBN, bool kStaged>
@@ -310,6 +312,27 @@ ALR_DEV void keep_logits_staged(const uint32_t (&rd)[16], const uint32_t (&rt)[1
     tma_store_2d(tm_zt, my_stage + kGStageBytes, v0, row0);
     tma_store_commit();
   }
+}
+
+// Keep one warp's 32 x 16 sub-chunk of z_d alone, fp16 (bf16 inputs), through the warp's two
+// staging buffers in turn (the store issued from a buffer two sub-chunks ago must have read it).
+ALR_DEV void keep_one_staged(const uint32_t (&r)[16], uint8_t* my_stage, uint32_t& n_stores,
+                             const CUtensorMap* tm, int v0, int row0, int lane) {
+  uint8_t* buf = my_stage + (n_stores & 1u) * kGStageBytes;
+  if (lane == 0) tma_store_wait_read_le1();
+  __syncwarp();
+  uint4* b = reinterpret_cast<uint4*>(buf + lane * 32);
+  b[0] = make_uint4(pack_f16x2(r[0], r[1]), pack_f16x2(r[2], r[3]), pack_f16x2(r[4], r[5]),
+                    pack_f16x2(r[6], r[7]));
+  b[1] = make_uint4(pack_f16x2(r[8], r[9]), pack_f16x2(r[10], r[11]), pack_f16x2(r[12], r[13]),
+                    pack_f16x2(r[14], r[15]));
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    tma_store_2d(tm, buf, v0, row0);
+    tma_store_commit();
+  }
+  ++n_stores;
 }
 
 // Keep one thread's 16 fp32 logits (fp32 inputs) with direct streaming stores: columns v0..
@@ -600,7 +623,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
       if constexpr (is_fwd(kMode)) stats_init(st);
       if constexpr (is_fwd(kMode) || kMode == kModeReadout)
         x = (args.corpus_tok != nullptr && row_ok) ? args.corpus_tok[row] : -1;
-      if constexpr (kMode == kModeTopkFwd || kMode == kModeTopkBwd) {
+      if constexpr (is_topk_fwd(kMode) || kMode == kModeTopkBwd) {
         if (row_ok) {
 #pragma unroll
           for (int i = 0; i < kTopK; ++i) ti[i] = args.top_idx[size_t(row) * kTopK + i];
@@ -656,7 +679,14 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
             }
             if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x);
             else stats_sub<false>(st, r0, r1, v0, nv, x);
-          } else if constexpr (kMode == kModeReadout || kMode == kModeTopkFwd) {
+          } else if constexpr (kMode == kModeReadout || is_topk_fwd(kMode)) {
+            if constexpr (kMode == kModeTopkFwdKeep) {
+              if constexpr (kStaged) {
+                keep_one_staged(r0, my_stage, n_stores, &tm_g, v0, rb * kBM + q * 32, lane);
+              } else if (row_ok) {
+                keep_logits_f32(r0, args.zd_out, size_t(row) * size_t(P.V) + size_t(v0), nv);
+              }
+            }
             float z[16];
             if (nv == kSub) load_masked<true>(z, r0, nv);
             else load_masked<false>(z, r0, nv);
@@ -762,7 +792,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
             o[(kRIdx + i) * fs] = __int_as_float(ti[i]);
           }
           o[kRZx * fs] = zx;
-        } else if constexpr (kMode == kModeTopkFwd) {
+        } else if constexpr (is_topk_fwd(kMode)) {
           o[kKM * fs] = m;
           o[kKS * fs] = s;
           o[kKBest * fs] = best;
@@ -858,6 +888,7 @@ cudaError_t by_mode(int mode, const CUtensorMap& a0, const CUtensorMap& a1, cons
     case kModeReadout: return by_width<Elem, kModeReadout>(a0, a1, w, g, g2, args, s);
     case kModeTopkFwd: return by_width<Elem, kModeTopkFwd>(a0, a1, w, g, g2, args, s);
     case kModeTopkBwd: return by_width<Elem, kModeTopkBwd>(a0, a1, w, g, g2, args, s);
+    case kModeTopkFwdKeep: return by_width<Elem, kModeTopkFwdKeep>(a0, a1, w, g, g2, args, s);
     default: return cudaErrorInvalidValue;
   }
 }

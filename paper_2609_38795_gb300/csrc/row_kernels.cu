@@ -572,7 +572,86 @@ __global__ void __launch_bounds__(256, sizeof(Z) == 2 ? 4 : 2) logits_grad_kerne
   }
 }
 
+__device__ __forceinline__ float load1(const __half* p) { return __half2float(*p); }
+__device__ __forceinline__ float load1(const float* p) { return *p; }
+__device__ __forceinline__ void store1(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+__device__ __forceinline__ void store1(float* p, float v) { *p = v; }
+
+// Gradient of the top-k + tail soft CE from the kept z_d: c beta q over the whole row, then
+// c (q - prob_i) at the row's label tokens, whose logits are read before the row is
+// overwritten (G may be the z_d buffer).  The label tokens of a row are distinct.
+template <typename Z, typename Gt>
+__global__ void __launch_bounds__(256, sizeof(Z) == 2 ? 4 : 2) topk_logits_grad_kernel(
+    const Z* zd, const int32_t* __restrict__ top_idx, const float* __restrict__ top_prob,
+    const float* __restrict__ tail, const float* __restrict__ tail_q,
+    const float* __restrict__ lse_d, const float* __restrict__ weight,
+    const float* __restrict__ weight_sum, float lam, int V, Gt* G) {
+  __shared__ float lab_g[kTopK];
+  __shared__ int lab_v[kTopK];
+  const int row = blockIdx.x;
+  const float ws = *weight_sum;
+  const float c = ws > 0.f ? lam * weight[row] / ws : 0.f;
+  const size_t base = size_t(row) * size_t(V);
+  const int n8 = V / 8;
+  if (c == 0.f) {
+    const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int i = threadIdx.x; i < n8; i += blockDim.x) store8(G + base + 8 * size_t(i), z);
+    return;
+  }
+  const float ad = -lse_d[row] * kLog2e;
+  const float tl = tail[row];
+  const float cb = c * (tl > 0.f ? 1.f - tl / tail_q[row] : 1.f);
+  if (threadIdx.x < kTopK) {
+    const int v = top_idx[size_t(row) * kTopK + threadIdx.x];
+    lab_v[threadIdx.x] = v;
+    if (v >= 0 && v < V)
+      lab_g[threadIdx.x] = c * (ex2(fmaf(load1(zd + base + v), kLog2e, ad)) -
+                                top_prob[size_t(row) * kTopK + threadIdx.x]);
+  }
+  __syncthreads();
+  for (int i0 = threadIdx.x; i0 < n8; i0 += kLogitsUnroll * blockDim.x) {
+    Raw8<Z> a[kLogitsUnroll];
+#pragma unroll
+    for (int u = 0; u < kLogitsUnroll; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n8) a[u].load(zd + base + 8 * size_t(i));
+    }
+#pragma unroll
+    for (int u = 0; u < kLogitsUnroll; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < n8) {
+        float x[8], g[8];
+        a[u].to_float(x);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) g[j] = cb * ex2(fmaf(x[j], kLog2e, ad));
+        store8(G + base + 8 * size_t(i), g);
+      }
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < kTopK) {
+    const int v = lab_v[threadIdx.x];
+    if (v >= 0 && v < V) store1(G + base + v, lab_g[threadIdx.x]);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_topk_logits_grad(int dtype, const void* zd, const int32_t* top_idx,
+                                    const float* top_prob, const float* tail, const float* tail_q,
+                                    const float* lse_d, const float* weight,
+                                    const float* weight_sum, float lam, int N, int V, void* G,
+                                    cudaStream_t s) {
+  if (dtype == 0)
+    topk_logits_grad_kernel<__half, __nv_bfloat16><<<N, 256, 0, s>>>(
+        static_cast<const __half*>(zd), top_idx, top_prob, tail, tail_q, lse_d, weight,
+        weight_sum, lam, V, static_cast<__nv_bfloat16*>(G));
+  else
+    topk_logits_grad_kernel<float, float><<<N, 256, 0, s>>>(
+        static_cast<const float*>(zd), top_idx, top_prob, tail, tail_q, lse_d, weight,
+        weight_sum, lam, V, static_cast<float*>(G));
+  return cudaGetLastError();
+}
 
 cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const float* lse_d,
                                const float* lse_t, const float* weight, const float* weight_sum,

@@ -105,7 +105,8 @@ def test_readout_exact_ties_and_small_vocabulary():
     assert np.array_equal(P.npi(g["top_idx"])[:, :2], r["idx"][:, :2])
 
 
-def gpu_topk_forward(Hd, W, B, labels, row_mask=None, weight_in=None, lam=1.0):
+def gpu_topk_forward(Hd, W, B, labels, row_mask=None, weight_in=None, lam=1.0, Zd=None):
+    """The top-k forward; with Zd given, the variant that also keeps z_d there."""
     N, d = Hd.shape
     V = W.shape[1]
     params = alr.make_params(N, d, V, B, Hd.dtype, lam=lam)
@@ -114,8 +115,13 @@ def gpu_topk_forward(Hd, W, B, labels, row_mask=None, weight_in=None, lam=1.0):
                gap_d=f(), weight=f(), loss_total=torch.zeros(1, device="cuda"),
                weight_sum=torch.zeros(1, device="cuda"))
     ws = torch.empty(alr.alr_topk_fwd_workspace_size(params), dtype=torch.uint8, device="cuda")
-    alr.alr_topk_loss_fwd(params, Hd, W, labels["idx"], labels["prob"], labels["tail"], out, ws,
-                          row_mask=row_mask, weight_in=weight_in)
+    if Zd is None:
+        alr.alr_topk_loss_fwd(params, Hd, W, labels["idx"], labels["prob"], labels["tail"], out, ws,
+                              row_mask=row_mask, weight_in=weight_in)
+    else:
+        alr.alr_topk_loss_fwd_keep_logits(params, Hd, W, labels["idx"], labels["prob"],
+                                          labels["tail"], Zd, out, ws, row_mask=row_mask,
+                                          weight_in=weight_in)
     torch.cuda.synchronize()
     return params, out
 
@@ -187,10 +193,13 @@ def random_labels(N, V, seed):
     return dict(idx=idx, prob=-np.sort(-raw[:, :K], axis=1), tail=raw[:, K])
 
 
-def test_text8b_full_batch_compact_labels():
+@pytest.mark.parametrize("keep", [True, False])
+def test_text8b_full_batch_compact_labels(keep):
     """The compact-label path at the text8b size (32768 rows, V = 151936): readout of every
     row on the GPU; sampled anchors against the oracle; the top-k loss with oracle labels on
-    the sampled anchors and random labels elsewhere; totals through properties."""
+    the sampled anchors and random labels elsewhere; totals through properties.  keep: the
+    step bench.py times (forward keeping z_d, G from it in place, dH and dW as two GEMM calls);
+    otherwise the recomputing backward."""
     wl = synthetic.WORKLOADS["text8b"]
     b = synthetic.slot_batch(wl.d, wl.V, wl.A, wl.B, 0.5, device="cuda", seed=4)
     Hd, Ht, W = b["Hd"], b["Ht"], b["W"]
@@ -203,8 +212,12 @@ def test_text8b_full_batch_compact_labels():
     lab_np = random_labels(wl.N, wl.V, seed=6)
     lab_np["idx"][rows], lab_np["prob"][rows], lab_np["tail"][rows] = r["idx"], r["prob"], r["tail"]
     lab = device_labels(lab_np)
-    params, out = gpu_topk_forward(Hd, W, wl.B, lab)
+    Zd = torch.empty(wl.N, wl.V, dtype=torch.float16, device="cuda") if keep else None
+    params, out = gpu_topk_forward(Hd, W, wl.B, lab, Zd=Zd)
     z_d = P.np64(Hd)[rows] @ W64
+    if keep:
+        kept = P.np64(Zd[torch.from_numpy(rows).cuda()])
+        assert np.all(np.abs(kept - z_d) <= 2.0 ** -11 * np.abs(z_d) + 1e-4)
     loss_r, tq_r = orc.top_k_soft_cross_entropy(z_d, r["idx"], r["prob"], r["tail"])
     assert P.rel_err(P.np64(out["loss_row"])[rows], loss_r).max() <= P.LOSS_RTOL
     np.testing.assert_allclose(P.np64(out["tail_q"])[rows], tq_r, rtol=1e-3, atol=1e-6)
@@ -214,7 +227,17 @@ def test_text8b_full_batch_compact_labels():
     L_host = (w_all * l_all).sum() / w_all.sum()
     assert abs(out["loss_total"].item() - L_host) <= 1e-5 * abs(L_host)
     dW = torch.zeros(wl.d, wl.V, device="cuda")
-    dH = gpu_topk_backward(params, Hd, W, lab, out, dW)
+    if keep:
+        G_dev = Zd.view(torch.bfloat16)
+        alr.alr_topk_logit_grad_from_logits(params, Zd, lab["idx"], lab["prob"], lab["tail"],
+                                            out["weight"], out["weight_sum"], out["lse_d"],
+                                            out["tail_q"], G_dev)
+        dH = torch.empty(wl.N, wl.d, device="cuda")
+        alr.alr_gemm(G_dev, W, dH, wl.N, wl.d, wl.V)
+        alr.alr_gemm(Hd, G_dev, dW, wl.d, wl.V, wl.N, a_mn=True, b_mn=True, accumulate=True)
+        torch.cuda.synchronize()
+    else:
+        dH = gpu_topk_backward(params, Hd, W, lab, out, dW)
     G = orc.top_k_logit_grad(z_d, r["idx"], r["prob"], r["tail"], w_all[rows], 1.0,
                              weight_sum=w_all.sum())
     assert P.max_norm_rel(P.np64(dH)[rows], G @ W64.T) <= P.GRAD_RTOL
@@ -222,3 +245,83 @@ def test_text8b_full_batch_compact_labels():
     rhs = torch.sum(dH * Hd.float(), dtype=torch.float64).item()
     assert abs(lhs - rhs) <= 1e-3 * abs(rhs)
     assert alr.alr_device_status() == alr.ALR_OK
+
+
+# ------------------------------------------------------------------ kept logits ---
+@pytest.mark.parametrize("dtype,shape,use_weight", [(torch.bfloat16, (10, 16, 200, 1000), False),
+                                                    (torch.bfloat16, (10, 16, 200, 1000), True),
+                                                    (torch.float32, (64, 8, 256, 4096), False),
+                                                    (torch.bfloat16, (16, 16, 1024, 40000), False)])
+def test_topk_keep_logits_forward_backward(dtype, shape, use_weight):
+    """The kept-logits top-k path: forward outputs bit-identical to the plain forward, the kept
+    z_d within its storage rounding of the oracle's, and G (written over z_d), dH and dW from
+    the kept logits against the oracle; masked rows get G = 0."""
+    A, B, d, V = shape
+    lam = 1.013441
+    b = synthetic.slot_batch(d, V, A, B, 0.5, dtype=dtype, device="cuda", seed=9 + V)
+    N = A * B
+    Hd, Ht, W = b["Hd"], b["Ht"], b["W"]
+    lab_r = orc.label_readout(P.np64(Ht), P.np64(W), k=K)
+    lab = device_labels(lab_r)
+    mask = torch.ones(N, device="cuda")
+    mask[3::B] = 0.0
+    win = (torch.rand(N, generator=torch.Generator().manual_seed(3)) * mask.cpu()).cuda() if use_weight else None
+    kw = dict(row_mask=None if use_weight else mask, weight_in=win, lam=lam)
+    _, plain = gpu_topk_forward(Hd, W, B, lab, **kw)
+    Zd = torch.empty(N, V, dtype=alr.logits_dtype(dtype), device="cuda")
+    params, out = gpu_topk_forward(Hd, W, B, lab, Zd=Zd, **kw)
+    for k in plain:
+        a, c = plain[k].cpu(), out[k].cpu()
+        assert torch.equal(a.view(torch.int32), c.view(torch.int32)), k
+    idx, prob, tail = host_labels(lab)
+    z_d = P.np64(Hd) @ P.np64(W)
+    tol = (2.0 ** -11 * np.abs(z_d) + 1e-4) if dtype == torch.bfloat16 else (2.0 ** -8 * np.abs(z_d) + 4e-3)
+    assert np.all(np.abs(P.np64(Zd) - z_d) <= tol)
+    w_r = P.np64(win) if use_weight else orc.slot_weights(orc.MODE_ALR, B, 2.0, N, row_mask=P.np64(mask))
+    G = Zd.view(dtype)
+    dH = torch.empty(N, d, device="cuda")
+    dW = torch.zeros(d, V, device="cuda")
+    ws = torch.empty(max(alr.alr_bwd_from_logits_workspace_size(params), 16), dtype=torch.uint8,
+                     device="cuda")
+    alr.alr_topk_loss_bwd_from_logits(params, Hd, W, Zd, lab["idx"], lab["prob"], lab["tail"],
+                                      out["weight"], out["weight_sum"], out["lse_d"], out["tail_q"],
+                                      G, dH, dW, ws)
+    torch.cuda.synchronize()
+    G_r = orc.top_k_logit_grad(z_d, idx, prob, tail, w_r, lam)
+    assert P.max_norm_rel(P.np64(G), G_r) <= P.GRAD_RTOL
+    dH_r, dW_r = orc.slot_loss_backward(P.np64(Hd), P.np64(W), G_r)
+    assert P.max_norm_rel(P.np64(dH), dH_r) <= P.GRAD_RTOL
+    assert P.max_norm_rel(P.np64(dW), dW_r) <= P.GRAD_RTOL
+    if not use_weight:
+        assert np.all(P.np64(G)[3::B] == 0)
+    assert alr.alr_device_status() == alr.ALR_OK
+
+
+def test_topk_logit_grad_from_logits_elementwise():
+    """G from oracle-made fp16 logits and labels against the oracle element by element (bf16
+    output rounding 2^-8 relative, plus the fp32 exponentials), in place over z_d; the label
+    tokens of each row, the tail factor and a masked row included."""
+    N, B, V, lam = 32, 16, 5000, 0.9
+    g = torch.Generator().manual_seed(21)
+    Zd = (torch.randn(N, V, generator=g) * 2.0).half()
+    zd = Zd.double().numpy()
+    lab = random_labels(N, V, seed=22)
+    w = orc.slot_weights(orc.MODE_ALR, B, 2.0, N)
+    w[5] = 0.0
+    lse = orc.log_sum_exp(zd)
+    q = orc.softmax(zd)
+    tail_q = 1.0 - np.take_along_axis(q, lab["idx"], axis=1).sum(axis=1)
+    ref = orc.top_k_logit_grad(zd, lab["idx"], lab["prob"], lab["tail"], w, lam)
+    params = alr.make_params(N, 64, V, B, torch.bfloat16, lam=lam)
+    f32 = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float32)).cuda()  # noqa: E731
+    zd_dev = Zd.cuda()
+    dl = device_labels(lab)
+    G = zd_dev.view(torch.bfloat16)
+    alr.alr_topk_logit_grad_from_logits(params, zd_dev, dl["idx"], dl["prob"], dl["tail"], f32(w),
+                                        f32([w.sum()]), f32(lse), f32(tail_q), G)
+    torch.cuda.synchronize()
+    got = P.np64(G)
+    c = lam * w / w.sum()
+    tol = 2.0 ** -8 * np.abs(ref) + 1e-5 * c[:, None] * (q + 1e-3)
+    assert np.all(np.abs(got - ref) <= tol), np.abs(got - ref).max()
+    assert np.all(got[5] == 0)
