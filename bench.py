@@ -48,8 +48,11 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-anchors", type=int, default=1)
+    ap.add_argument("--step", choices=["keep", "recompute"], default="keep",
+                    help="the timed step: the forward keeps the logits for the backward (default), "
+                         "or the backward recomputes them; the other one is timed beside it")
     ap.add_argument("--no-recompute", action="store_true",
-                    help="skip the measurement of the step that recomputes the logits")
+                    help="skip the measurement of the other step variant")
     ap.add_argument("--no-topk", action="store_true",
                     help="skip the compact-label (top-8 + tail) step measurement")
     ap.add_argument("--anchors", type=int, default=0,
@@ -363,11 +366,12 @@ def check_device_status(what):
         raise RuntimeError(f"{what}: device status: {alr.alr_last_error()}")
 
 
-def time_recompute(wl, x, device, K, warmup):
-    """The step whose backward recomputes both head products instead of reading kept logits
-    (12 NdV tensor flops, no logit storage)."""
+def time_variant(wl, x, device, K, warmup, keep):
+    """The other step variant, timed beside the headline one: keep=False, the backward
+    recomputes both head products (12 NdV tensor flops, no logit storage); keep=True, the
+    forward keeps the logits (8 NdV)."""
     import torch
-    st = Step(wl, x, device, keep=False)
+    st = Step(wl, x, device, keep=keep)
     for _ in range(warmup):
         st.run()
     torch.cuda.synchronize()
@@ -383,9 +387,11 @@ def time_recompute(wl, x, device, K, warmup):
     NdV = wl.N * wl.d * wl.V
     phase = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
              for i, p in enumerate(Step.PHASES)}
-    out = {"what": "same step, logits recomputed by the backward (nothing kept)",
-           "ms_per_step": ms, "rows_per_s": wl.N / (ms / 1e3),
-           "executed_tflops_12NdV": 12 * NdV / (ms / 1e3) / 1e12, "phase_ms": phase,
+    what = ("same step, logits kept by the forward for the backward" if keep else
+            "same step, logits recomputed by the backward (nothing kept)")
+    out = {"what": what, "ms_per_step": ms, "rows_per_s": wl.N / (ms / 1e3),
+           ("executed_tflops_8NdV" if keep else "executed_tflops_12NdV"):
+               (8 if keep else 12) * NdV / (ms / 1e3) / 1e12, "phase_ms": phase,
            "gpu_launches": Step.KERNELS_PER_STEP * K, "loss": st.sl.out["loss_total"].item()}
     del st
     torch.cuda.empty_cache()
@@ -438,7 +444,8 @@ def run_gpu(args, rank, world, local_rank):
         import dataclasses
         wl = dataclasses.replace(wl, A=args.anchors, S=max(1, args.anchors // 128))
     x = make_inputs(wl, args.sigma, device, seed=rank)
-    step = Step(wl, x, device)
+    keep = args.step == "keep"
+    step = Step(wl, x, device, keep=keep)
     for _ in range(args.warmup):
         step.run()
     torch.cuda.synchronize()
@@ -508,8 +515,8 @@ def run_gpu(args, rank, world, local_rank):
 
     gather = gather_bandwidth(device) if rank == 0 else None
     topk = time_topk(step, K, args.warmup) if (rank == 0 and not args.no_topk) else None
-    recompute = (time_recompute(wl, x, device, K, args.warmup)
-                 if (rank == 0 and not args.no_recompute) else None)
+    other = (time_variant(wl, x, device, K, args.warmup, keep=not keep)
+             if (rank == 0 and not args.no_recompute) else None)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -526,8 +533,11 @@ def run_gpu(args, rank, world, local_rank):
     ms_step = total_ms / K
     rows_per_s = job_rows_per_s(world, wl.N, K, total_ms)
     algo_tf = 8 * NdV / (ms_step / 1e3) / 1e12
+    exec_tf = (8 if keep else 12) * NdV / (ms_step / 1e3) / 1e12
     # dominant kernel by measured time (the tensor-core phases); its flops per launch
     flops = {"fwd": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
+    if not keep:
+        flops["logit_grad"] = 4 * NdV
     # the logit gradient from kept logits streams z_d, z_t (fp16) in and G (bf16) out
     g_bytes = 6 * wl.N * wl.V
     dom = max(flops, key=lambda p: phase_ms[p])
@@ -540,21 +550,22 @@ def run_gpu(args, rank, world, local_rank):
                                f"sigma={args.sigma} feature buffer {wl.S}x{wl.L}",
                    "global_batch_rows": world * wl.N, "l2": "inputs larger than L2 "
                    "(W 1.24 GB, H 268 MB each, kept logits 2 x 10 GB)", "parallelism": f"replicas{world}"},
-        "tensor_tflops": {"executed_8NdV": algo_tf, "algorithmic_8NdV": algo_tf,
-                          "pct_peak_executed": algo_tf / pk["bf16"],
+        "tensor_tflops": {"executed": exec_tf, "algorithmic_8NdV": algo_tf,
+                          "pct_peak_executed": exec_tf / pk["bf16"],
                           "pct_peak_algorithmic": algo_tf / pk["bf16"],
                           "peak_tflops": pk["bf16"], "peak_source": pk["source"]},
         "phase_ms": phase_ms,
         "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved,
                      "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
                      "frac": achieved / pk["bf16_sustained"],
-                     "frac_of_burst_peak": achieved / pk["bf16"], "traffic": kernel_traffic(dom),
+                     "frac_of_burst_peak": achieved / pk["bf16"], "traffic": kernel_traffic(dom if keep else dom + "_recompute"),
                      "peak_note": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
                      "flops_per_launch": flops[dom]},
-        "logit_grad_hbm": {"bytes": g_bytes, "GB/s": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9,
-                           "frac_of_hbm": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9 / pk["hbm"],
-                           "traffic": kernel_traffic("logit_grad")},
-        "recompute": recompute,
+        "logit_grad_hbm": ({"bytes": g_bytes, "GB/s": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9,
+                            "frac_of_hbm": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9 / pk["hbm"],
+                            "traffic": kernel_traffic("logit_grad")} if keep else None),
+        "step": "forward keeps the logits" if keep else "backward recomputes the logits",
+        ("recompute" if keep else "keep"): other,
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
         "compact_labels": topk,
