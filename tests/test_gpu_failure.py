@@ -24,7 +24,12 @@ def _lib():
     assert alr.alr_device_supported() == alr.ALR_OK, alr.alr_last_error()
 
 
-def test_withheld_stage_times_out_and_context_survives():
+@pytest.mark.parametrize("form", ["single", "mcast"])
+def test_withheld_stage_times_out_and_context_survives(form, monkeypatch):
+    """Both forms of the fused kernel: single CTAs, and clusters of two CTAs that feed each
+    other's stages by multicast (every CTA of the cluster then runs out on its own barriers
+    and both meet at the closing cluster barrier)."""
+    monkeypatch.setenv("ALR_LOSS_FORM", form)
     A, B, d, V = 16, 16, 256, 1024
     b = synthetic.slot_batch(d, V, A, B, 0.5, dtype=torch.bfloat16, device="cuda", seed=9)
     sl = alr.SlotLoss(A * B, d, V, B)
