@@ -233,7 +233,8 @@ BwdLayout bwd_layout(const alr_params* p, bool with_g = true) {
 // wins: multicast halves the B traffic out of L2 and runs 6 % faster than single CTAs at the
 // same clock and power.  The pair form issues more products per clock but draws more power
 // per product and settles at a clock ~20 % lower.  tf32 products always run on single CTAs.
-enum GemmForm { kGemmSingle = 0, kGemmMcast = 1, kGemmPair = 2 };
+//   "mcast4"  as "mcast" with clusters of four CTAs, each loading a quarter of the B tile.
+enum GemmForm { kGemmSingle = 0, kGemmMcast = 1, kGemmPair = 2, kGemmMcast4 = 3 };
 
 GemmForm gemm_form(int dtype) {
   if (dtype != ALR_BF16) return kGemmSingle;
@@ -241,11 +242,18 @@ GemmForm gemm_form(int dtype) {
   if (v == nullptr) return kGemmMcast;
   if (strcmp(v, "single") == 0) return kGemmSingle;
   if (strcmp(v, "pair") == 0) return kGemmPair;
+  if (strcmp(v, "mcast4") == 0) return kGemmMcast4;
   return kGemmMcast;
 }
 
 // Rows of a K-major B box (B columns loaded by one copy).
-uint32_t gemm_b_rows(int dtype) { return gemm_form(dtype) == kGemmSingle ? 256 : 128; }
+uint32_t gemm_b_rows(int dtype) {
+  switch (gemm_form(dtype)) {
+    case kGemmSingle: return 256;
+    case kGemmMcast4: return 64;
+    default: return 128;
+  }
+}
 
 alr::GemmArgs gemm_plan(int M, int Nc, int K, float* C, int64_t ldc, int sms) {
   alr::GemmArgs g{};
@@ -291,18 +299,21 @@ int launch_gemm(int dt, bool a_mn, bool b_mn, bool acc, const CUtensorMap& ma,
     g.status = alr::device_status_ptr();
     if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
     e = alr::launch_pair_gemm(a_mn, b_mn, acc, ma, mb, g, s);
-  } else if (form == kGemmMcast) {
-    const int pairs = alr::plain_gemm_mc_max_pairs();
-    if (pairs < 1) return fail(ALR_ERR_CUDA, "%s: no CTA cluster of the GEMM fits on this device", what);
-    // 128-row blocks in pairs: n_mb counts pairs, raster groups of 8 pairs
+  } else if (form == kGemmMcast || form == kGemmMcast4) {
+    const int cl = form == kGemmMcast4 ? 4 : 2;
+    const int clusters = alr::plain_gemm_mc_max_clusters(cl);
+    if (clusters < 1)
+      return fail(ALR_ERR_CUDA, "%s: no CTA cluster of the GEMM fits on this device", what);
+    // 128-row blocks in groups of `cl`: n_mb counts groups, raster groups of 16 row blocks
     alr::GemmArgs g = gemm_plan(M, Nc, K, C, ldc, sms);
-    g.n_mb = ((M + 127) / 128 + 1) / 2;
-    g.group_m = g.n_mb < 8 ? g.n_mb : 8;
+    g.n_mb = ((M + 127) / 128 + cl - 1) / cl;
+    const int gm = 16 / cl;
+    g.group_m = g.n_mb < gm ? g.n_mb : gm;
     g.n_tiles = g.n_mb * g.n_nb;
-    g.grid = 2 * (pairs < g.n_tiles ? pairs : g.n_tiles);
+    g.grid = cl * (clusters < g.n_tiles ? clusters : g.n_tiles);
     g.status = alr::device_status_ptr();
     if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-    e = alr::launch_plain_gemm_mc(a_mn, b_mn, acc, ma, mb, g, s);
+    e = alr::launch_plain_gemm_mc(cl, a_mn, b_mn, acc, ma, mb, g, s);
   } else {
     alr::GemmArgs g = gemm_plan(M, Nc, K, C, ldc, sms);
     g.status = alr::device_status_ptr();

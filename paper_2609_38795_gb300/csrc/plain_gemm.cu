@@ -6,11 +6,11 @@
 // a 4-stage TMA pipeline with 128-byte swizzle, persistent CTAs over raster groups of
 // `group_m` row blocks.  Warp roles as in loss_gemm.cu.
 //
-// Multicast form (kMc, bf16): clusters of two CTAs compute the two 128-row tiles 2i, 2i + 1
-// against the same 256 columns of B.  Each CTA loads its own A rows and one 128-column half of
-// the B tile, multicast into both CTAs' stage, so every B byte leaves L2 once per pair; a stage
-// is refilled only after both CTAs' products have read it (both MMA issuers' commits arrive on
-// both CTAs' empty barriers).
+// Multicast form (kMc = 2 or 4 CTAs per cluster, bf16): the CTAs of a cluster compute the
+// 128-row tiles kMc i .. kMc i + kMc - 1 against the same 256 columns of B.  Each CTA loads its
+// own A rows and a 1 / kMc share of the B tile, multicast into every CTA's stage, so every B
+// byte leaves L2 once per cluster; a stage is refilled only after all the cluster's products
+// have read it (every MMA issuer's commit arrives on every CTA's empty barrier).
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -74,26 +74,29 @@ ALR_DEV void load_operand(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, i
   }
 }
 
-// B half of the multicast form: `kExtent` / 2 MN rows starting at half `r`, into the same
-// offsets of both CTAs.
-template <typename Elem, bool kMN, int kExtent>
-ALR_DEV void load_operand_half_mc(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int mn0,
-                                  int kb, int r) {
+// B share of the multicast form: `kExtent` / kParts MN rows starting at share `r`, into the same
+// offsets of every CTA of the cluster.
+template <typename Elem, bool kMN, int kExtent, int kParts>
+ALR_DEV void load_operand_share_mc(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int mn0,
+                                   int kb, int r) {
   using G = Geo<Elem>;
-  constexpr int kHalfExt = kExtent / 2;
+  constexpr int kShare = kExtent / kParts;
+  constexpr uint16_t kMask = uint16_t((1u << kParts) - 1u);
   if constexpr (kMN) {
+    static_assert(kShare % G::kChunkMN == 0, "share of whole 128-byte chunks");
 #pragma unroll
-    for (int c = 0; c < kHalfExt / G::kChunkMN; ++c) {
-      const int cc = r * (kHalfExt / G::kChunkMN) + c;
+    for (int c = 0; c < kShare / G::kChunkMN; ++c) {
+      const int cc = r * (kShare / G::kChunkMN) + c;
       tma_load_2d_mc(dst + cc * G::kChunkBytes, map, bar, mn0 + cc * G::kChunkMN, kb * G::kKE,
-                     0x3);
+                     kMask);
     }
   } else {
-    tma_load_2d_mc(dst + r * kHalfExt * 128, map, bar, kb * G::kKE, mn0 + r * kHalfExt, 0x3);
+    tma_load_2d_mc(dst + r * kShare * 128, map, bar, kb * G::kKE, mn0 + r * kShare, kMask);
   }
 }
 
-template <typename Elem, bool kAMN, bool kBMN, bool kAcc, bool kMc>
+// kMc: CTAs per multicast cluster (0: none).
+template <typename Elem, bool kAMN, bool kBMN, bool kAcc, int kMc>
 __global__ void __launch_bounds__(kThreads, 1)
     plain_gemm_kernel(const __grid_constant__ CUtensorMap tm_a,
                       const __grid_constant__ CUtensorMap tm_b, const GemmArgs args) {
@@ -111,7 +114,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const AbortFlag ab{abort_word, args.status};
-  // kMc: tiles are handed out per cluster, and CTA `rank` takes row block 2 mb + rank
+  // kMc: tiles are handed out per cluster, and CTA `rank` takes row block kMc mb + rank
   const int rank = kMc ? int(cluster_ctarank()) : 0;
   const int t0 = kMc ? int(cluster_id_x()) : int(blockIdx.x);
   const int t_step = kMc ? int(n_clusters_x()) : int(gridDim.x);
@@ -119,7 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&full_bar[i], 1);
-      mbar_init(&empty_bar[i], kMc ? 2 : 1);
+      mbar_init(&empty_bar[i], kMc ? kMc : 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);
@@ -152,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = t0; ok && t < args.n_tiles; t += t_step) {
         int mb, nb;
         decode_tile(args, t, mb, nb);
-        if (kMc) mb = 2 * mb + rank;
+        if (kMc) mb = kMc * mb + rank;
         for (int kb = 0; kb < n_kb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1, ab)) {
             ok = false;
@@ -162,8 +165,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive_expect_tx(&full_bar[stage], kStageBytes);
           load_operand<Elem, kAMN, kBM>(sb, &tm_a, &full_bar[stage], mb * kBM, kb);
           if constexpr (kMc)
-            load_operand_half_mc<Elem, kBMN, kBN>(sb + kABytes, &tm_b, &full_bar[stage], nb * kBN,
-                                                  kb, rank);
+            load_operand_share_mc<Elem, kBMN, kBN, kMc>(sb + kABytes, &tm_b, &full_bar[stage],
+                                                        nb * kBN, kb, rank);
           else
             load_operand<Elem, kBMN, kBN>(sb + kABytes, &tm_b, &full_bar[stage], nb * kBN, kb);
           armed |= 1u << stage;
@@ -202,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 operand_desc<Elem, kBMN>(sa + kABytes, kk), idesc,
                                 (kb > 0 || kk > 0) ? 1u : 0u);
           }
-          if constexpr (kMc) mma_commit_mc(&empty_bar[stage], 0x3);
+          if constexpr (kMc) mma_commit_mc(&empty_bar[stage], uint16_t((1u << kMc) - 1u));
           else mma_commit(&empty_bar[stage]);
           if (++stage == kStages) {
             stage = 0;
@@ -227,7 +230,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int t = t0; t < args.n_tiles; t += t_step) {
       int mb, nb;
       decode_tile(args, t, mb, nb);
-      if (kMc) mb = 2 * mb + rank;
+      if (kMc) mb = kMc * mb + rank;
       if (!warp_wait(&tfull_bar[abuf], aphase, ab)) break;
       tc_fence_after();
       const int m = mb * kBM + q * 32 + lane;
@@ -280,7 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <typename Elem, bool kAMN, bool kBMN, bool kAcc, bool kMc = false>
+template <typename Elem, bool kAMN, bool kBMN, bool kAcc, int kMc = 0>
 cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,
                      cudaStream_t s) {
   auto kern = plain_gemm_kernel<Elem, kAMN, kBMN, kAcc, kMc>;
@@ -294,7 +297,7 @@ cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs&
     cudaLaunchConfig_t cfg{};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.x = kMc;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.gridDim = dim3(unsigned(args.grid));
@@ -330,26 +333,25 @@ cudaError_t dispatch(bool a_mn, bool b_mn, bool acc, const CUtensorMap& a, const
   }
 }
 
-}  // namespace
+size_t plain_gemm_smem_bytes_impl() { return kSmemBytes; }
 
-size_t plain_gemm_smem_bytes(int) { return kSmemBytes; }
-
-int plain_gemm_mc_max_pairs() {
+template <int kMc>
+int max_clusters() {
   static int cached[64] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
   if (cached[dev] > 0) return cached[dev];
-  auto kern = plain_gemm_kernel<__nv_bfloat16, false, false, false, true>;
+  auto kern = plain_gemm_kernel<__nv_bfloat16, false, false, false, kMc>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            int(kSmemBytes)) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg{};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.x = kMc;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.gridDim = dim3(2);
+  cfg.gridDim = dim3(kMc);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.attrs = attr;
@@ -360,20 +362,35 @@ int plain_gemm_mc_max_pairs() {
   return n;
 }
 
-cudaError_t launch_plain_gemm_mc(bool a_mn, bool b_mn, bool acc, const CUtensorMap& a,
-                                 const CUtensorMap& b, const GemmArgs& args, cudaStream_t s) {
+template <int kMc>
+cudaError_t launch_mc(bool a_mn, bool b_mn, bool acc, const CUtensorMap& a, const CUtensorMap& b,
+                      const GemmArgs& args, cudaStream_t s) {
   using E = __nv_bfloat16;
   const int key = (a_mn ? 4 : 0) | (b_mn ? 2 : 0) | (acc ? 1 : 0);
   switch (key) {
-    case 0: return launch_t<E, false, false, false, true>(a, b, args, s);
-    case 1: return launch_t<E, false, false, true, true>(a, b, args, s);
-    case 2: return launch_t<E, false, true, false, true>(a, b, args, s);
-    case 3: return launch_t<E, false, true, true, true>(a, b, args, s);
-    case 4: return launch_t<E, true, false, false, true>(a, b, args, s);
-    case 5: return launch_t<E, true, false, true, true>(a, b, args, s);
-    case 6: return launch_t<E, true, true, false, true>(a, b, args, s);
-    default: return launch_t<E, true, true, true, true>(a, b, args, s);
+    case 0: return launch_t<E, false, false, false, kMc>(a, b, args, s);
+    case 1: return launch_t<E, false, false, true, kMc>(a, b, args, s);
+    case 2: return launch_t<E, false, true, false, kMc>(a, b, args, s);
+    case 3: return launch_t<E, false, true, true, kMc>(a, b, args, s);
+    case 4: return launch_t<E, true, false, false, kMc>(a, b, args, s);
+    case 5: return launch_t<E, true, false, true, kMc>(a, b, args, s);
+    case 6: return launch_t<E, true, true, false, kMc>(a, b, args, s);
+    default: return launch_t<E, true, true, true, kMc>(a, b, args, s);
   }
+}
+
+}  // namespace
+
+size_t plain_gemm_smem_bytes(int) { return plain_gemm_smem_bytes_impl(); }
+
+int plain_gemm_mc_max_clusters(int cluster) {
+  return cluster == 4 ? max_clusters<4>() : max_clusters<2>();
+}
+
+cudaError_t launch_plain_gemm_mc(int cluster, bool a_mn, bool b_mn, bool acc, const CUtensorMap& a,
+                                 const CUtensorMap& b, const GemmArgs& args, cudaStream_t s) {
+  if (cluster == 4) return launch_mc<4>(a_mn, b_mn, acc, a, b, args, s);
+  return launch_mc<2>(a_mn, b_mn, acc, a, b, args, s);
 }
 
 cudaError_t launch_plain_gemm(int dtype, bool a_mn, bool b_mn, bool accumulate,

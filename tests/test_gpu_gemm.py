@@ -32,7 +32,7 @@ def _operands(M, Nc, K, dtype, a_mn, b_mn, seed):
     return A_st, B_st, ref
 
 
-@pytest.mark.parametrize("form", ["single", "mcast", "pair"])
+@pytest.mark.parametrize("form", ["single", "mcast", "mcast4", "pair"])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("a_mn,b_mn", list(itertools.product([False, True], repeat=2)))
 @pytest.mark.parametrize("shape", [(200, 264, 200), (256, 512, 1024), (8, 8, 8),
