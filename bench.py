@@ -54,6 +54,9 @@ def parse_args():
                          "or the backward recomputes them; the other one is timed beside it")
     ap.add_argument("--no-recompute", action="store_true",
                     help="skip the measurement of the other step variant")
+    ap.add_argument("--no-erase", action="store_true",
+                    help="skip the erase-mode steps and the accepted-length histograms at other "
+                         "noise levels")
     ap.add_argument("--no-topk", action="store_true",
                     help="skip the compact-label (top-8 + tail) step measurement")
     ap.add_argument("--anchors", type=int, default=0,
@@ -215,6 +218,23 @@ def time_oracle(wl, inputs, n_anchors, reps, budget_s=30.0):
     return rows * len(times) / sum(times), times
 
 
+def time_oracle_single_thread(sigma, n_anchors):
+    """The oracle on one host core: this script's reference arm in a child process whose BLAS
+    and OpenMP pools are limited to one thread (one step over the same bounded sample)."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               RANK="0", WORLD_SIZE="1")
+    cmd = [sys.executable, os.path.abspath(__file__), "--impl", "reference", "--steps", "1",
+           "--warmup", "0", "--sigma", str(sigma), "--cpu-sample-anchors", str(n_anchors)]
+    try:
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=300)
+        line = [ln for ln in r.stdout.splitlines() if ln.startswith("{")][-1]
+        j = json.loads(line)
+        return {"value": j["value"], "unit": j["unit"], "cores": 1,
+                "seconds": j["ms_per_step"] / 1e3}
+    except (subprocess.SubprocessError, IndexError, ValueError, KeyError) as e:
+        return {"unavailable": f"{type(e).__name__}"}
+
+
 # ------------------------------------------------------------- gather bandwidth ---
 def gather_bandwidth(device, reps=24, warmup=4, n_sets=4):
     """IRA gather at the vl7b shape (512 anchors x 16 rows of d=3584 bf16 from a feature
@@ -273,12 +293,13 @@ class Step:
     PHASES = ["gather", "fwd", "accept_len", "logit_grad", "dH_gemm", "dW_gemm"]
     KERNELS_PER_STEP = 8   # gather, fwd (loss, combine, finalize), accept, logit grad, dH, dW
 
-    def __init__(self, wl, inputs, device, keep=True):
+    def __init__(self, wl, inputs, device, keep=True, mode=0, corpus_tok=None):
         import torch
         from paper_2609_38795_gb300 import alr
         self.alr, self.wl, self.x, self.keep = alr, wl, inputs, keep
+        self.corpus_tok = corpus_tok
         self.sl = alr.SlotLoss(wl.N, wl.d, wl.V, wl.B, dtype=torch.bfloat16, device=device,
-                               keep_logits=keep)
+                               keep_logits=keep, mode=mode)
         self.G = (self.sl.G if keep else
                   torch.empty(wl.N, wl.V, dtype=torch.bfloat16, device=device))
         self.dH = torch.empty(wl.N, wl.d, dtype=torch.float32, device=device)
@@ -290,7 +311,7 @@ class Step:
         rec(0)
         alr.alr_gather_ira_blocks(x["F"], x["seq"], x["pos"], wl.B, x["Ht"], x["row_valid"])
         rec(1)
-        sl.forward(x["Hd"], x["Ht"], x["W"], row_mask=x["row_valid"])
+        sl.forward(x["Hd"], x["Ht"], x["W"], row_mask=x["row_valid"], corpus_tok=self.corpus_tok)
         rec(2)
         sl.accept(active=x["row_valid"])
         rec(3)
@@ -397,6 +418,53 @@ def time_variant(wl, x, device, K, warmup, keep):
     del st
     torch.cuda.empty_cache()
     return out
+
+
+def time_erase(wl, x, device, K, warmup, argmax_t):
+    """The kept-logits step in the erase comparator's modes (Eq. 2): corpus tokens are the
+    greedy target tokens, each replaced with probability 0.2 by a uniform token.  The label rows
+    are the same as in ALR mode, so the difference is the cost of the weighting only."""
+    import torch
+    from paper_2609_38795_gb300 import alr, synthetic
+    mask, rnd = synthetic.corpus_replacement(wl.N, wl.V, 0.2, device=device, seed=3)
+    tok = synthetic.corpus_tokens(argmax_t, mask, rnd)
+    out = {"workload": "erase: as text8b, sigma 0.5, corpus = greedy target token replaced "
+                       "w.p. 0.2"}
+    for name, mode in (("soft", alr.ALR_MODE_ERASE_SOFT), ("hard", alr.ALR_MODE_ERASE_HARD)):
+        st = Step(wl, x, device, keep=True, mode=mode, corpus_tok=tok)
+        for _ in range(warmup):
+            st.run()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(K):
+            st.run()
+        b.record()
+        torch.cuda.synchronize()
+        check_device_status(f"erase ({name}) steps")
+        ms = a.elapsed_time(b) / K
+        out[name] = {"ms_per_step": ms, "rows_per_s": wl.N / (ms / 1e3),
+                     "loss": st.sl.out["loss_total"].item(),
+                     "weight_sum": st.sl.out["weight_sum"].item()}
+        del st
+        torch.cuda.empty_cache()
+    return out
+
+
+def acc_hist_by_sigma(wl, step, device, sigmas):
+    """Accepted-length histogram of one step at other drafter noise levels (the same seeded
+    target features and head; only the drafter's noise scale changes)."""
+    import torch
+    hist = {}
+    x0 = step.x
+    for sg in sigmas:
+        step.x = make_inputs(wl, sg, device, seed=0)
+        step.run()
+        torch.cuda.synchronize()
+        hist[str(sg)] = step.sl.hist.cpu().tolist()
+    step.x = x0
+    torch.cuda.empty_cache()
+    return hist
 
 
 def time_topk(step, K, warmup):
@@ -546,6 +614,12 @@ def run_gpu(args, rank, world, local_rank):
     topk = time_topk(step, K, args.warmup) if (rank == 0 and not args.no_topk) else None
     other = (time_variant(wl, x, device, K, args.warmup, keep=not keep)
              if (rank == 0 and not args.no_recompute) else None)
+    erase = (time_erase(wl, x, device, K, args.warmup, step.sl.out["argmax_t"].clone())
+             if (rank == 0 and not args.no_erase) else None)
+    hist_sigma = None
+    if rank == 0 and not args.no_erase:
+        hist_sigma = acc_hist_by_sigma(wl, step, device, [0.25, 1.0])
+        hist_sigma[str(args.sigma)] = acc_hist
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -553,7 +627,8 @@ def run_gpu(args, rank, world, local_rank):
         cpu = {"value": rps, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                "sample": f"{args.cpu_sample_anchors} anchor(s) x {wl.B} rows of the {WORKLOAD} "
                          f"workload, full d={wl.d} and V={wl.V}, fwd+bwd in fp64, "
-                         f"{len(ts)} repetition(s), {sum(ts):.1f} s"}
+                         f"{len(ts)} repetition(s), {sum(ts):.1f} s",
+               "single_thread": time_oracle_single_thread(args.sigma, args.cpu_sample_anchors)}
     if rank != 0:
         return None
 
@@ -584,6 +659,8 @@ def run_gpu(args, rank, world, local_rank):
                           "pct_peak_algorithmic": algo_tf / pk["bf16"],
                           "peak_tflops": pk["bf16"], "peak_source": pk["source"]},
         "phase_ms": phase_ms,
+        "fwd": {"rows_per_s": world * wl.N / (phase_ms["fwd"] / 1e3),
+                "tflops_4NdV": 4 * NdV / (phase_ms["fwd"] / 1e3) / 1e12},
         "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved,
                      "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
                      "frac": achieved / pk["bf16_sustained"],
@@ -598,7 +675,8 @@ def run_gpu(args, rank, world, local_rank):
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
         "compact_labels": topk,
-        "loss": loss, "acc_hist": acc_hist,
+        "loss": loss, "acc_hist": acc_hist, "acc_hist_by_sigma": hist_sigma,
+        "erase": erase,
         "clocks": clk,
         "cpu_baseline": cpu,
     }
