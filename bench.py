@@ -82,12 +82,26 @@ KERNEL_SOURCES = ["paper_2609_38795_gb300/csrc/loss_gemm.cu",
                   "paper_2609_38795_gb300/csrc/kernels.h"]
 
 
-def kernel_sources_sha256():
+def _code_only(text):
+    """Source text without comments and blank space: a change to a comment is no change to the
+    kernel the counters were taken from."""
+    import re
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
+def kernel_sources_sha256(read=None):
+    """Digest of the kernel sources' code.  `read(rel)` returns a file's text (default: the
+    working tree)."""
     import hashlib
+    if read is None:
+        def read(rel):
+            with open(os.path.join(ROOT, rel), encoding="utf-8") as f:
+                return f.read()
     h = hashlib.sha256()
     for rel in KERNEL_SOURCES:
-        with open(os.path.join(ROOT, rel), "rb") as f:
-            h.update(f.read())
+        h.update(_code_only(read(rel)).encode())
     return h.hexdigest()
 
 

@@ -345,7 +345,7 @@ ALR_DEV void keep_logits_f32(const uint32_t (&r)[16], void* base, size_t off, in
     if (4 * i < nv) __stcs(p + i, make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]));
 }
 
-// Warp-uniform bounded wait: lane 0 waits, the verdict is broadcast.
+// Warp-uniform bounded wait: lane 0 waits and broadcasts the outcome.
 ALR_DEV bool warp_wait(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
   int ok = 1;
   if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, ab) ? 1 : 0;
