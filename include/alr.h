@@ -25,6 +25,12 @@
  *              on on-chip pipelines give up after a bounded time and record ALR_ERR_TIMEOUT
  *              in a per-device status word that alr_device_status() reads.
  *   Inputs.    Outputs are unspecified when the inputs contain NaN or Inf.
+ *   Kernel forms (environment, read at every call; results do not depend on them except for
+ *              floating-point rounding of the GEMMs, and the loss kernels' outputs not at all):
+ *              ALR_GEMM_FORM = mcast (default: clusters of two CTAs share each B tile by TMA
+ *              multicast) | single | mcast4 | pair (CTA pairs with M = 256 tcgen05 products)
+ *              selects the bf16 GEMM kernel; ALR_LOSS_FORM = single (default) | mcast selects
+ *              the fused loss kernels' form.  fp32 (tf32) products always run on single CTAs.
  */
 #ifndef ALR_H
 #define ALR_H
