@@ -153,19 +153,22 @@ bool loss_multicast(const alr_params* p) {
   return v != nullptr && strcmp(v, "mcast") == 0;
 }
 
-alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
+// two_rows: the single-operand modes (readout, top-k), whose units hold two row blocks.
+alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd, bool two_rows = false) {
   alr::LossPlan P{};
   P.N = int(p->N);
   P.d = p->d;
   P.V = p->V;
   P.B = p->B;
   P.bn = ALR_LOSS_BN;
-  P.mc = loss_multicast(p) ? 1 : 0;
-  // row blocks, or row-block pairs for the multicast form (which places sms / 2 clusters)
+  P.mc = (!two_rows && loss_multicast(p)) ? 1 : 0;
+  // row blocks; row-block pairs for the two-row modes and for the multicast form (which
+  // places sms / 2 clusters); raster groups of 8 row blocks either way
   const int rb = int((p->N + 127) / 128);
-  P.n_rb = P.mc ? (rb + 1) / 2 : rb;
+  const bool pairs = P.mc || two_rows;
+  P.n_rb = pairs ? (rb + 1) / 2 : rb;
   const int slots = P.mc ? sms / 2 : sms;
-  const int group = P.mc ? 4 : 8;
+  const int group = pairs ? 4 : 8;
   P.n_vt = (p->V + P.bn - 1) / P.bn;
   P.group_rows = P.n_rb < group ? P.n_rb : group;
   if (bwd) {
@@ -175,7 +178,8 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd) {
     if (vs < 1) vs = 1;
     P.n_vs = vs < P.n_vt ? vs : P.n_vt;
   }
-  P.n_parts = P.n_vs * (P.bn / 64);
+  // partial records per row and split: one per epilogue column group
+  P.n_parts = P.n_vs * (P.bn / (two_rows ? 128 : 64));
   P.n_units = P.n_rb * P.n_vs;
   P.grid = sms < P.n_units ? sms : P.n_units;
   return P;
@@ -189,8 +193,9 @@ struct FwdLayout {
   size_t part_off, anchor_off, wt_off, total;
 };
 
-FwdLayout fwd_layout(const alr_params* p, int sms, int fields = alr::kPFields) {
-  const alr::LossPlan P = loss_plan(p, sms, false);
+FwdLayout fwd_layout(const alr_params* p, int sms, int fields = alr::kPFields,
+                     bool two_rows = false) {
+  const alr::LossPlan P = loss_plan(p, sms, false, two_rows);
   FwdLayout L{};
   L.part_off = 0;
   L.anchor_off = round_up(size_t(fields) * P.n_parts * size_t(P.N) * sizeof(float), 1024);
@@ -543,7 +548,7 @@ int logit_grad_impl(const alr_params* p, const void* Hd, const void* Ht, const v
       (rc = make_map(&m_gs, G, dt, p->V, p->N, p->V * es, 16, 32, CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
     return rc;
   alr::LossArgs args{};
-  args.plan = loss_plan(p, info.sms, true);
+  args.plan = loss_plan(p, info.sms, true, topk);
   args.G = G;
   args.lse_d = lse_d;
   args.lse_t = lse_t;
@@ -720,7 +725,7 @@ size_t alr_readout_workspace_size(const alr_params* p) {
   if (check_params(p) != ALR_OK) return 0;
   DevInfo info;
   if (device_info(&info) != ALR_OK) return 0;
-  return fwd_layout(p, info.sms, alr::kRFields).total;
+  return fwd_layout(p, info.sms, alr::kRFields, true).total;
 }
 
 int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
@@ -737,7 +742,7 @@ int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
     return fail(ALR_ERR_INVALID_ARG, "Ht and W must be 16-byte aligned");
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  const FwdLayout lay = fwd_layout(p, info.sms, alr::kRFields);
+  const FwdLayout lay = fwd_layout(p, info.sms, alr::kRFields, true);
   if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
   const int dt = p->dtype;
   const size_t es = elem_size(dt);
@@ -747,7 +752,7 @@ int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
   if ((rc = make_map(&m_h, Ht, dt, p->d, p->N, p->d * es, k_per_row(dt), 128)) != ALR_OK) return rc;
   if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
   alr::LossArgs args{};
-  args.plan = loss_plan(p, info.sms, false);
+  args.plan = loss_plan(p, info.sms, false, true);
   args.part = reinterpret_cast<float*>(ws + lay.part_off);
   args.corpus_tok = corpus_tok;
   args.status = alr::device_status_ptr();
@@ -764,7 +769,7 @@ size_t alr_topk_fwd_workspace_size(const alr_params* p) {
   if (check_params(p) != ALR_OK) return 0;
   DevInfo info;
   if (device_info(&info) != ALR_OK) return 0;
-  return fwd_layout(p, info.sms, alr::kKFields).total;
+  return fwd_layout(p, info.sms, alr::kKFields, true).total;
 }
 
 }  // extern "C"
@@ -787,7 +792,7 @@ int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int3
     return fail(ALR_ERR_INVALID_ARG, "Hd and W must be 16-byte aligned");
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  const FwdLayout lay = fwd_layout(p, info.sms, alr::kKFields);
+  const FwdLayout lay = fwd_layout(p, info.sms, alr::kKFields, true);
   if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
   const int dt = p->dtype;
   const size_t es = elem_size(dt);
@@ -797,7 +802,7 @@ int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int3
   if ((rc = make_map(&m_h, Hd, dt, p->d, p->N, p->d * es, k_per_row(dt), 128)) != ALR_OK) return rc;
   if ((rc = head_map(&m_w, p, W, ws + lay.wt_off, s)) != ALR_OK) return rc;
   alr::LossArgs args{};
-  args.plan = loss_plan(p, info.sms, false);
+  args.plan = loss_plan(p, info.sms, false, true);
   args.part = reinterpret_cast<float*>(ws + lay.part_off);
   args.top_idx = top_idx;
   args.zd_out = Zd;

@@ -20,13 +20,16 @@
 //   kModeTopkBwd z_d only, recomputed: the gradient of that loss;
 //   kModeTopkFwdKeep  kModeTopkFwd that also writes z_d (fp16 for bf16 inputs, fp32 else).
 //
-// Accumulators: the dual modes use 2 x kBN TMEM columns per tile (single-buffered at kBN =
-// 256), the single-operand modes kBN columns (double-buffered, so their epilogue overlaps the
-// next tile's products).
+// Accumulators: 2 x kBN TMEM columns per tile (single-buffered at kBN = 256).  The dual modes
+// hold z_d and z_t of one 128-row block; the single-operand modes (readout, top-k) hold one
+// logit tile of each of two row blocks (rows 256 i .. 256 i + 255), so that they too read every
+// head tile from shared memory once for two products.
 //
 // Warp roles: warp 0 issues TMA loads, warp 1 owns tensor memory and issues the MMAs from one
 // lane, warps 2.. run the epilogue: warp w reads TMEM lanes 32(w%4)..+31 (one row per thread)
-// and the 64 columns [64 g, 64 g + 64) of the tile, g = (w-2)/4, in 16-column sub-chunks.
+// in 16-column sub-chunks; in the dual modes it takes columns [64 g, 64 g + 64) of both tiles,
+// g = (w-2)/4; in the two-row modes columns [128 h, 128 h + 128) of row block b's tile,
+// b = ((w-2)/4) % 2, h = (w-2)/8.
 // Every pipeline wait is bounded (tc_common.cuh).
 //
 // Multicast form (kMc, bf16 inputs, 256-column tiles): clusters of two CTAs take row blocks
@@ -65,6 +68,8 @@ constexpr bool is_fwd(int mode) { return mode == kModeFwd || mode == kModeFwdKee
 constexpr bool is_dual(int mode) { return is_fwd(mode) || mode == kModeBwd; }
 constexpr bool is_grad(int mode) { return mode == kModeBwd || mode == kModeTopkBwd; }
 constexpr bool is_topk_fwd(int mode) { return mode == kModeTopkFwd || mode == kModeTopkFwdKeep; }
+// Single-operand modes: one product per row block, two row blocks per unit.
+constexpr bool is_two_rows(int mode) { return !is_dual(mode); }
 // Modes whose epilogue writes 16-bit [N, V] tiles through shared staging and TMA stores: the
 // bf16 gradient (two buffers per warp, double-buffered) and the kept fp16 logits (one buffer
 // per logit matrix).  fp32 outputs are written directly.
@@ -74,13 +79,15 @@ constexpr bool is_staged(int mode, int elem_bytes) {
 
 template <int kMode, int kBN, bool kStaged>
 struct Shape {
-  static constexpr int kATiles = is_dual(kMode) ? 2 : 1;
+  static constexpr bool kTwoRows = is_two_rows(kMode);
+  static constexpr int kATiles = 2;                    // (H_d, H_t) or two row blocks of H
   static constexpr int kBTileBytes = kBN * 128;
   static constexpr int kStageBytes = kATiles * kATileBytes + kBTileBytes;
-  static constexpr int kAccCols = kATiles * kBN;       // z_d columns, then z_t columns
+  static constexpr int kAccCols = kATiles * kBN;       // first tile's columns, then the second's
   static constexpr int kAccBufs = 512 / kAccCols;
-  static constexpr int kColGroups = kBN / kColsPerWarp;
-  static constexpr int kEpiWarps = 4 * kColGroups;
+  static constexpr int kWarpCols = kTwoRows ? 2 * kColsPerWarp : kColsPerWarp;
+  static constexpr int kColGroups = kBN / kWarpCols;   // partial records per row and split
+  static constexpr int kEpiWarps = 4 * (kBN / kColsPerWarp);
   static constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
   static constexpr int kStaging = kStaged ? kEpiWarps * 2 * kGStageBytes : 0;
   static constexpr int kFit = (kSmemBudget - 1024 - kCtrlBytes - kStaging) / kStageBytes;
@@ -447,7 +454,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
   }
   if (threadIdx.x == 32) {
     tma_prefetch_desc(&tm_a0);
-    if (kDual) tma_prefetch_desc(&tm_a1);
+    if (kDual) tma_prefetch_desc(&tm_a1);  // the two-row modes read both tiles from tm_a0
     tma_prefetch_desc(&tm_w);
     if (kStaged) tma_prefetch_desc(&tm_g);
     if (kStaged && kMode == kModeFwdKeep) tma_prefetch_desc(&tm_g2);
@@ -493,9 +500,14 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
             uint8_t* sb = stage_mem + stage * S::kStageBytes;
             uint8_t* sw = sb + S::kATiles * kATileBytes;
             mbar_arrive_expect_tx(&full_bar[stage], S::kStageBytes);
-            tma_load_2d(sb, &tm_a0, &full_bar[stage], kb * G::kKE, rb * kBM);
-            if constexpr (kDual)
+            if constexpr (kDual) {
+              tma_load_2d(sb, &tm_a0, &full_bar[stage], kb * G::kKE, rb * kBM);
               tma_load_2d(sb + kATileBytes, &tm_a1, &full_bar[stage], kb * G::kKE, rb * kBM);
+            } else {  // row blocks 2 rb and 2 rb + 1
+              tma_load_2d(sb, &tm_a0, &full_bar[stage], kb * G::kKE, 2 * rb * kBM);
+              tma_load_2d(sb + kATileBytes, &tm_a0, &full_bar[stage], kb * G::kKE,
+                          (2 * rb + 1) * kBM);
+            }
             if constexpr (kMc) {
               // this CTA's half of the head tile, into both CTAs' stage
               constexpr int kHalfChunks = kBN / G::kChunkMN / 2;
@@ -561,9 +573,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
                        : sdesc_sw128(swb + kk * 32, 16, 1024);
               const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
               mma_issue<G::kTf32>(d_acc, sdesc_sw128(sa + kk * 32, 16, 1024), bd, idesc, acc);
-              if constexpr (kDual)
-                mma_issue<G::kTf32>(d_acc + kBN, sdesc_sw128(sa + kATileBytes + kk * 32, 16, 1024),
-                                    bd, idesc, acc);
+              mma_issue<G::kTf32>(d_acc + kBN, sdesc_sw128(sa + kATileBytes + kk * 32, 16, 1024),
+                                  bd, idesc, acc);
             }
             if constexpr (kMc) mma_commit_mc(&empty_bar[stage], 0x3);
             else mma_commit(&empty_bar[stage]);
@@ -586,10 +597,15 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
     }
   } else {
     // -------------------------------------------------------------------- epilogue ---
+    // a warp may only read the TMEM lane quarter warp % 4; each run of four consecutive
+    // epilogue warps covers the four quarters
     const int q = warp & 3;
-    const int cg = (warp - kEpiWarp0) >> 2;
+    const int e = (warp - kEpiWarp0) >> 2;                  // which run of four warps
+    const int blk = S::kTwoRows ? (e & 1) : 0;              // row block of the unit's pair
+    const int cg = S::kTwoRows ? (e >> 1) : e;              // column group of the tile
     const int row_in_tile = q * 32 + lane;
-    const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(cg * kColsPerWarp);
+    const uint32_t lane_addr = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(blk * kBN) +
+                               uint32_t(cg * S::kWarpCols);
     uint8_t* my_stage = gstage + (warp - kEpiWarp0) * 2 * kGStageBytes;
     uint32_t n_stores = 0;
     int abuf = 0;
@@ -599,6 +615,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
       int rb, vs;
       decode_unit(P, u, rb, vs);
       if (kMc) rb = 2 * rb + rank;
+      if (S::kTwoRows) rb = 2 * rb + blk;
       const int vt1 = split_begin(P, vs + 1);
       const int row = rb * kBM + row_in_tile;
       const bool row_ok = row < P.N;
@@ -653,9 +670,9 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
         }
         tc_fence_after();
         const uint32_t tb = lane_addr + uint32_t(abuf * S::kAccCols);
-        const int vbase = vt * kBN + cg * kColsPerWarp;
+        const int vbase = vt * kBN + cg * S::kWarpCols;
 #pragma unroll 1
-        for (int c = 0; c < kColsPerWarp / kSub; ++c) {
+        for (int c = 0; c < S::kWarpCols / kSub; ++c) {
           uint32_t r0[16], r1[16];
           tmem_ld16(tb + c * kSub, r0);
           if constexpr (kDual) tmem_ld16(tb + kBN + c * kSub, r1);
@@ -871,7 +888,7 @@ cudaError_t by_width(const CUtensorMap& a0, const CUtensorMap& a1, const CUtenso
                      const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
                      cudaStream_t s) {
   if (args.plan.bn == 128) return launch_impl<Elem, kMode, 128, false>(a0, a1, w, g, g2, args, s);
-  if constexpr (sizeof(Elem) == 2) {
+  if constexpr (sizeof(Elem) == 2 && is_dual(kMode)) {
     if (args.plan.mc) return launch_impl<Elem, kMode, 256, true>(a0, a1, w, g, g2, args, s);
   }
   return launch_impl<Elem, kMode, 256, false>(a0, a1, w, g, g2, args, s);

@@ -73,9 +73,12 @@ def compare_readout(g, r, prob_rtol=1e-3):
 
 
 @pytest.mark.parametrize("dtype,shape", [(torch.bfloat16, (10, 16, 200, 1000)),
+                                         (torch.bfloat16, (17, 16, 200, 1000)),
                                          (torch.float32, (64, 8, 256, 4096)),
                                          (torch.bfloat16, (64, 16, 2048, 32000))])
 def test_readout_matches_oracle(dtype, shape):
+    """Row counts of 1.25, 2.1, 4 and 8 row blocks of 128: the readout's units take two row
+    blocks each, so the last unit may hold a partial block or none."""
     A, B, d, V = shape
     b = synthetic.slot_batch(d, V, A, B, 0.5, dtype=dtype, device="cuda", seed=A + V)
     N = A * B
@@ -148,6 +151,7 @@ def host_labels(lab):
 
 @pytest.mark.parametrize("dtype,shape,use_weight", [(torch.bfloat16, (10, 16, 200, 1000), False),
                                                     (torch.bfloat16, (10, 16, 200, 1000), True),
+                                                    (torch.bfloat16, (17, 16, 200, 1000), False),
                                                     (torch.float32, (64, 8, 256, 4096), False)])
 def test_topk_loss_forward_backward(dtype, shape, use_weight):
     A, B, d, V = shape
