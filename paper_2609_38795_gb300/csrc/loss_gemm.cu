@@ -710,16 +710,25 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
             const float cm = max16(z);
             lse_update(m, s, z, cm);
             if constexpr (kMode == kModeReadout) {
-              if (cm > tk[kTopK - 1]) {   // some column of this sub-chunk enters the top k
-#pragma unroll
-                for (int j = 0; j < kSub; ++j)
-                  if (z[j] > tk[kTopK - 1]) topk_insert(tk, ti, z[j], v0 + j);
-              }
               const int xr = x - v0;
               if (xr >= 0 && xr < nv) {
 #pragma unroll
                 for (int j = 0; j < kSub; ++j)
                   if (j == xr) zx = z[j];
+              }
+              // the sub-chunk's entrants, largest first (equal values lowest column first, so
+              // each goes below the equal ones already listed): one pass per entrant instead
+              // of one per column
+              float c = cm;
+#pragma unroll 1
+              while (c > tk[kTopK - 1]) {
+                int jj = kSub - 1;
+#pragma unroll
+                for (int j = kSub - 1; j >= 0; --j) jj = (z[j] == c) ? j : jj;
+                topk_insert(tk, ti, c, v0 + jj);
+#pragma unroll
+                for (int j = 0; j < kSub; ++j) z[j] = (j == jj) ? -INFINITY : z[j];
+                c = max16(z);
               }
             } else {
               top2_update(best, sec, bidx, z, cm, v0);
