@@ -619,6 +619,18 @@ int check_workspace(void* workspace, size_t ws_bytes, size_t need) {
   return ALR_OK;
 }
 
+// Arguments of the dH / dW products of the backward passes from kept logits.
+int check_head_grad_args(const alr_params* p, const void* Hd, const void* W, const float* dHd,
+                         const float* dW, void* workspace, size_t ws_bytes) {
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if (Hd == nullptr || W == nullptr || dHd == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "Hd, W and dHd must be non-NULL");
+  if (!aligned16(Hd) || !aligned16(W) || !aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
+    return fail(ALR_ERR_INVALID_ARG, "Hd, W, dHd and dW must be 16-byte aligned");
+  return check_workspace(workspace, ws_bytes, bwd_layout(p, false).total);
+}
+
 int check_topk_labels(const alr_params* p, const int32_t* idx, const float* prob,
                       const float* tail) {
   if (p->V < alr::kTopK)
@@ -707,18 +719,16 @@ int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
                                   const float* weight_sum, const float* lse_d, const float* lse_t,
                                   void* G, float* dHd, float* dW, void* workspace,
                                   size_t ws_bytes, void* stream) {
-  int rc = alr_logit_grad_from_logits(p, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, stream);
+  // everything is validated before the gradient kernel overwrites anything
+  int rc = check_head_grad_args(p, Hd, W, dHd, dW, workspace, ws_bytes);
   if (rc != ALR_OK) return rc;
-  if (Hd == nullptr || W == nullptr || dHd == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "Hd, W and dHd must be non-NULL");
-  if (!aligned16(Hd) || !aligned16(W) || !aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
-    return fail(ALR_ERR_INVALID_ARG, "Hd, W, dHd and dW must be 16-byte aligned");
-  const BwdLayout lay = bwd_layout(p, false);
-  if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
+  if ((rc = alr_logit_grad_from_logits(p, Zd, Zt, weight, weight_sum, lse_d, lse_t, G,
+                                       stream)) != ALR_OK)
+    return rc;
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  return head_grads_impl(p, Hd, W, G, dHd, dW, static_cast<uint8_t*>(workspace), lay, info,
-                         static_cast<cudaStream_t>(stream));
+  return head_grads_impl(p, Hd, W, G, dHd, dW, static_cast<uint8_t*>(workspace),
+                         bwd_layout(p, false), info, static_cast<cudaStream_t>(stream));
 }
 
 size_t alr_readout_workspace_size(const alr_params* p) {
@@ -875,19 +885,16 @@ int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
                                   const float* tail, const float* weight, const float* weight_sum,
                                   const float* lse_d, const float* tail_q, void* G, float* dHd,
                                   float* dW, void* workspace, size_t ws_bytes, void* stream) {
-  int rc = alr_topk_logit_grad_from_logits(p, Zd, top_idx, top_prob, tail, weight, weight_sum,
-                                           lse_d, tail_q, G, stream);
+  // everything is validated before the gradient kernel overwrites anything
+  int rc = check_head_grad_args(p, Hd, W, dHd, dW, workspace, ws_bytes);
   if (rc != ALR_OK) return rc;
-  if (Hd == nullptr || W == nullptr || dHd == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "Hd, W and dHd must be non-NULL");
-  if (!aligned16(Hd) || !aligned16(W) || !aligned16(dHd) || (dW != nullptr && !aligned16(dW)))
-    return fail(ALR_ERR_INVALID_ARG, "Hd, W, dHd and dW must be 16-byte aligned");
-  const BwdLayout lay = bwd_layout(p, false);
-  if ((rc = check_workspace(workspace, ws_bytes, lay.total)) != ALR_OK) return rc;
+  if ((rc = alr_topk_logit_grad_from_logits(p, Zd, top_idx, top_prob, tail, weight, weight_sum,
+                                            lse_d, tail_q, G, stream)) != ALR_OK)
+    return rc;
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  return head_grads_impl(p, Hd, W, G, dHd, dW, static_cast<uint8_t*>(workspace), lay, info,
-                         static_cast<cudaStream_t>(stream));
+  return head_grads_impl(p, Hd, W, G, dHd, dW, static_cast<uint8_t*>(workspace),
+                         bwd_layout(p, false), info, static_cast<cudaStream_t>(stream));
 }
 
 int alr_topk_logit_grad(const alr_params* p, const void* Hd, const void* W,

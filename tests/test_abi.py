@@ -68,3 +68,16 @@ def test_argument_errors_are_reported_without_a_launch(libalr):
     rc = lib.alr_gather_ira_blocks(None, 1, 8, 12, alr.ALR_BF16, None, None, None, 2, 4, None,
                                    None, None)
     assert rc == alr.ALR_ERR_INVALID_ARG                   # 12 * 2 bytes is not a multiple of 16
+    # the backward passes from kept logits validate dH's arguments before the gradient kernel
+    # would overwrite z_d: a missing dHd is reported before anything else is looked at
+    good = alr.make_params(N=32, d=64, V=128, B=16)
+    fake = ctypes.c_void_p(1 << 20)                        # never dereferenced on this path
+    rc = lib.alr_slot_loss_bwd_from_logits(ctypes.byref(good), fake, fake, fake, fake, fake,
+                                           fake, fake, fake, fake, None, None, None, 0, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    assert "dHd" in lib.alr_last_error().decode()
+    rc = lib.alr_topk_loss_bwd_from_logits(ctypes.byref(good), fake, fake, fake, fake, fake,
+                                           fake, fake, fake, fake, fake, fake, None, None,
+                                           None, 0, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    assert "dHd" in lib.alr_last_error().decode()
