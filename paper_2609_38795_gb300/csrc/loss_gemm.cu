@@ -37,6 +37,7 @@
 // own hidden-state tiles and one 128-column half of every head tile, multicast into both CTAs'
 // stage, so each W byte leaves L2 once per pair; a stage is refilled only after both CTAs'
 // products have read it.  Under the power cap the saved L2 traffic is saved energy.
+#include <atomic>
 #include <cuda_fp16.h>
 
 #include "kernels.h"
@@ -873,20 +874,22 @@ cudaError_t launch_impl(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
     return cudaGetLastError();
   } else {
     // as many clusters as fit at once (one CTA per SM), at most one per unit
-    static int max_clusters[64] = {0};
+    // per-device, per-kernel occupancy, computed once (concurrent first calls agree)
+    static std::atomic<int> max_clusters[64];
     int dev = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     cudaLaunchAttribute attr[1];
-    if (max_clusters[dev] == 0) {
+    int known = max_clusters[dev].load(std::memory_order_relaxed);
+    if (known == 0) {
       cudaLaunchConfig_t q = cluster2_config(attr, 2, S::kThreads, S::kSmem, s);
       int n = 0;
       if ((e = cudaOccupancyMaxActiveClusters(&n, kern, &q)) != cudaSuccess) return e;
       if (n < 1) return cudaErrorInvalidConfiguration;
-      max_clusters[dev] = n;
+      max_clusters[dev].store(n, std::memory_order_relaxed);
+      known = n;
     }
-    const int clusters = max_clusters[dev] < args.plan.n_units ? max_clusters[dev]
-                                                               : args.plan.n_units;
+    const int clusters = known < args.plan.n_units ? known : args.plan.n_units;
     cudaLaunchConfig_t cfg = cluster2_config(attr, unsigned(2 * clusters), S::kThreads, S::kSmem, s);
     return cudaLaunchKernelEx(&cfg, kern, a0, a1, w, g, g2, args);
   }

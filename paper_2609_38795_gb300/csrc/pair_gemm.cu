@@ -14,6 +14,8 @@
 // barrier); the products' commit releases the stage in both CTAs at once (multicast), and
 // the epilogue warps of both CTAs release an accumulator buffer on the even CTA's barrier.
 // Every wait is bounded (tc_common.cuh).
+#include <atomic>
+
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -289,10 +291,12 @@ cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs&
 size_t pair_gemm_smem_bytes() { return kSmemBytes; }
 
 int pair_gemm_max_pairs() {
-  static int cached[64] = {0};
+  // per-device occupancy, computed once (concurrent first calls compute the same value)
+  static std::atomic<int> cached[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  if (cached[dev] > 0) return cached[dev];
+  const int known = cached[dev].load(std::memory_order_relaxed);
+  if (known > 0) return known;
   auto kern = pair_gemm_kernel<false, false, false>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            int(kSmemBytes)) != cudaSuccess)
@@ -310,7 +314,7 @@ int pair_gemm_max_pairs() {
   cfg.numAttrs = 1;
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) return 0;
-  cached[dev] = n;
+  cached[dev].store(n, std::memory_order_relaxed);
   return n;
 }
 

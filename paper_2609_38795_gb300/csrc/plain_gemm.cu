@@ -11,6 +11,8 @@
 // own A rows and a 1 / kMc share of the B tile, multicast into every CTA's stage, so every B
 // byte leaves L2 once per cluster; a stage is refilled only after all the cluster's products
 // have read it (every MMA issuer's commit arrives on every CTA's empty barrier).
+#include <atomic>
+
 #include "kernels.h"
 #include "tc_common.cuh"
 
@@ -337,10 +339,12 @@ size_t plain_gemm_smem_bytes_impl() { return kSmemBytes; }
 
 template <int kMc>
 int max_clusters() {
-  static int cached[64] = {0};
+  // per-device occupancy, computed once (concurrent first calls compute the same value)
+  static std::atomic<int> cached[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  if (cached[dev] > 0) return cached[dev];
+  const int known = cached[dev].load(std::memory_order_relaxed);
+  if (known > 0) return known;
   auto kern = plain_gemm_kernel<__nv_bfloat16, false, false, false, kMc>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            int(kSmemBytes)) != cudaSuccess)
@@ -358,7 +362,7 @@ int max_clusters() {
   cfg.numAttrs = 1;
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) return 0;
-  cached[dev] = n;
+  cached[dev].store(n, std::memory_order_relaxed);
   return n;
 }
 
