@@ -254,8 +254,9 @@ def gather_bandwidth(device, reps=24, warmup=4, n_sets=4):
     """IRA gather at the vl7b shape (512 anchors x 16 rows of d=3584 bf16 from a feature
     buffer [32, 2048, d]).  Inputs larger than L2: the launches cycle through n_sets feature
     buffers and output buffers (4 x 58.7 MB read + 4 x 58.7 MB written per cycle, > L2), so no
-    launch finds its rows in L2; reps back-to-back launches are timed with CUDA events and the
-    mean launch time is reported."""
+    launch finds its rows in L2.  The reps launches are captured once in a CUDA graph and the
+    graph's replay is timed with CUDA events (mean time per launch); the same launches issued
+    one by one from the host are timed beside it (`us_per_launch_stream`)."""
     import torch
     from paper_2609_38795_gb300 import alr, synthetic
     wl = synthetic.WORKLOADS["vl7b"]
@@ -273,19 +274,36 @@ def gather_bandwidth(device, reps=24, warmup=4, n_sets=4):
     torch.cuda.synchronize()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
+
+    def launches():
+        for i in range(reps):
+            F, seq, pos, out, valid = sets[i % n_sets]
+            alr.alr_gather_ira_blocks(F, seq, pos, wl.B, out, valid)
+
     a.record()
-    for i in range(reps):
-        F, seq, pos, out, valid = sets[i % n_sets]
-        alr.alr_gather_ira_blocks(F, seq, pos, wl.B, out, valid)
+    launches()
+    b.record()
+    torch.cuda.synchronize()
+    ms_stream = a.elapsed_time(b) / reps
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        launches()
+    graph.replay()
+    torch.cuda.synchronize()
+    a.record()
+    graph.replay()
     b.record()
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / reps
+    check_device_status("gather")
     nbytes = 2 * wl.N * wl.d * 2 + wl.N * 4       # rows read + rows written + row_valid
     gbs = nbytes / (ms / 1e3) / 1e9
     return {"workload": f"vl7b: {wl.A} anchors x {wl.B} rows, d={wl.d}, feature buffer "
                         f"{wl.S}x{wl.L}", "bytes": nbytes, "us_per_launch": ms * 1e3,
-            "GB/s": gbs, "l2": f"inputs larger than L2 ({n_sets} rotating input/output sets)",
-            "reps": reps}
+            "GB/s": gbs, "us_per_launch_stream": ms_stream * 1e3,
+            "GB/s_stream": nbytes / (ms_stream / 1e3) / 1e9,
+            "l2": f"inputs larger than L2 ({n_sets} rotating input/output sets)",
+            "reps": reps, "timing": "one CUDA graph of reps launches, replayed"}
 
 
 # ------------------------------------------------------------------------ GPU arm ---
