@@ -59,6 +59,9 @@ def parse_args():
                          "noise levels")
     ap.add_argument("--no-topk", action="store_true",
                     help="skip the compact-label (top-8 + tail) step measurement")
+    ap.add_argument("--gather-only", action="store_true",
+                    help="profiling only: run just the IRA gather measurement and print its "
+                         "result (no step, a little over 2 GB of device memory)")
     ap.add_argument("--anchors", type=int, default=0,
                     help="profiling only: fewer anchors than the workload (config says so)")
     return ap.parse_args()
@@ -762,6 +765,18 @@ def main():
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args)), flush=True)
+        return
+    if args.gather_only:
+        import torch
+        from paper_2609_38795_gb300 import alr, build_lib
+        torch.cuda.set_device(local_rank)
+        build_lib.build()
+        alr.lib()
+        if rank == 0:
+            g = gather_bandwidth(f"cuda:{local_rank}")
+            pk = peaks()
+            print(json.dumps({"ira_gather": dict(g, frac_of_hbm=g["GB/s"] / pk["hbm"],
+                                                  hbm_peak_gbs=pk["hbm"])}), flush=True)
         return
     if world > 1:
         import torch
