@@ -486,6 +486,13 @@ def time_erase(wl, x, device, K, warmup, argmax_t):
     return out
 
 
+def mean_accepted_tokens(hist):
+    """MAT of Sec. 4: the mean over anchors of (accepted slots + 1), from a histogram whose
+    entry n counts the anchors with n accepted slots."""
+    total = sum(hist)
+    return None if total == 0 else 1.0 + sum(n * c for n, c in enumerate(hist)) / total
+
+
 def acc_hist_by_sigma(wl, step, device, sigmas):
     """Accepted-length histogram of one step at other drafter noise levels (the same seeded
     target features and head; only the drafter's noise scale changes)."""
@@ -711,6 +718,10 @@ def run_gpu(args, rank, world, local_rank):
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
         "compact_labels": topk,
         "loss": loss, "acc_hist": acc_hist, "acc_hist_by_sigma": hist_sigma,
+        # mean accepted length per anchor + 1: the tokens a verification round yields (MAT)
+        "mat": mean_accepted_tokens(acc_hist),
+        "mat_by_sigma": (None if hist_sigma is None else
+                         {sg: mean_accepted_tokens(h) for sg, h in hist_sigma.items()}),
         "erase": erase,
         "clocks": clk,
         "cpu_baseline": cpu,
