@@ -9,6 +9,8 @@
 #include <cstring>
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "alr.h"
 #include "kernels.h"
 
@@ -29,6 +31,17 @@ int cuda_fail(cudaError_t e, const char* what) {
 }
 
 std::mutex g_mu;
+
+// Every compute entry point opens an NVTX range named after itself, so a profiler attached to
+// the process shows each call as a span on the host timeline (and ncu can filter launches by
+// it).  With no tool attached, push and pop return after one branch each.
+struct Range {
+  explicit Range(const char* name) { nvtxRangePushA(name); }
+  ~Range() { nvtxRangePop(); }
+  Range(const Range&) = delete;
+  Range& operator=(const Range&) = delete;
+};
+#define ALR_RANGE() const Range alr_nvtx_range_(__func__)
 
 // Test hook state: when set, the next forward launch withholds its first pipeline stage.
 std::atomic<int> g_withhold_next{0};
@@ -452,6 +465,7 @@ int alr_device_status(void* stream, int clear) {
 int alr_gather_ira_blocks(const void* feat, int32_t S, int32_t L, int32_t d, int32_t dtype,
                           const int32_t* seq, const int32_t* pos, const int32_t* valid_len,
                           int32_t A, int32_t B, void* out, float* row_valid, void* stream) {
+  ALR_RANGE();
   if (dtype != ALR_BF16 && dtype != ALR_F32) return fail(ALR_ERR_UNSUPPORTED, "dtype %d", dtype);
   if (S < 1 || L < 1 || d < 1 || A < 0 || B < 1)
     return fail(ALR_ERR_INVALID_ARG, "bad sizes S=%d L=%d d=%d A=%d B=%d", S, L, d, A, B);
@@ -481,6 +495,7 @@ size_t alr_fwd_workspace_size(const alr_params* p) {
 int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const void* W,
                       const float* row_mask, const int32_t* corpus_tok, const alr_fwd_outputs* out,
                       void* workspace, size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, nullptr, nullptr, out, workspace, ws_bytes,
                   stream);
 }
@@ -489,6 +504,7 @@ int alr_slot_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const voi
                                   const void* W, const float* row_mask, const int32_t* corpus_tok,
                                   void* Zd, void* Zt, const alr_fwd_outputs* out, void* workspace,
                                   size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   if (Zd == nullptr || Zt == nullptr)
     return fail(ALR_ERR_INVALID_ARG, "Zd and Zt must be non-NULL");
   if (!aligned16(Zd) || !aligned16(Zt))
@@ -652,6 +668,7 @@ size_t alr_logit_grad_workspace_size(const alr_params* p) {
 int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const void* W,
                    const float* weight, const float* weight_sum, const float* lse_d,
                    const float* lse_t, void* G, void* workspace, size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   DevInfo info;
   int rc = check_bwd_args(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, &info);
   if (rc != ALR_OK) return rc;
@@ -668,6 +685,7 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
                       const float* weight, const float* weight_sum, const float* lse_d,
                       const float* lse_t, float* dHd, float* dW, void* workspace, size_t ws_bytes,
                       void* stream) {
+  ALR_RANGE();
   DevInfo info;
   int rc = check_bwd_args(p, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, &info);
   if (rc != ALR_OK) return rc;
@@ -693,6 +711,7 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
 int alr_logit_grad_from_logits(const alr_params* p, const void* Zd, const void* Zt,
                                const float* weight, const float* weight_sum, const float* lse_d,
                                const float* lse_t, void* G, void* stream) {
+  ALR_RANGE();
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if (Zd == nullptr || Zt == nullptr || G == nullptr || weight == nullptr ||
@@ -719,6 +738,7 @@ int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
                                   const float* weight_sum, const float* lse_d, const float* lse_t,
                                   void* G, float* dHd, float* dW, void* workspace,
                                   size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   // everything is validated before the gradient kernel overwrites anything
   int rc = check_head_grad_args(p, Hd, W, dHd, dW, workspace, ws_bytes);
   if (rc != ALR_OK) return rc;
@@ -742,6 +762,7 @@ int alr_label_readout(const alr_params* p, const void* Ht, const void* W,
                       const int32_t* corpus_tok, int32_t* top_idx, float* top_prob, float* tail,
                       float* lse_t, int32_t* argmax_t, float* gap_t, float* logp_x,
                       void* workspace, size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if (Ht == nullptr || W == nullptr || top_idx == nullptr || top_prob == nullptr || tail == nullptr)
@@ -844,6 +865,7 @@ int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const 
                       const float* top_prob, const float* tail, const float* row_mask,
                       const float* weight_in, const alr_topk_fwd_outputs* out, void* workspace,
                       size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, nullptr, out,
                        workspace, ws_bytes, stream);
 }
@@ -853,6 +875,7 @@ int alr_topk_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const voi
                                   const float* row_mask, const float* weight_in, void* Zd,
                                   const alr_topk_fwd_outputs* out, void* workspace,
                                   size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   if (Zd == nullptr || !aligned16(Zd))
     return fail(ALR_ERR_INVALID_ARG, "Zd must be non-NULL and 16-byte aligned");
   return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, Zd, out,
@@ -863,6 +886,7 @@ int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const i
                                     const float* top_prob, const float* tail, const float* weight,
                                     const float* weight_sum, const float* lse_d,
                                     const float* tail_q, void* G, void* stream) {
+  ALR_RANGE();
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
@@ -885,6 +909,7 @@ int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
                                   const float* tail, const float* weight, const float* weight_sum,
                                   const float* lse_d, const float* tail_q, void* G, float* dHd,
                                   float* dW, void* workspace, size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   // everything is validated before the gradient kernel overwrites anything
   int rc = check_head_grad_args(p, Hd, W, dHd, dW, workspace, ws_bytes);
   if (rc != ALR_OK) return rc;
@@ -902,6 +927,7 @@ int alr_topk_logit_grad(const alr_params* p, const void* Hd, const void* W,
                         const float* weight, const float* weight_sum, const float* lse_d,
                         const float* tail_q, void* G, void* workspace, size_t ws_bytes,
                         void* stream) {
+  ALR_RANGE();
   DevInfo info;
   int rc = check_bwd_args(p, Hd, Hd, W, weight, weight_sum, lse_d, lse_d, &info);
   if (rc != ALR_OK) return rc;
@@ -922,6 +948,7 @@ int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const 
                       const float* top_prob, const float* tail, const float* weight,
                       const float* weight_sum, const float* lse_d, const float* tail_q,
                       float* dHd, float* dW, void* workspace, size_t ws_bytes, void* stream) {
+  ALR_RANGE();
   DevInfo info;
   int rc = check_bwd_args(p, Hd, Hd, W, weight, weight_sum, lse_d, lse_d, &info);
   if (rc != ALR_OK) return rc;
@@ -949,6 +976,7 @@ int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* vali
                    const int32_t* rollout_len, const int32_t* offsets, const int32_t* rollout_tok,
                    const int32_t* corpus_anchor_tok, int32_t* seq, int32_t* pos,
                    int32_t* valid_len, int32_t* ctx_len, int32_t* anchor_tok, void* stream) {
+  ALR_RANGE();
   if (S < 0 || K < 2 || max_blocks < 1)
     return fail(ALR_ERR_INVALID_ARG, "bad sizes S=%d K=%d max_blocks=%d", S, K, max_blocks);
   if (S == 0) return ALR_OK;
@@ -968,6 +996,7 @@ int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* vali
 
 int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,
                    int32_t A, int32_t B, int32_t* acc_len, int64_t* hist, void* stream) {
+  ALR_RANGE();
   if (A < 0 || B < 1 || B > 32) return fail(ALR_ERR_INVALID_ARG, "bad sizes A=%d B=%d", A, B);
   if (A > 0 && (argmax_d == nullptr || argmax_t == nullptr || acc_len == nullptr))
     return fail(ALR_ERR_INVALID_ARG, "argmax_d, argmax_t and acc_len must be non-NULL");
@@ -984,6 +1013,7 @@ int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float
 int alr_erase_weights(const float* logp_x, const int32_t* corpus_tok, const int32_t* argmax_t,
                       const float* row_mask, int32_t A, int32_t B, float gamma, int32_t hard,
                       float* weight, void* stream) {
+  ALR_RANGE();
   if (A < 0 || B < 1 || B > 32) return fail(ALR_ERR_INVALID_ARG, "bad sizes A=%d B=%d", A, B);
   if (!(gamma > 0.f)) return fail(ALR_ERR_INVALID_ARG, "gamma must be > 0");
   if (A == 0) return ALR_OK;
@@ -1002,6 +1032,7 @@ int alr_erase_weights(const float* logp_x, const int32_t* corpus_tok, const int3
 
 int alr_gemm(int32_t dtype, int32_t a_mn, int32_t b_mn, int32_t accumulate, const void* A,
              const void* B, float* C, int32_t M, int32_t Nc, int32_t K, void* stream) {
+  ALR_RANGE();
   if (dtype != ALR_BF16 && dtype != ALR_F32) return fail(ALR_ERR_UNSUPPORTED, "dtype %d", dtype);
   if (M < 1 || Nc < 1 || K < 1) return fail(ALR_ERR_INVALID_ARG, "bad sizes M=%d Nc=%d K=%d", M, Nc, K);
   if (A == nullptr || B == nullptr || C == nullptr)
