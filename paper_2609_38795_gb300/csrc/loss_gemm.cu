@@ -48,6 +48,7 @@ namespace {
 
 constexpr int kBM = 128;                 // rows per tile = TMEM lanes
 constexpr int kEpiWarp0 = 2;
+constexpr int kEpiBarrier = 1;           // named barrier of the epilogue warps (0 is __syncthreads)
 constexpr int kColsPerWarp = 64;
 constexpr int kSub = 16;                 // columns per TMEM load / processing step
 constexpr int kATileBytes = kBM * 128;   // a 128-row operand over 128 bytes of K
@@ -95,8 +96,8 @@ struct Shape {
   static constexpr int kStages = kFit < 4 ? kFit : 4;
   static constexpr size_t kSmem = 1024 + size_t(kStages) * kStageBytes + kStaging + kCtrlBytes;
   // control block: full / empty barrier per stage, full / empty per accumulator buffer, the
-  // drain barrier, the TMEM address and the abort word
-  static_assert((2 * kStages + 2 * kAccBufs + 1) * 8 + 8 <= kCtrlBytes, "control block");
+  // drain barrier, the TMEM address, the abort word and the epilogue's two tile-ready words
+  static_assert((2 * kStages + 2 * kAccBufs + 1) * 8 + 16 <= kCtrlBytes, "control block");
 };
 
 // Unit u -> (row block, vocabulary split).  Units go group by group (group_rows row blocks);
@@ -428,6 +429,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
   uint64_t* drain_bar = tempty_bar + S::kAccBufs;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile int* abort_word = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* tile_ready = abort_word + 1;   // [2], alternating by accumulator tile
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -665,7 +667,21 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
       Elem* grow = static_cast<Elem*>(args.G) + size_t(row_ok ? row : 0) * size_t(P.V);
 
       for (int vt = split_begin(P, vs); vt < vt1; ++vt) {
-        if (!warp_wait(&tfull_bar[abuf], aphase, ab)) {
+        // The first epilogue warp waits for the accumulator and posts the outcome; the other
+        // warps wait in a named barrier, descheduled, instead of each polling the mbarrier.
+        // All epilogue warps pass the same barriers in the same order and follow the one
+        // posted outcome, so they leave the loop together.  The word alternates between two
+        // slots (consecutive tiles differ in the buffer's parity, or in the phase when there
+        // is one buffer): a slot is rewritten only two barriers later, after every warp has
+        // read it.
+        volatile int* ready = tile_ready + (S::kAccBufs == 1 ? int(aphase) : (abuf & 1));
+        if (warp == kEpiWarp0) {
+          const bool w = warp_wait(&tfull_bar[abuf], aphase, ab);
+          if (lane == 0) *ready = w ? 1 : 0;
+          __syncwarp();
+        }
+        named_bar_sync(kEpiBarrier, S::kEpiWarps * 32);
+        if (*ready == 0) {
           ok = false;
           break;
         }

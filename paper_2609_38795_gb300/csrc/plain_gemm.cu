@@ -23,6 +23,9 @@ constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kThreads = 256;
 constexpr int kEpiWarp0 = 4;
+constexpr int kEpiWarps = 4;
+constexpr int kEpiBarrier = 1;                    // named barrier of the epilogue warps
+static_assert(kEpiWarp0 + kEpiWarps == kThreads / 32, "the epilogue warps end the block");
 constexpr int kStages = 4;
 constexpr int kABytes = kBM * 128;                // 16 KB
 constexpr int kBBytes = kBN * 128;                // 32 KB
@@ -112,6 +115,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* drain_bar = tempty_bar + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile int* abort_word = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* tile_ready = abort_word + 1;   // [2], one per accumulator buffer
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -128,7 +132,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);
-      mbar_init(&tempty_bar[i], 4);
+      mbar_init(&tempty_bar[i], kEpiWarps);
     }
     mbar_init(drain_bar, 1);
     *abort_word = 0;
@@ -233,7 +237,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       int mb, nb;
       decode_tile(args, t, mb, nb);
       if (kMc) mb = kMc * mb + rank;
-      if (!warp_wait(&tfull_bar[abuf], aphase, ab)) break;
+      // The first epilogue warp waits for the accumulator and posts the outcome in the
+      // buffer's word; the others wait, descheduled, in a named barrier.  Every epilogue warp
+      // passes the same barriers and follows the one outcome, so they leave together; a word
+      // is rewritten only two barriers later, after every warp has read it.
+      if (warp == kEpiWarp0) {
+        const bool w = warp_wait(&tfull_bar[abuf], aphase, ab);
+        if (lane == 0) tile_ready[abuf] = w ? 1 : 0;
+        __syncwarp();
+      }
+      named_bar_sync(kEpiBarrier, kEpiWarps * 32);
+      if (tile_ready[abuf] == 0) break;
       tc_fence_after();
       const int m = mb * kBM + q * 32 + lane;
       const bool m_ok = m < args.M;

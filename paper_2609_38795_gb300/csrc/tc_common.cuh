@@ -103,8 +103,10 @@ ALR_DEV void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
 }
 
 // One bounded probe of the phase with the given parity.  A thread whose phase is not yet
-// complete is suspended in hardware until the phase completes or kSuspendHintNs elapses, so
-// waiting warps do not spin through issue slots (and power) while the tensor cores work.
+// complete is suspended in hardware until the phase completes or at most kSuspendHintNs
+// elapses.  In practice it wakes far more often (a waiting thread of the loss kernel probes
+// every few tens of cycles while the CTA's barriers are busy), so kernels keep the number of
+// waiting warps small: one warp waits and the others sleep in a named barrier.
 constexpr uint32_t kSuspendHintNs = 20000;
 
 ALR_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
@@ -126,9 +128,9 @@ struct AbortFlag {
   int* status;   // per-device status word in global memory
 };
 
-// A suspended waiter wakes whenever its barrier (or its CTA's barriers) change state, which
-// during a tile happens every few hundred cycles; the clock and the abort word are checked
-// only on every kWaitCheckEvery-th wake-up, so a wake-up costs a handful of instructions.
+// A suspended waiter wakes every few tens of cycles while the CTA's barriers are busy; the
+// clock and the abort word are checked only on every kWaitCheckEvery-th wake-up, so a wake-up
+// costs a handful of instructions.
 constexpr uint32_t kWaitCheckEvery = 16;
 
 // Wait until the phase with the given parity has completed.  Returns false (after recording
