@@ -402,10 +402,10 @@ int fwd_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
   // bf16 inputs keep fp16 logits through TMA stores of 16-column x 32-row boxes
   CUtensorMap m_zd = m_w, m_zt = m_w;
   if (Zd != nullptr && dt == ALR_BF16) {
-    if ((rc = make_map(&m_zd, Zd, kMapF16, p->V, p->N, p->V * 2, 16, 32,
+    if ((rc = make_map(&m_zd, Zd, kMapF16, p->V, p->N, uint64_t(p->V) * 2, 16, 32,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
       return rc;
-    if ((rc = make_map(&m_zt, Zt, kMapF16, p->V, p->N, p->V * 2, 16, 32,
+    if ((rc = make_map(&m_zt, Zt, kMapF16, p->V, p->N, uint64_t(p->V) * 2, 16, 32,
                        CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
       return rc;
   }
@@ -841,7 +841,7 @@ int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int3
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
   CUtensorMap m_zd = m_w;
   if (Zd != nullptr && dt == ALR_BF16 &&
-      (rc = make_map(&m_zd, Zd, kMapF16, p->V, p->N, p->V * 2, 16, 32,
+      (rc = make_map(&m_zd, Zd, kMapF16, p->V, p->N, uint64_t(p->V) * 2, 16, 32,
                      CU_TENSOR_MAP_SWIZZLE_NONE)) != ALR_OK)
     return rc;
   cudaError_t e = alr::launch_loss_kernel(Zd != nullptr ? alr::kModeTopkFwdKeep : alr::kModeTopkFwd,
