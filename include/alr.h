@@ -104,12 +104,15 @@ int alr_device_status(void* stream, int clear);
 
 /*
  * Test hook for the failure-detection path (the paper has no counterpart).  With enable != 0,
- * the next alr_slot_loss_fwd launch on any thread withholds the first pipeline stage of each
- * CTA: nothing ever fills it, so the MMA issuer's bounded wait runs out after about 1.5 s, every
- * role of the CTA leaves its loop (copies in flight are waited for, tensor memory is released)
- * and the kernel records ALR_ERR_TIMEOUT in the device status word.  That call's outputs are
- * meaningless; alr_device_status() then returns ALR_ERR_TIMEOUT and the context stays usable.
- * Nothing faults, traps or hangs.  The hook disarms itself after one launch.
+ * the next launch, on any thread, of the fused loss kernel by a forward (alr_slot_loss_fwd,
+ * alr_slot_loss_fwd_keep_logits, alr_slot_loss_fwd_noalloc) or of a tensor-core GEMM in the
+ * single or multicast form (alr_gemm, and the dH / dW products of the backward entry points)
+ * withholds the first pipeline stage of each CTA: nothing ever fills it, so the MMA issuer's
+ * bounded wait runs out after about 1.5 s, every role of the CTA leaves its loop (copies in
+ * flight are waited for, tensor memory is released) and the kernel records ALR_ERR_TIMEOUT in
+ * the device status word.  That call's outputs are meaningless; alr_device_status() then
+ * returns ALR_ERR_TIMEOUT and the context stays usable.  Nothing faults, traps or hangs.  The
+ * hook disarms itself after one launch.
  */
 int alr_debug_withhold_next_stage(int enable);
 

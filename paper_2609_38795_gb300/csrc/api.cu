@@ -43,7 +43,8 @@ struct Range {
 };
 #define ALR_RANGE() const Range alr_nvtx_range_(__func__)
 
-// Test hook state: when set, the next forward launch withholds its first pipeline stage.
+// Test hook state: when set, the next launch of the fused loss kernel by a forward, or of the
+// plain GEMM (single or multicast form), withholds its first pipeline stage.
 std::atomic<int> g_withhold_next{0};
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -331,11 +332,13 @@ int launch_gemm(int dt, bool a_mn, bool b_mn, bool acc, const CUtensorMap& ma,
     g.grid = cl * (clusters < g.n_tiles ? clusters : g.n_tiles);
     g.status = alr::device_status_ptr();
     if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+    g.withhold_first_stage = g_withhold_next.exchange(0);
     e = alr::launch_plain_gemm_mc(cl, a_mn, b_mn, acc, ma, mb, g, s);
   } else {
     alr::GemmArgs g = gemm_plan(M, Nc, K, C, ldc, sms);
     g.status = alr::device_status_ptr();
     if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
+    g.withhold_first_stage = g_withhold_next.exchange(0);
     e = alr::launch_plain_gemm(dt, a_mn, b_mn, acc, ma, mb, g, s);
   }
   if (e != cudaSuccess) return cuda_fail(e, what);

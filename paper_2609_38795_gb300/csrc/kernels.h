@@ -107,6 +107,7 @@ struct GemmArgs {
   int n_tiles;
   int grid;
   int* status;
+  int withhold_first_stage;   // test hook: the producer never fills its first stage
 };
 // a_mn / b_mn: operand stored MN-major (A as [K, M], B as [K, Nc]) instead of K-major
 // (A as [M, K], B as [Nc, K]).  accumulate: C += A B instead of C = A B.

@@ -155,7 +155,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int stage = 0;
+      // test hook: start filling at stage 1, so stage 0, the MMA issuer's first, stays empty;
+      // its bounded wait runs out and every role of the CTA takes the timeout path
+      int stage = args.withhold_first_stage ? 1 : 0;
       uint32_t phase = 0, armed = 0, armed_par = 0;
       bool ok = true;
       for (int t = t0; ok && t < args.n_tiles; t += t_step) {

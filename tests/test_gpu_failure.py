@@ -48,3 +48,29 @@ def test_withheld_stage_times_out_and_context_survives(form, monkeypatch):
     assert alr.alr_device_status() == alr.ALR_OK
     r = orc.slot_loss_forward(P.np64(b["Hd"]), P.np64(b["Ht"]), P.np64(b["W"]), B)
     P.compare_forward(P.fwd_to_numpy(sl), r)
+
+
+@pytest.mark.parametrize("form", ["single", "mcast", "mcast4"])
+def test_withheld_gemm_stage_times_out_and_context_survives(form, monkeypatch):
+    """The tensor-core GEMM in its single-CTA and multicast-cluster forms: the withheld stage
+    makes every CTA give up (one epilogue warp sees the abort and the others follow it out of
+    their named barrier), the timeout is reported, and the next product is correct."""
+    monkeypatch.setenv("ALR_GEMM_FORM", form)
+    M, Nc, K = 1024, 768, 512
+    g = torch.Generator(device="cuda").manual_seed(5)
+    A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
+    Bm = torch.randn(Nc, K, device="cuda", generator=g).to(torch.bfloat16)
+    C = torch.zeros(M, Nc, device="cuda")
+    assert alr.alr_device_status(clear=True) == alr.ALR_OK
+    alr.alr_debug_withhold_next_stage(True)
+    t0 = time.monotonic()
+    alr.alr_gemm(A, Bm, C, M, Nc, K)
+    rc = alr.alr_device_status(clear=True)
+    waited = time.monotonic() - t0
+    assert rc == alr.ALR_ERR_TIMEOUT, alr.alr_last_error()
+    assert waited < 20.0
+    alr.alr_gemm(A, Bm, C, M, Nc, K)
+    torch.cuda.synchronize()
+    assert alr.alr_device_status() == alr.ALR_OK
+    ref = P.np64(A) @ P.np64(Bm).T
+    assert P.max_norm_rel(P.np64(C), ref) <= 1e-3
