@@ -135,8 +135,54 @@ def _check(rc):
         raise AlrError(rc, lib().alr_last_error().decode())
 
 
-def _ptr(t):
-    return None if t is None else t.data_ptr()
+_I32, _I64, _F32 = torch.int32, torch.int64, torch.float32
+
+
+def _ptr(t, name="tensor", numel=None, dtype=None):
+    """Device pointer of a tensor argument (None stays NULL), after the checks the C ABI cannot
+    make on a bare pointer: a tensor on the current CUDA device, contiguous, of the expected
+    element type, holding at least `numel` elements.  A wrong buffer is refused here rather
+    than read or written out of bounds by a kernel."""
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch.Tensor, got {type(t).__name__}")
+    if not t.is_cuda or t.device.index != torch.cuda.current_device():
+        raise ValueError(f"{name} must be on the current CUDA device (got {t.device})")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype} (got {t.dtype})")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements, fewer than the {numel} needed")
+    return t.data_ptr()
+
+
+def _in_dtype(params):
+    return torch.bfloat16 if params.dtype == ALR_BF16 else torch.float32
+
+
+def _logit_dtype(params):
+    return torch.float16 if params.dtype == ALR_BF16 else torch.float32
+
+
+def _fwd_outputs(params, out):
+    N = params.N
+    spec = dict(loss_row=(N, _F32), ent_row=(N, _F32), lse_d=(N, _F32), lse_t=(N, _F32),
+                argmax_d=(N, _I32), argmax_t=(N, _I32), gap_d=(N, _F32), gap_t=(N, _F32),
+                logp_x=(N, _F32), weight=(N, _F32), loss_total=(1, _F32), weight_sum=(1, _F32))
+    return AlrFwdOutputs(**{f: _ptr(out.get(f), f, *spec[f]) for f in _FWD_FIELDS})
+
+
+def _topk_outputs(params, out):
+    N = params.N
+    spec = dict(loss_row=(N, _F32), lse_d=(N, _F32), tail_q=(N, _F32), argmax_d=(N, _I32),
+                gap_d=(N, _F32), weight=(N, _F32), loss_total=(1, _F32), weight_sum=(1, _F32))
+    return AlrTopkFwdOutputs(**{f: _ptr(out.get(f), f, *spec[f]) for f in _TOPK_FIELDS})
+
+
+def _ws(ws):
+    return _ptr(ws, "workspace")
 
 
 def _stream(stream=None):
@@ -180,9 +226,14 @@ def alr_debug_withhold_next_stage(enable=True) -> int:
 
 def alr_gather_ira_blocks(feat, seq, pos, B, out, row_valid=None, valid_len=None, stream=None):
     S, L, d = feat.shape
-    _check(lib().alr_gather_ira_blocks(_ptr(feat), S, L, d, dtype_code(feat.dtype), _ptr(seq),
-                                       _ptr(pos), _ptr(valid_len), seq.numel(), B, _ptr(out),
-                                       _ptr(row_valid), _stream(stream)))
+    A = seq.numel()
+    dt = feat.dtype
+    _check(lib().alr_gather_ira_blocks(_ptr(feat, "feat"), S, L, d, dtype_code(dt),
+                                       _ptr(seq, "seq", A, _I32), _ptr(pos, "pos", A, _I32),
+                                       _ptr(valid_len, "valid_len", A, _I32), A, B,
+                                       _ptr(out, "out", A * B * d, dt),
+                                       _ptr(row_valid, "row_valid", A * B, _F32),
+                                       _stream(stream)))
 
 
 def alr_fwd_workspace_size(params) -> int:
@@ -193,42 +244,72 @@ def alr_bwd_workspace_size(params) -> int:
     return lib().alr_bwd_workspace_size(ctypes.byref(params))
 
 
+def _heads(params, Hd=None, Ht=None, W=None):
+    """Pointers of the hidden states [N, d] and the head [d, V] (input element type)."""
+    N, d, V, dt = params.N, params.d, params.V, _in_dtype(params)
+    return (_ptr(Hd, "Hd", N * d, dt), _ptr(Ht, "Ht", N * d, dt), _ptr(W, "W", d * V, dt))
+
+
 def alr_slot_loss_fwd(params, Hd, Ht, W, out: dict, workspace, row_mask=None, corpus_tok=None,
                       stream=None):
-    o = AlrFwdOutputs(**{f: _ptr(out.get(f)) for f in _FWD_FIELDS})
-    _check(lib().alr_slot_loss_fwd(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W),
-                                   _ptr(row_mask), _ptr(corpus_tok), ctypes.byref(o),
-                                   _ptr(workspace), workspace.numel() * workspace.element_size(),
-                                   _stream(stream)))
+    N = params.N
+    hd, ht, w = _heads(params, Hd, Ht, W)
+    o = _fwd_outputs(params, out)
+    _check(lib().alr_slot_loss_fwd(ctypes.byref(params), hd, ht, w,
+                                   _ptr(row_mask, "row_mask", N, _F32),
+                                   _ptr(corpus_tok, "corpus_tok", N, _I32), ctypes.byref(o),
+                                   _ws(workspace), _nbytes(workspace), _stream(stream)))
 
 
 def alr_slot_loss_fwd_noalloc(params, Hd, Ht, W, out: dict, row_mask=None, corpus_tok=None,
                               stream=None):
     """alr_slot_loss_fwd without a workspace (scratch in the library's fixed device array)."""
-    o = AlrFwdOutputs(**{f: _ptr(out.get(f)) for f in _FWD_FIELDS})
-    _check(lib().alr_slot_loss_fwd_noalloc(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W),
-                                           _ptr(row_mask), _ptr(corpus_tok), ctypes.byref(o),
-                                           _stream(stream)))
+    N = params.N
+    hd, ht, w = _heads(params, Hd, Ht, W)
+    o = _fwd_outputs(params, out)
+    _check(lib().alr_slot_loss_fwd_noalloc(ctypes.byref(params), hd, ht, w,
+                                           _ptr(row_mask, "row_mask", N, _F32),
+                                           _ptr(corpus_tok, "corpus_tok", N, _I32),
+                                           ctypes.byref(o), _stream(stream)))
+
+
+def _row_stats(params, weight, weight_sum, lse_d, fourth=None, fourth_name="lse_t"):
+    """Pointers of the per-row forward results the backward reads: weight [N], weight_sum [1],
+    lse_d [N] and lse_t (full vocabulary) or tail_q (top-k) [N]."""
+    N = params.N
+    return (_ptr(weight, "weight", N, _F32), _ptr(weight_sum, "weight_sum", 1, _F32),
+            _ptr(lse_d, "lse_d", N, _F32), _ptr(fourth, fourth_name, N, _F32))
+
+
+def _head_grads(params, dHd, dW):
+    N, d, V = params.N, params.d, params.V
+    return _ptr(dHd, "dHd", N * d, _F32), _ptr(dW, "dW", d * V, _F32)
 
 
 def alr_slot_loss_bwd(params, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, dHd, dW, workspace,
                       stream=None):
-    _check(lib().alr_slot_loss_bwd(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W),
-                                   _ptr(weight), _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t),
-                                   _ptr(dHd), _ptr(dW), _ptr(workspace),
-                                   workspace.numel() * workspace.element_size(), _stream(stream)))
+    hd, ht, w = _heads(params, Hd, Ht, W)
+    wt, ws_, ld, lt = _row_stats(params, weight, weight_sum, lse_d, lse_t)
+    dh, dw = _head_grads(params, dHd, dW)
+    _check(lib().alr_slot_loss_bwd(ctypes.byref(params), hd, ht, w, wt, ws_, ld, lt, dh, dw,
+                                   _ws(workspace), _nbytes(workspace), _stream(stream)))
 
 
 def alr_logit_grad_workspace_size(params) -> int:
     return lib().alr_logit_grad_workspace_size(ctypes.byref(params))
 
 
+def _grad_matrix(params, G):
+    return _ptr(G, "G", params.N * params.V, _in_dtype(params))
+
+
 def alr_logit_grad(params, Hd, Ht, W, weight, weight_sum, lse_d, lse_t, G, workspace=None,
                    stream=None):
-    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    _check(lib().alr_logit_grad(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W), _ptr(weight),
-                                _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t), _ptr(G),
-                                _ptr(workspace), nbytes, _stream(stream)))
+    hd, ht, w = _heads(params, Hd, Ht, W)
+    wt, ws_, ld, lt = _row_stats(params, weight, weight_sum, lse_d, lse_t)
+    _check(lib().alr_logit_grad(ctypes.byref(params), hd, ht, w, wt, ws_, ld, lt,
+                                _grad_matrix(params, G), _ws(workspace), _nbytes(workspace),
+                                _stream(stream)))
 
 
 def _nbytes(ws):
@@ -240,19 +321,28 @@ def logits_dtype(t_dtype):
     return torch.float16 if t_dtype == torch.bfloat16 else torch.float32
 
 
+def _logits(params, Z, name):
+    return _ptr(Z, name, params.N * params.V, _logit_dtype(params))
+
+
 def alr_slot_loss_fwd_keep_logits(params, Hd, Ht, W, Zd, Zt, out: dict, workspace, row_mask=None,
                                   corpus_tok=None, stream=None):
-    o = AlrFwdOutputs(**{f: _ptr(out.get(f)) for f in _FWD_FIELDS})
-    _check(lib().alr_slot_loss_fwd_keep_logits(ctypes.byref(params), _ptr(Hd), _ptr(Ht), _ptr(W),
-                                               _ptr(row_mask), _ptr(corpus_tok), _ptr(Zd),
-                                               _ptr(Zt), ctypes.byref(o), _ptr(workspace),
+    N = params.N
+    hd, ht, w = _heads(params, Hd, Ht, W)
+    o = _fwd_outputs(params, out)
+    _check(lib().alr_slot_loss_fwd_keep_logits(ctypes.byref(params), hd, ht, w,
+                                               _ptr(row_mask, "row_mask", N, _F32),
+                                               _ptr(corpus_tok, "corpus_tok", N, _I32),
+                                               _logits(params, Zd, "Zd"), _logits(params, Zt, "Zt"),
+                                               ctypes.byref(o), _ws(workspace),
                                                _nbytes(workspace), _stream(stream)))
 
 
 def alr_logit_grad_from_logits(params, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, stream=None):
-    _check(lib().alr_logit_grad_from_logits(ctypes.byref(params), _ptr(Zd), _ptr(Zt), _ptr(weight),
-                                            _ptr(weight_sum), _ptr(lse_d), _ptr(lse_t), _ptr(G),
-                                            _stream(stream)))
+    wt, ws_, ld, lt = _row_stats(params, weight, weight_sum, lse_d, lse_t)
+    _check(lib().alr_logit_grad_from_logits(ctypes.byref(params), _logits(params, Zd, "Zd"),
+                                            _logits(params, Zt, "Zt"), wt, ws_, ld, lt,
+                                            _grad_matrix(params, G), _stream(stream)))
 
 
 def alr_bwd_from_logits_workspace_size(params) -> int:
@@ -261,11 +351,14 @@ def alr_bwd_from_logits_workspace_size(params) -> int:
 
 def alr_slot_loss_bwd_from_logits(params, Hd, W, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, dHd,
                                   dW, workspace=None, stream=None):
-    _check(lib().alr_slot_loss_bwd_from_logits(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(Zd),
-                                               _ptr(Zt), _ptr(weight), _ptr(weight_sum),
-                                               _ptr(lse_d), _ptr(lse_t), _ptr(G), _ptr(dHd),
-                                               _ptr(dW), _ptr(workspace), _nbytes(workspace),
-                                               _stream(stream)))
+    hd, _, w = _heads(params, Hd, None, W)
+    wt, ws_, ld, lt = _row_stats(params, weight, weight_sum, lse_d, lse_t)
+    dh, dw = _head_grads(params, dHd, dW)
+    _check(lib().alr_slot_loss_bwd_from_logits(ctypes.byref(params), hd, w,
+                                               _logits(params, Zd, "Zd"),
+                                               _logits(params, Zt, "Zt"), wt, ws_, ld, lt,
+                                               _grad_matrix(params, G), dh, dw, _ws(workspace),
+                                               _nbytes(workspace), _stream(stream)))
 
 
 def alr_readout_workspace_size(params) -> int:
@@ -275,96 +368,143 @@ def alr_readout_workspace_size(params) -> int:
 def alr_label_readout(params, Ht, W, out: dict, workspace, corpus_tok=None, stream=None):
     """out: top_idx [N, 8] int32, top_prob [N, 8], tail [N]; optional lse_t, argmax_t, gap_t,
     logp_x."""
-    _check(lib().alr_label_readout(ctypes.byref(params), _ptr(Ht), _ptr(W), _ptr(corpus_tok),
-                                   _ptr(out["top_idx"]), _ptr(out["top_prob"]), _ptr(out["tail"]),
-                                   _ptr(out.get("lse_t")), _ptr(out.get("argmax_t")),
-                                   _ptr(out.get("gap_t")), _ptr(out.get("logp_x")),
-                                   _ptr(workspace), _nbytes(workspace), _stream(stream)))
+    N, k = params.N, ALR_TOPK
+    _, ht, w = _heads(params, None, Ht, W)
+    _check(lib().alr_label_readout(ctypes.byref(params), ht, w,
+                                   _ptr(corpus_tok, "corpus_tok", N, _I32),
+                                   _ptr(out["top_idx"], "top_idx", N * k, _I32),
+                                   _ptr(out["top_prob"], "top_prob", N * k, _F32),
+                                   _ptr(out["tail"], "tail", N, _F32),
+                                   _ptr(out.get("lse_t"), "lse_t", N, _F32),
+                                   _ptr(out.get("argmax_t"), "argmax_t", N, _I32),
+                                   _ptr(out.get("gap_t"), "gap_t", N, _F32),
+                                   _ptr(out.get("logp_x"), "logp_x", N, _F32),
+                                   _ws(workspace), _nbytes(workspace), _stream(stream)))
 
 
 def alr_topk_fwd_workspace_size(params) -> int:
     return lib().alr_topk_fwd_workspace_size(ctypes.byref(params))
 
 
+def _labels(params, top_idx, top_prob, tail):
+    N, k = params.N, ALR_TOPK
+    return (_ptr(top_idx, "top_idx", N * k, _I32), _ptr(top_prob, "top_prob", N * k, _F32),
+            _ptr(tail, "tail", N, _F32))
+
+
 def alr_topk_loss_fwd(params, Hd, W, top_idx, top_prob, tail, out: dict, workspace,
                       row_mask=None, weight_in=None, stream=None):
-    o = AlrTopkFwdOutputs(**{f: _ptr(out.get(f)) for f in _TOPK_FIELDS})
-    _check(lib().alr_topk_loss_fwd(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(top_idx),
-                                   _ptr(top_prob), _ptr(tail), _ptr(row_mask), _ptr(weight_in),
-                                   ctypes.byref(o), _ptr(workspace), _nbytes(workspace),
-                                   _stream(stream)))
+    N = params.N
+    hd, _, w = _heads(params, Hd, None, W)
+    o = _topk_outputs(params, out)
+    _check(lib().alr_topk_loss_fwd(ctypes.byref(params), hd, w,
+                                   *_labels(params, top_idx, top_prob, tail),
+                                   _ptr(row_mask, "row_mask", N, _F32),
+                                   _ptr(weight_in, "weight_in", N, _F32), ctypes.byref(o),
+                                   _ws(workspace), _nbytes(workspace), _stream(stream)))
 
 
 def alr_topk_logit_grad(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum, lse_d,
                         tail_q, G, workspace=None, stream=None):
-    _check(lib().alr_topk_logit_grad(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(top_idx),
-                                     _ptr(top_prob), _ptr(tail), _ptr(weight), _ptr(weight_sum),
-                                     _ptr(lse_d), _ptr(tail_q), _ptr(G), _ptr(workspace),
-                                     _nbytes(workspace), _stream(stream)))
+    hd, _, w = _heads(params, Hd, None, W)
+    wt, ws_, ld, tq = _row_stats(params, weight, weight_sum, lse_d, tail_q, "tail_q")
+    _check(lib().alr_topk_logit_grad(ctypes.byref(params), hd, w,
+                                     *_labels(params, top_idx, top_prob, tail), wt, ws_, ld, tq,
+                                     _grad_matrix(params, G), _ws(workspace), _nbytes(workspace),
+                                     _stream(stream)))
 
 
 def alr_topk_loss_bwd(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum, lse_d, tail_q,
                       dHd, dW, workspace, stream=None):
-    _check(lib().alr_topk_loss_bwd(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(top_idx),
-                                   _ptr(top_prob), _ptr(tail), _ptr(weight), _ptr(weight_sum),
-                                   _ptr(lse_d), _ptr(tail_q), _ptr(dHd), _ptr(dW),
-                                   _ptr(workspace), _nbytes(workspace), _stream(stream)))
+    hd, _, w = _heads(params, Hd, None, W)
+    wt, ws_, ld, tq = _row_stats(params, weight, weight_sum, lse_d, tail_q, "tail_q")
+    dh, dw = _head_grads(params, dHd, dW)
+    _check(lib().alr_topk_loss_bwd(ctypes.byref(params), hd, w,
+                                   *_labels(params, top_idx, top_prob, tail), wt, ws_, ld, tq,
+                                   dh, dw, _ws(workspace), _nbytes(workspace), _stream(stream)))
 
 
 def alr_topk_loss_fwd_keep_logits(params, Hd, W, top_idx, top_prob, tail, Zd, out: dict,
                                   workspace, row_mask=None, weight_in=None, stream=None):
-    o = AlrTopkFwdOutputs(**{f: _ptr(out.get(f)) for f in _TOPK_FIELDS})
-    _check(lib().alr_topk_loss_fwd_keep_logits(ctypes.byref(params), _ptr(Hd), _ptr(W),
-                                               _ptr(top_idx), _ptr(top_prob), _ptr(tail),
-                                               _ptr(row_mask), _ptr(weight_in), _ptr(Zd),
-                                               ctypes.byref(o), _ptr(workspace),
-                                               _nbytes(workspace), _stream(stream)))
+    N = params.N
+    hd, _, w = _heads(params, Hd, None, W)
+    o = _topk_outputs(params, out)
+    _check(lib().alr_topk_loss_fwd_keep_logits(ctypes.byref(params), hd, w,
+                                               *_labels(params, top_idx, top_prob, tail),
+                                               _ptr(row_mask, "row_mask", N, _F32),
+                                               _ptr(weight_in, "weight_in", N, _F32),
+                                               _logits(params, Zd, "Zd"), ctypes.byref(o),
+                                               _ws(workspace), _nbytes(workspace),
+                                               _stream(stream)))
 
 
 def alr_topk_logit_grad_from_logits(params, Zd, top_idx, top_prob, tail, weight, weight_sum,
                                     lse_d, tail_q, G, stream=None):
-    _check(lib().alr_topk_logit_grad_from_logits(ctypes.byref(params), _ptr(Zd), _ptr(top_idx),
-                                                 _ptr(top_prob), _ptr(tail), _ptr(weight),
-                                                 _ptr(weight_sum), _ptr(lse_d), _ptr(tail_q),
-                                                 _ptr(G), _stream(stream)))
+    wt, ws_, ld, tq = _row_stats(params, weight, weight_sum, lse_d, tail_q, "tail_q")
+    _check(lib().alr_topk_logit_grad_from_logits(ctypes.byref(params), _logits(params, Zd, "Zd"),
+                                                 *_labels(params, top_idx, top_prob, tail),
+                                                 wt, ws_, ld, tq, _grad_matrix(params, G),
+                                                 _stream(stream)))
 
 
 def alr_topk_loss_bwd_from_logits(params, Hd, W, Zd, top_idx, top_prob, tail, weight, weight_sum,
                                   lse_d, tail_q, G, dHd, dW, workspace=None, stream=None):
-    _check(lib().alr_topk_loss_bwd_from_logits(ctypes.byref(params), _ptr(Hd), _ptr(W), _ptr(Zd),
-                                               _ptr(top_idx), _ptr(top_prob), _ptr(tail),
-                                               _ptr(weight), _ptr(weight_sum), _ptr(lse_d),
-                                               _ptr(tail_q), _ptr(G), _ptr(dHd), _ptr(dW),
-                                               _ptr(workspace), _nbytes(workspace),
+    hd, _, w = _heads(params, Hd, None, W)
+    wt, ws_, ld, tq = _row_stats(params, weight, weight_sum, lse_d, tail_q, "tail_q")
+    dh, dw = _head_grads(params, dHd, dW)
+    _check(lib().alr_topk_loss_bwd_from_logits(ctypes.byref(params), hd, w,
+                                               _logits(params, Zd, "Zd"),
+                                               *_labels(params, top_idx, top_prob, tail),
+                                               wt, ws_, ld, tq, _grad_matrix(params, G), dh, dw,
+                                               _ws(workspace), _nbytes(workspace),
                                                _stream(stream)))
 
 
 def alr_ira_blocks(K, max_blocks, valid_anchors, rollout_len, offsets, out: dict,
                    rollout_tok=None, corpus_anchor_tok=None, stream=None):
     """out: seq, pos, valid_len (int32 [S*max_blocks]); optional ctx_len, anchor_tok."""
-    _check(lib().alr_ira_blocks(valid_anchors.numel(), K, max_blocks, _ptr(valid_anchors),
-                                _ptr(rollout_len), _ptr(offsets), _ptr(rollout_tok),
-                                _ptr(corpus_anchor_tok), _ptr(out["seq"]), _ptr(out["pos"]),
-                                _ptr(out["valid_len"]), _ptr(out.get("ctx_len")),
-                                _ptr(out.get("anchor_tok")), _stream(stream)))
+    S = valid_anchors.numel()
+    half = max_blocks // 2
+    P = max_blocks - half
+    T = S * max_blocks
+    _check(lib().alr_ira_blocks(S, K, max_blocks, _ptr(valid_anchors, "valid_anchors", S, _I32),
+                                _ptr(rollout_len, "rollout_len", S * P, _I32),
+                                _ptr(offsets, "offsets", S * half, _I32),
+                                _ptr(rollout_tok, "rollout_tok", S * P * K, _I32),
+                                _ptr(corpus_anchor_tok, "corpus_anchor_tok", T, _I32),
+                                _ptr(out["seq"], "seq", T, _I32), _ptr(out["pos"], "pos", T, _I32),
+                                _ptr(out["valid_len"], "valid_len", T, _I32),
+                                _ptr(out.get("ctx_len"), "ctx_len", T, _I32),
+                                _ptr(out.get("anchor_tok"), "anchor_tok", T, _I32),
+                                _stream(stream)))
 
 
 def alr_accept_len(argmax_d, argmax_t, B, acc_len, hist=None, active=None, stream=None):
     A = argmax_d.numel() // B
-    _check(lib().alr_accept_len(_ptr(argmax_d), _ptr(argmax_t), _ptr(active), A, B,
-                                _ptr(acc_len), _ptr(hist), _stream(stream)))
+    N = A * B
+    _check(lib().alr_accept_len(_ptr(argmax_d, "argmax_d", N, _I32),
+                                _ptr(argmax_t, "argmax_t", N, _I32),
+                                _ptr(active, "active", N, _F32), A, B,
+                                _ptr(acc_len, "acc_len", A, _I32),
+                                _ptr(hist, "hist", B + 1, _I64), _stream(stream)))
 
 
 def alr_erase_weights(B, gamma, hard, weight, logp_x=None, corpus_tok=None, argmax_t=None,
                       row_mask=None, stream=None):
     A = weight.numel() // B
-    _check(lib().alr_erase_weights(_ptr(logp_x), _ptr(corpus_tok), _ptr(argmax_t), _ptr(row_mask),
-                                   A, B, float(gamma), int(hard), _ptr(weight), _stream(stream)))
+    N = A * B
+    _check(lib().alr_erase_weights(_ptr(logp_x, "logp_x", N, _F32),
+                                   _ptr(corpus_tok, "corpus_tok", N, _I32),
+                                   _ptr(argmax_t, "argmax_t", N, _I32),
+                                   _ptr(row_mask, "row_mask", N, _F32), A, B, float(gamma),
+                                   int(hard), _ptr(weight, "weight", N, _F32), _stream(stream)))
 
 
 def alr_gemm(A, B, C, M, Nc, K, a_mn=False, b_mn=False, accumulate=False, stream=None):
-    _check(lib().alr_gemm(dtype_code(A.dtype), int(a_mn), int(b_mn), int(accumulate), _ptr(A),
-                          _ptr(B), _ptr(C), M, Nc, K, _stream(stream)))
+    dt = A.dtype
+    _check(lib().alr_gemm(dtype_code(dt), int(a_mn), int(b_mn), int(accumulate),
+                          _ptr(A, "A", M * K, dt), _ptr(B, "B", Nc * K, dt),
+                          _ptr(C, "C", M * Nc, _F32), M, Nc, K, _stream(stream)))
 
 
 # ------------------------------------------------------------------ convenience ---

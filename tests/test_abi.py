@@ -81,3 +81,21 @@ def test_argument_errors_are_reported_without_a_launch(libalr):
                                            None, 0, None)
     assert rc == alr.ALR_ERR_INVALID_ARG
     assert "dHd" in lib.alr_last_error().decode()
+
+
+def test_binding_refuses_host_and_malformed_tensors_before_any_call(libalr):
+    """The C ABI takes bare device pointers and cannot check a buffer behind one, so the binding
+    does: host tensors, non-tensors and (on any machine) the wrong buffers raise before the
+    library sees a pointer."""
+    import torch
+    N, d, V, B = 32, 64, 128, 16
+    params = alr.make_params(N, d, V, B, torch.bfloat16)
+    host = torch.zeros(N * d, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="CUDA device"):
+        alr.alr_gemm(host, host, torch.zeros(N * N), N, N, d)
+    with pytest.raises(ValueError, match="CUDA device"):
+        alr.alr_slot_loss_fwd_noalloc(params, host, host, torch.zeros(d * V, dtype=torch.bfloat16),
+                                      {})
+    with pytest.raises(TypeError, match="torch.Tensor"):
+        alr._ptr(host.float().numpy(), "Hd")
+    assert alr._ptr(None, "row_mask") is None

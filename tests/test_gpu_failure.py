@@ -74,3 +74,26 @@ def test_withheld_gemm_stage_times_out_and_context_survives(form, monkeypatch):
     assert alr.alr_device_status() == alr.ALR_OK
     ref = P.np64(A) @ P.np64(Bm).T
     assert P.max_norm_rel(P.np64(C), ref) <= 1e-3
+
+
+def test_binding_refuses_wrong_device_buffers():
+    """Buffers the kernels would read or write out of bounds, or misread, are refused by the
+    binding with the argument's name, and nothing is launched (the status stays clean)."""
+    N, d, V, B = 64, 64, 256, 16
+    params = alr.make_params(N, d, V, B, torch.bfloat16)
+    bf = lambda *s: torch.zeros(*s, dtype=torch.bfloat16, device="cuda")  # noqa: E731
+    Hd, W = bf(N, d), bf(d, V)
+    out = {f: torch.zeros(N, device="cuda") for f in alr._FWD_FIELDS}
+    out["argmax_d"] = torch.zeros(N, dtype=torch.int32, device="cuda")
+    out["argmax_t"] = torch.zeros(N, dtype=torch.int32, device="cuda")
+    with pytest.raises(ValueError, match="Ht holds"):
+        alr.alr_slot_loss_fwd_noalloc(params, Hd, bf(N - 1, d), W, out)
+    with pytest.raises(ValueError, match="W must be contiguous"):
+        alr.alr_slot_loss_fwd_noalloc(params, Hd, Hd, bf(V, d).t(), out)
+    bad = dict(out, argmax_d=torch.zeros(N, dtype=torch.int64, device="cuda"))
+    with pytest.raises(ValueError, match="argmax_d must be torch.int32"):
+        alr.alr_slot_loss_fwd_noalloc(params, Hd, Hd, W, bad)
+    with pytest.raises(ValueError, match="C holds"):
+        alr.alr_gemm(Hd, Hd, torch.zeros(N, N - 1, device="cuda"), N, N, d)
+    torch.cuda.synchronize()
+    assert alr.alr_device_status() == alr.ALR_OK
