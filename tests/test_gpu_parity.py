@@ -130,6 +130,36 @@ def test_ragged_bf16_forward_backward(mode):
     assert np.all(P.np64(dH)[5::B] == 0)                   # masked rows get no gradient
 
 
+@pytest.mark.parametrize("keep", [True, False])
+def test_large_ragged_step(keep):
+    """Ragged at scale, through the whole step (forward, accepted length, backward), with the
+    logits kept and recomputed: N = 2000 rows (15.6 row tiles, the last raster group partial),
+    d = 1000 (a K tail of 40), V = 60000 (234.4 vocabulary tiles, split unevenly over the
+    CTAs), one masked row per anchor, lambda off its default.  Every row of the forward and
+    of dH against the oracle, dW on every 7th column."""
+    A, B, d, V, lam = 125, 16, 1000, 60000, 1.013441
+    Hd, Ht, W = _inputs(d, V, A, B, 0.5, torch.bfloat16, seed=31)
+    mask = torch.ones(A * B, device="cuda")
+    mask[7::B] = 0.0
+    sl = alr.SlotLoss(A * B, d, V, B, lam=lam, keep_logits=keep)
+    sl.forward(Hd, Ht, W, row_mask=mask)
+    acc, hist = sl.accept(active=mask)
+    dH = torch.empty(A * B, d, device="cuda")
+    dW = torch.zeros(d, V, device="cuda")
+    sl.backward(Hd, Ht, W, dH, dW)
+    torch.cuda.synchronize()
+    assert alr.alr_device_status() == alr.ALR_OK
+    r = _oracle_fwd(Hd, Ht, W, B, lam=lam, row_mask=P.np64(mask))
+    P.compare_forward(P.fwd_to_numpy(sl), r)
+    acc_r, _ = orc.accept_len(r["argmax_d"], r["argmax_t"], B, active=P.np64(mask))
+    P.compare_accept(P.npi(acc), P.npi(hist), acc_r, r["gap_d"], r["gap_t"], B)
+    G = orc.logit_grad(r["z_d"], r["z_t"], r["weight"], lam)
+    assert P.max_norm_rel(P.np64(dH), G @ P.np64(W).T) <= P.GRAD_RTOL
+    cols = np.arange(0, V, 7)
+    assert P.max_norm_rel(P.np64(dW)[:, cols], P.np64(Hd).T @ G[:, cols]) <= P.GRAD_RTOL
+    assert np.all(P.np64(dH)[7::B] == 0)
+
+
 def test_small_bf16_forward_full_parity():
     """The small workload (d=2048, V=32000, B=16, 256 anchors): every row, forward only."""
     wl = synthetic.WORKLOADS["small"]
