@@ -75,10 +75,12 @@ def compare_readout(g, r, prob_rtol=1e-3):
 @pytest.mark.parametrize("dtype,shape", [(torch.bfloat16, (10, 16, 200, 1000)),
                                          (torch.bfloat16, (17, 16, 200, 1000)),
                                          (torch.float32, (64, 8, 256, 4096)),
-                                         (torch.bfloat16, (64, 16, 2048, 32000))])
+                                         (torch.bfloat16, (64, 16, 2048, 32000)),
+                                         (torch.bfloat16, (125, 16, 1000, 60000))])
 def test_readout_matches_oracle(dtype, shape):
-    """Row counts of 1.25, 2.1, 4 and 8 row blocks of 128: the readout's units take two row
-    blocks each, so the last unit may hold a partial block or none."""
+    """Row counts of 1.25, 2.1, 4, 8 and 15.6 row blocks of 128: the readout's units take two
+    row blocks each, so the last unit may hold a partial block or none; the last shape also
+    has a K tail (d = 1000) and a partial vocabulary tile (V = 60000)."""
     A, B, d, V = shape
     b = synthetic.slot_batch(d, V, A, B, 0.5, dtype=dtype, device="cuda", seed=A + V)
     N = A * B
@@ -255,7 +257,8 @@ def test_text8b_full_batch_compact_labels(keep):
 @pytest.mark.parametrize("dtype,shape,use_weight", [(torch.bfloat16, (10, 16, 200, 1000), False),
                                                     (torch.bfloat16, (10, 16, 200, 1000), True),
                                                     (torch.float32, (64, 8, 256, 4096), False),
-                                                    (torch.bfloat16, (16, 16, 1024, 40000), False)])
+                                                    (torch.bfloat16, (16, 16, 1024, 40000), False),
+                                                    (torch.bfloat16, (125, 16, 1000, 60000), False)])
 def test_topk_keep_logits_forward_backward(dtype, shape, use_weight):
     """The kept-logits top-k path: forward outputs bit-identical to the plain forward, the kept
     z_d within its storage rounding of the oracle's, and G (written over z_d), dH and dW from
