@@ -177,15 +177,33 @@ def test_small_bf16_forward_full_parity():
     assert near < wl.N // 4
 
 
+@pytest.mark.parametrize("keep", [False, True])
 @pytest.mark.parametrize("B", [1, 3, 32])
-def test_degenerate_shapes(B):
-    """Vocabulary smaller than one tile, hidden size below one pipeline stage, B = 1 and 32."""
+def test_degenerate_shapes(B, keep):
+    """Vocabulary smaller than one tile, hidden size below one pipeline stage, B = 1 and 32,
+    through the whole step; with the logits kept, the kept z_d / z_t (their 16-column store
+    boxes cut at V = 24) are checked too."""
     A, d, V = 7, 8, 24
     Hd, Ht, W = _inputs(d, V, A, B, 1.0, torch.bfloat16, seed=B)
     W = (W.float() * 20).to(torch.bfloat16)                  # sharpen the tiny problem
-    sl = P.gpu_forward(Hd, Ht, W, B)
+    N = A * B
+    sl = alr.SlotLoss(N, d, V, B, keep_logits=keep)
+    sl.forward(Hd, Ht, W)
+    torch.cuda.synchronize()
     r = _oracle_fwd(Hd, Ht, W, B)
     P.compare_forward(P.fwd_to_numpy(sl), r)
+    if keep:
+        for z_g, z_r in ((sl.Zd, r["z_d"]), (sl.Zt, r["z_t"])):
+            assert np.all(np.abs(P.np64(z_g) - z_r) <= 2.0 ** -11 * np.abs(z_r) + 1e-4)
+    dH = torch.empty(N, d, device="cuda")
+    dW = torch.zeros(d, V, device="cuda")
+    sl.backward(Hd, Ht, W, dH, dW)
+    torch.cuda.synchronize()
+    G = orc.logit_grad(r["z_d"], r["z_t"], r["weight"], 1.0)
+    dH_r, dW_r = orc.slot_loss_backward(P.np64(Hd), P.np64(W), G)
+    assert P.max_norm_rel(P.np64(dH), dH_r) <= P.GRAD_RTOL
+    assert P.max_norm_rel(P.np64(dW), dW_r) <= P.GRAD_RTOL
+    assert alr.alr_device_status() == alr.ALR_OK
 
 
 def test_identical_hidden_states_give_entropy_and_full_acceptance():
