@@ -99,3 +99,31 @@ def test_binding_refuses_host_and_malformed_tensors_before_any_call(libalr):
     with pytest.raises(TypeError, match="torch.Tensor"):
         alr._ptr(host.float().numpy(), "Hd")
     assert alr._ptr(None, "row_mask") is None
+
+
+def test_last_error_is_per_host_thread(libalr):
+    """alr_last_error() belongs to the calling thread: two threads that fail different calls at
+    the same time each read back their own message."""
+    import threading
+    lib = alr.lib()
+    barrier = threading.Barrier(2)
+    seen = {}
+
+    def fail_with(tag, params):
+        out = alr.AlrFwdOutputs()
+        for _ in range(200):
+            barrier.wait()
+            rc = lib.alr_slot_loss_fwd(ctypes.byref(params), None, None, None, None, None,
+                                       ctypes.byref(out), None, 0, None)
+            barrier.wait()
+            seen.setdefault(tag, set()).add((rc, lib.alr_last_error().decode()))
+
+    t1 = threading.Thread(target=fail_with, args=("B", alr.make_params(N=30, d=64, V=128, B=16)))
+    t2 = threading.Thread(target=fail_with, args=("d", alr.make_params(N=32, d=12, V=128, B=16)))
+    t1.start(), t2.start()
+    t1.join(), t2.join()
+    assert len(seen["B"]) == 1 and len(seen["d"]) == 1
+    (rc_b, msg_b), = seen["B"]
+    (rc_d, msg_d), = seen["d"]
+    assert rc_b == rc_d == alr.ALR_ERR_INVALID_ARG
+    assert "multiple of B" in msg_b and "d = 12" in msg_d
