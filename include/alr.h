@@ -404,7 +404,8 @@ int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
  * accepted; MAT tau = acc + 1, Sec. 4).
  *   argmax_d, argmax_t [A*B] int32; active [A*B] float or NULL (rows with active <= 0 stop
  *   the count).  acc_len [A] int32 output; hist [B+1] int64 or NULL, overwritten with
- *   hist[n] = #{a : acc_len[a] = n}.
+ *   hist[n] = #{a : acc_len[a] = n}.  A = 0 is allowed: hist is then all zero and no kernel
+ *   is launched.
  */
 int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,
                    int32_t A, int32_t B, int32_t* acc_len, int64_t* hist, void* stream);

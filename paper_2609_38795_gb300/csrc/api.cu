@@ -1006,7 +1006,13 @@ int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float
   DevInfo info;
   int rc = require_sm103(&info);
   if (rc != ALR_OK) return rc;
-  if (A == 0 && hist == nullptr) return ALR_OK;
+  if (A == 0) {   // no anchors: an all-zero histogram, no kernel to launch
+    if (hist == nullptr) return ALR_OK;
+    cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(int64_t) * size_t(B + 1),
+                                    static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "histogram clear");
+    return ALR_OK;
+  }
   cudaError_t e = alr::launch_accept_len(argmax_d, argmax_t, active, A, B, acc_len, hist,
                                          static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "accept_len launch");

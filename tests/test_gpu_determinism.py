@@ -1,8 +1,8 @@
 """Run-to-run reproducibility of the whole step through the C ABI: the same inputs give
-bit-identical outputs on every call.  No reduction of the path uses atomics: the partial
-statistics of the vocabulary splits are merged in a fixed order, the accepted-length
-histogram is counted per anchor and summed in order, and every GEMM tile accumulates its K
-range in one fixed order."""
+bit-identical outputs on every call.  No floating-point reduction of the path uses atomics:
+the partial statistics of the vocabulary splits are merged in a fixed order and every GEMM
+tile accumulates its K range in one fixed order; the only atomic adds are the integer counts
+of the accepted-length histogram, which are exact in any order."""
 
 import pytest
 import torch

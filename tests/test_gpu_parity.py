@@ -81,6 +81,26 @@ def test_gather_empty_batch():
     alr.alr_gather_ira_blocks(F, e, e, 4, out)
 
 
+def test_empty_batches_elsewhere():
+    """No anchors: the accepted-length call still writes an all-zero histogram, the erase
+    weights and the IRA block plan are no-ops, and the loss refuses N = 0 (a loss over no rows
+    has no normaliser) with an argument error; nothing faults and the status stays clean."""
+    B = 16
+    ei = torch.empty(0, dtype=torch.int32, device="cuda")
+    ef = torch.empty(0, device="cuda")
+    hist = torch.full((B + 1,), 7, dtype=torch.int64, device="cuda")
+    alr.alr_accept_len(ei, ei, B, ei, hist)
+    alr.alr_erase_weights(B, 2.0, False, ef, logp_x=ef)
+    out = {k: torch.empty(0, dtype=torch.int32, device="cuda") for k in ("seq", "pos", "valid_len")}
+    alr.alr_ira_blocks(15, 128, ei, ei, ei, out)
+    torch.cuda.synchronize()
+    assert hist.cpu().tolist() == [0] * (B + 1)
+    with pytest.raises(alr.AlrError) as err:
+        alr.alr_slot_loss_fwd_noalloc(alr.make_params(0, 64, 256, B), None, None, None, {})
+    assert err.value.code == alr.ALR_ERR_INVALID_ARG
+    assert alr.alr_device_status() == alr.ALR_OK
+
+
 # ------------------------------------------------------------------------ forward ---
 def test_tiny_fp32_forward_backward_full_parity():
     """The tiny fp32 workload (d=256, V=4096, B=8, 64 anchors), every row and gradient."""
