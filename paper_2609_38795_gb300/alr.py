@@ -479,8 +479,15 @@ def alr_ira_blocks(K, max_blocks, valid_anchors, rollout_len, offsets, out: dict
                                 _stream(stream)))
 
 
+def _anchors(t, B, name):
+    """Anchor count of a per-row tensor of A*B entries."""
+    if B < 1 or t.numel() % B != 0:
+        raise ValueError(f"{name} holds {t.numel()} rows, not a whole number of anchors of B = {B}")
+    return t.numel() // B
+
+
 def alr_accept_len(argmax_d, argmax_t, B, acc_len, hist=None, active=None, stream=None):
-    A = argmax_d.numel() // B
+    A = _anchors(argmax_d, B, "argmax_d")
     N = A * B
     _check(lib().alr_accept_len(_ptr(argmax_d, "argmax_d", N, _I32),
                                 _ptr(argmax_t, "argmax_t", N, _I32),
@@ -491,7 +498,7 @@ def alr_accept_len(argmax_d, argmax_t, B, acc_len, hist=None, active=None, strea
 
 def alr_erase_weights(B, gamma, hard, weight, logp_x=None, corpus_tok=None, argmax_t=None,
                       row_mask=None, stream=None):
-    A = weight.numel() // B
+    A = _anchors(weight, B, "weight")
     N = A * B
     _check(lib().alr_erase_weights(_ptr(logp_x, "logp_x", N, _F32),
                                    _ptr(corpus_tok, "corpus_tok", N, _I32),

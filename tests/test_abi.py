@@ -96,6 +96,9 @@ def test_binding_refuses_host_and_malformed_tensors_before_any_call(libalr):
     with pytest.raises(ValueError, match="CUDA device"):
         alr.alr_slot_loss_fwd_noalloc(params, host, host, torch.zeros(d * V, dtype=torch.bfloat16),
                                       {})
+    with pytest.raises(ValueError, match="whole number of anchors"):
+        alr.alr_accept_len(torch.zeros(20, dtype=torch.int32), torch.zeros(20, dtype=torch.int32),
+                           16, torch.zeros(1, dtype=torch.int32))
     with pytest.raises(TypeError, match="torch.Tensor"):
         alr._ptr(host.float().numpy(), "Hd")
     assert alr._ptr(None, "row_mask") is None
