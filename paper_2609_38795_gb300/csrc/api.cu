@@ -177,7 +177,9 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd, bool two_rows = 
   P.bn = ALR_LOSS_BN;
   P.mc = (!two_rows && loss_multicast(p)) ? 1 : 0;
   // row blocks; row-block pairs for the two-row modes and for the multicast form (which
-  // places sms / 2 clusters); raster groups of 8 row blocks either way
+  // places sms / 2 clusters).  The vocabulary splits are sized so that one round of the grid
+  // covers 8 row blocks (152 CTAs / 8 = 19 splits: 32 units per CTA at 256 row blocks); the
+  // forward's raster groups span two rounds (16 row blocks), the recomputing backward's one.
   const int rb = int((p->N + 127) / 128);
   const bool pairs = P.mc || two_rows;
   P.n_rb = pairs ? (rb + 1) / 2 : rb;
@@ -191,6 +193,11 @@ alr::LossPlan loss_plan(const alr_params* p, int sms, bool bwd, bool two_rows = 
     int vs = slots / P.group_rows;
     if (vs < 1) vs = 1;
     P.n_vs = vs < P.n_vt ? vs : P.n_vt;
+    // two rounds per raster group: twice the row blocks share each W split, so W leaves
+    // DRAM about half as often, with the same number of units per CTA (forward 49.8 against
+    // 50.0 ms at the text8b size, three alternating A/B rounds)
+    const int wide = 2 * group;
+    P.group_rows = P.n_rb < wide ? P.n_rb : wide;
   }
   // partial records per row and split: one per epilogue column group
   P.n_parts = P.n_vs * (P.bn / (two_rows ? 128 : 64));
