@@ -59,6 +59,9 @@ def parse_args():
                          "noise levels")
     ap.add_argument("--no-topk", action="store_true",
                     help="skip the compact-label (top-8 + tail) step measurement")
+    ap.add_argument("--no-other-workloads", action="store_true",
+                    help="skip the vl7b step and the small-workload forward measured beside the "
+                         "headline workload")
     ap.add_argument("--gather-only", action="store_true",
                     help="profiling only: run just the IRA gather measurement and print its "
                          "result (no step, a little over 2 GB of device memory)")
@@ -495,6 +498,70 @@ def time_erase(wl, x, device, K, warmup, argmax_t):
     return out
 
 
+def time_other_workloads(device, K, warmup):
+    """Beside the headline workload, two configurations timed for reference (not bench
+    lines): the vl7b step (gather from its 32 x 2048 feature buffer, forward keeping the
+    logits, accepted length, gradient, dH, dW) and the small workload's forward alone.  The
+    small forward's head (131 MB) is about the size of L2, so L2 is flushed (a 256 MB write)
+    before every timed repetition; the vl7b inputs are larger than L2."""
+    import torch
+    from paper_2609_38795_gb300 import alr, synthetic
+    out = {}
+    wl = synthetic.WORKLOADS["vl7b"]
+    x = make_inputs(wl, 0.5, device, seed=7)
+    st = Step(wl, x, device, keep=True)
+    for _ in range(warmup):
+        st.run()
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(K)]
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for k in range(K):
+        st.run(ev[k])
+    b.record()
+    torch.cuda.synchronize()
+    check_device_status("vl7b step")
+    ms = a.elapsed_time(b) / K
+    phase = {p: sum(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(K)) / K
+             for i, p in enumerate(Step.PHASES)}
+    NdV = wl.N * wl.d * wl.V
+    out["vl7b_step"] = {
+        "workload": f"vl7b: d={wl.d} V={wl.V} B={wl.B} A={wl.A} rows={wl.N}, feature buffer "
+                    f"{wl.S}x{wl.L}", "ms_per_step": ms, "rows_per_s": wl.N / (ms / 1e3),
+        "executed_tflops_8NdV": 8 * NdV / (ms / 1e3) / 1e12, "phase_ms": phase,
+        "fwd_rows_per_s": wl.N / (phase["fwd"] / 1e3),
+        "loss": st.sl.out["loss_total"].item()}
+    del st, x
+    torch.cuda.empty_cache()
+
+    wl = synthetic.WORKLOADS["small"]
+    bt = synthetic.slot_batch(wl.d, wl.V, wl.A, wl.B, wl.sigma, dtype=torch.bfloat16,
+                              device=device, seed=8)
+    sl = alr.SlotLoss(wl.N, wl.d, wl.V, wl.B)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    for _ in range(warmup):
+        sl.forward(bt["Hd"], bt["Ht"], bt["W"])
+    times = []
+    for _ in range(K):
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        sl.forward(bt["Hd"], bt["Ht"], bt["W"])
+        e1.record()
+        times.append((e0, e1))
+    torch.cuda.synchronize()
+    check_device_status("small forward")
+    ms = sum(e0.elapsed_time(e1) for e0, e1 in times) / K
+    out["small_forward"] = {
+        "workload": f"small: d={wl.d} V={wl.V} B={wl.B} A={wl.A} rows={wl.N}",
+        "ms": ms, "rows_per_s": wl.N / (ms / 1e3),
+        "tflops_4NdV": 4 * wl.N * wl.d * wl.V / (ms / 1e3) / 1e12,
+        "l2": "flushed (256 MB write) before every repetition", "gpu_launches": 3 * K}
+    del sl, bt, flush
+    torch.cuda.empty_cache()
+    return out
+
+
 def mean_accepted_tokens(hist):
     """MAT of Sec. 4: the mean over anchors of (accepted slots + 1), from a histogram whose
     entry n counts the anchors with n accepted slots."""
@@ -667,6 +734,8 @@ def run_gpu(args, rank, world, local_rank):
              if (rank == 0 and not args.no_recompute) else None)
     erase = (time_erase(wl, x, device, K, args.warmup, step.sl.out["argmax_t"].clone())
              if (rank == 0 and not args.no_erase) else None)
+    others = (time_other_workloads(device, K, args.warmup)
+              if (rank == 0 and not args.no_other_workloads and not args.anchors) else None)
     hist_sigma = None
     if rank == 0 and not args.no_erase:
         hist_sigma = acc_hist_by_sigma(wl, step, device, [0.25, 1.0])
@@ -732,6 +801,7 @@ def run_gpu(args, rank, world, local_rank):
         "mat_by_sigma": (None if hist_sigma is None else
                          {sg: mean_accepted_tokens(h) for sg, h in hist_sigma.items()}),
         "erase": erase,
+        "other_workloads": others,
         "clocks": clk,
         "cpu_baseline": cpu,
     }
