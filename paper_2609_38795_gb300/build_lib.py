@@ -6,6 +6,7 @@ Usage:  python -m paper_2609_38795_gb300.build_lib [--force] [-v]
 from __future__ import annotations
 
 import concurrent.futures as cf
+import fcntl
 import hashlib
 import os
 import shutil
@@ -53,10 +54,25 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     os.makedirs(OUT_DIR, exist_ok=True)
     stamp = os.path.join(OUT_DIR, "libalr.stamp")
     fp = _fingerprint(nvcc) + "|" + " ".join(extra_flags)
-    if not force and os.path.exists(LIB) and os.path.exists(stamp):
+
+    def up_to_date():
+        if force or not (os.path.exists(LIB) and os.path.exists(stamp)):
+            return False
         with open(stamp) as f:
-            if f.read() == fp:
-                return LIB
+            return f.read() == fp
+
+    if up_to_date():
+        return LIB
+    # One builder at a time (the ranks of a torchrun launch all call build()); whoever gets
+    # the lock second finds the library built and up to date.
+    with open(os.path.join(OUT_DIR, "build.lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        if up_to_date():
+            return LIB
+        return _build_locked(nvcc, stamp, fp, verbose, extra_flags)
+
+
+def _build_locked(nvcc, stamp, fp, verbose, extra_flags):
     objs = []
 
     def compile_one(src):
