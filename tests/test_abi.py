@@ -130,3 +130,62 @@ def test_last_error_is_per_host_thread(libalr):
     (rc_d, msg_d), = seen["d"]
     assert rc_b == rc_d == alr.ALR_ERR_INVALID_ARG
     assert "multiple of B" in msg_b and "d = 12" in msg_d
+
+
+def test_error_paths_reject_before_any_device_work(libalr):
+    """Table of invalid calls through the raw C ABI.  The pointers are fakes that must never be
+    dereferenced: every case is refused by argument validation, with its own status and
+    message, before the library looks for a device (on a machine without one, a case that
+    slipped past validation would report the missing device instead and fail here)."""
+    lib = alr.lib()
+    A16, MIS = ctypes.c_void_p(0x10000), ctypes.c_void_p(0x10002)    # aligned / misaligned
+    out = alr.AlrFwdOutputs(**{f: 0x20000 for f in alr._FWD_FIELDS})
+
+    def fwd(params, hd=A16, ht=A16, w=A16, ws=A16, nbytes=1 << 30, tok=None):
+        return lib.alr_slot_loss_fwd(ctypes.byref(params), hd, ht, w, None, tok,
+                                     ctypes.byref(out), ws, nbytes, None)
+
+    P = alr.make_params
+    bad = alr.AlrParams(N=32, d=64, V=128, B=16, dtype=7, mode=0, lam=1.0, gamma=2.0)
+    cases = [
+        ("dtype", lambda: fwd(bad), alr.ALR_ERR_UNSUPPORTED, "dtype 7"),
+        ("mode", lambda: fwd(P(32, 64, 128, 16, mode=5)), alr.ALR_ERR_UNSUPPORTED, "mode 5"),
+        ("B too large", lambda: fwd(P(64, 64, 128, 64)), alr.ALR_ERR_INVALID_ARG, "B = 64"),
+        ("N too large", lambda: fwd(P((1 << 31), 64, 128, 16)), alr.ALR_ERR_INVALID_ARG, "too large"),
+        ("d not a multiple of 8", lambda: fwd(P(32, 60, 128, 16)), alr.ALR_ERR_INVALID_ARG, "d = 60"),
+        ("V too small", lambda: fwd(P(32, 64, 0, 16)), alr.ALR_ERR_INVALID_ARG, "V = 0"),
+        ("gamma", lambda: fwd(P(32, 64, 128, 16, gamma=0.0)), alr.ALR_ERR_INVALID_ARG, "gamma"),
+        ("lambda NaN", lambda: fwd(P(32, 64, 128, 16, lam=float("nan"))), alr.ALR_ERR_INVALID_ARG,
+         "lambda"),
+        ("NULL head", lambda: fwd(P(32, 64, 128, 16), w=None), alr.ALR_ERR_INVALID_ARG, "non-NULL"),
+        ("misaligned Ht", lambda: fwd(P(32, 64, 128, 16), ht=MIS), alr.ALR_ERR_INVALID_ARG,
+         "16-byte aligned"),
+        ("erase without tokens", lambda: fwd(P(32, 64, 128, 16, mode=1)), alr.ALR_ERR_INVALID_ARG,
+         "corpus_tok"),
+        ("gemm Nc % 4", lambda: lib.alr_gemm(alr.ALR_BF16, 0, 0, 0, A16, A16, A16, 8, 6, 64, None),
+         alr.ALR_ERR_INVALID_ARG, "Nc % 4"),
+        ("gemm tf32 MN-major", lambda: lib.alr_gemm(alr.ALR_F32, 1, 0, 0, A16, A16, A16, 8, 8, 8,
+                                                    None), alr.ALR_ERR_UNSUPPORTED, "K-major"),
+        ("gemm misaligned C", lambda: lib.alr_gemm(alr.ALR_BF16, 0, 0, 0, A16, A16, MIS, 8, 8, 64,
+                                                   None), alr.ALR_ERR_INVALID_ARG, "aligned"),
+        ("gather row bytes", lambda: lib.alr_gather_ira_blocks(A16, 1, 8, 12, alr.ALR_BF16, A16, A16,
+                                                               None, 4, 16, A16, None, None),
+         alr.ALR_ERR_INVALID_ARG, "16 bytes"),
+        ("gather NULL out", lambda: lib.alr_gather_ira_blocks(A16, 1, 8, 64, alr.ALR_BF16, A16, A16,
+                                                              None, 4, 16, None, None, None),
+         alr.ALR_ERR_INVALID_ARG, "non-NULL"),
+        ("accept B", lambda: lib.alr_accept_len(A16, A16, None, 4, 33, A16, None, None),
+         alr.ALR_ERR_INVALID_ARG, "B=33"),
+        ("erase gamma", lambda: lib.alr_erase_weights(A16, None, None, None, 4, 16, 0.0, 0, A16,
+                                                      None), alr.ALR_ERR_INVALID_ARG, "gamma"),
+        ("hard gate inputs", lambda: lib.alr_erase_weights(None, None, None, None, 4, 16, 2.0, 1,
+                                                           A16, None),
+         alr.ALR_ERR_INVALID_ARG, "corpus_tok and argmax_t"),
+        ("ira K", lambda: lib.alr_ira_blocks(2, 1, 8, A16, A16, A16, None, None, A16, A16, A16,
+                                             None, None, None), alr.ALR_ERR_INVALID_ARG, "K=1"),
+    ]
+    for name, call, code, text in cases:
+        rc = call()
+        msg = lib.alr_last_error().decode()
+        assert rc == code, (name, rc, msg)
+        assert text in msg, (name, msg)
