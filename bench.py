@@ -781,6 +781,12 @@ def run_gpu(args, rank, world, local_rank):
         "phase_ms": phase_ms,
         "fwd": {"rows_per_s": world * wl.N / (phase_ms["fwd"] / 1e3),
                 "tflops_4NdV": 4 * NdV / (phase_ms["fwd"] / 1e3) / 1e12},
+        # each tensor phase against the sustained peak (the phases run inside a long step)
+        "phase_tflops": {ph: {"tflops": fl / (phase_ms[ph] / 1e3) / 1e12,
+                              "frac_of_sustained": fl / (phase_ms[ph] / 1e3) / 1e12
+                              / pk["bf16_sustained"]}
+                         for ph, fl in (("fwd", 4 * NdV), ("dH_gemm", 2 * NdV),
+                                        ("dW_gemm", 2 * NdV))},
         "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved,
                      "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
                      "frac": achieved / pk["bf16_sustained"],
