@@ -334,8 +334,8 @@ def make_inputs(wl, sigma, device, seed):
 
 class Step:
     """Buffers and the sequence of C-ABI calls of one step.  keep: the forward keeps both
-    logit matrices (fp16) and G is computed from them in place of z_d; otherwise G is
-    computed by recomputing both head products."""
+    logit matrices (fp16 relative to 16-column group references) and G is computed from them
+    in place of z_d; otherwise G is computed by recomputing both head products."""
     N_PHASES = 6
     PHASES = ["gather", "fwd", "accept_len", "logit_grad", "dH_gemm", "dW_gemm"]
     KERNELS_PER_STEP = 8   # gather, fwd (loss, combine, finalize), accept, logit grad, dH, dW
@@ -364,8 +364,9 @@ class Step:
         rec(3)
         o = sl.out
         if self.keep:
-            alr.alr_logit_grad_from_logits(sl.params, sl.Zd, sl.Zt, o["weight"], o["weight_sum"],
-                                           o["lse_d"], o["lse_t"], self.G)
+            alr.alr_logit_grad_from_logits(sl.params, sl.Zd, sl.Zt, sl.Zd_ref, sl.Zt_ref,
+                                           o["weight"], o["weight_sum"], o["lse_d"], o["lse_t"],
+                                           self.G)
         else:
             alr.alr_logit_grad(sl.params, x["Hd"], x["Ht"], x["W"], o["weight"],
                                o["weight_sum"], o["lse_d"], o["lse_t"], self.G)
@@ -411,15 +412,15 @@ class TopkStep:
         alr.alr_label_readout(self.params, x["Ht"], x["W"], lab, self.ws_r)
         rec(1)
         alr.alr_topk_loss_fwd_keep_logits(self.params, x["Hd"], x["W"], lab["top_idx"],
-                                          lab["top_prob"], lab["tail"], s.sl.Zd, o, self.ws_f,
-                                          row_mask=x["row_valid"])
+                                          lab["top_prob"], lab["tail"], s.sl.Zd, s.sl.Zd_ref, o,
+                                          self.ws_f, row_mask=x["row_valid"])
         rec(2)
         alr.alr_accept_len(o["argmax_d"], lab["argmax_t"], wl.B, s.sl.acc_len, s.sl.hist,
                            active=x["row_valid"])
         rec(3)
-        alr.alr_topk_logit_grad_from_logits(self.params, s.sl.Zd, lab["top_idx"], lab["top_prob"],
-                                            lab["tail"], o["weight"], o["weight_sum"],
-                                            o["lse_d"], o["tail_q"], s.G)
+        alr.alr_topk_logit_grad_from_logits(self.params, s.sl.Zd, s.sl.Zd_ref, lab["top_idx"],
+                                            lab["top_prob"], lab["tail"], o["weight"],
+                                            o["weight_sum"], o["lse_d"], o["tail_q"], s.G)
         rec(4)
         alr.alr_gemm(s.G, x["W"], s.dH, wl.N, wl.d, wl.V)
         rec(5)
@@ -762,8 +763,9 @@ def run_gpu(args, rank, world, local_rank):
     flops = {"fwd": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
     if not keep:
         flops["logit_grad"] = 4 * NdV
-    # the logit gradient from kept logits streams z_d, z_t (fp16) in and G (bf16) out
-    g_bytes = 6 * wl.N * wl.V
+    # the logit gradient from kept logits streams z_d, z_t (fp16) and their 16-column group
+    # references (fp16) in and G (bf16) out
+    g_bytes = 6 * wl.N * wl.V + 4 * wl.N * ((wl.V + 15) // 16)
     dom = max(flops, key=lambda p: phase_ms[p])
     achieved = flops[dom] / (phase_ms[dom] / 1e3) / 1e12
     out = {

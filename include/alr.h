@@ -238,29 +238,52 @@ int alr_logit_grad(const alr_params* p, const void* Hd, const void* Ht, const vo
  * results costs 2 * N * V logit elements of device memory (fp16 for bf16 inputs: 2 x 9.96 GB
  * at N = 32768, V = 151936) and spares the backward those two products.  The gradient is the
  * one of Eq. 1 with respect to z_d, as in alr_slot_loss_bwd.
+ *
+ * Storage of a kept logit matrix Z of bf16 inputs: fp16 values relative to group references.
+ * The columns of a row go in groups of ALR_KEEP_GROUP; group c of row r has the reference
+ *     R[c, r] = the largest logit of the group, rounded up to fp16,
+ * and each logit is kept as Z[r, v] = fp16(z[r, v] - R[v / 16, r]) (rounded to nearest), so
+ *     z[r, v] = Z[r, v] + R[v / 16, r]   (both fp16, added in fp32).
+ * Rounding then moves z by at most 2^-11 (R - z) instead of 2^-11 |z|: the error is small
+ * exactly where the softmax weight exp(z - lse) is large (lse >= every z of the row), and the
+ * relative error of q = exp(z - lse) stays near 2^-11 (1 + ln(1/q)) however large the logits
+ * are (trained heads reach |z| of 30-40, where plain fp16 would move q by ~2 %).
+ * R is stored group-major: [alr_kept_ref_groups(V), N] fp16 (uint16_t bits), R[c, r] at
+ * c * N + r, so that the forward writes the references of 32 consecutive rows as one run.
+ * fp32 inputs keep plain fp32 logits and no references (their *_ref arguments are ignored
+ * and may be NULL).  |z| must stay below 65504.
  * ------------------------------------------------------------------------------------- */
+#define ALR_KEEP_GROUP 16
+
+/* Number of 16-column groups of a row of V logits, ceil(V / 16): the leading dimension of a
+ * group-reference array [groups, N] (0 for V < 1). */
+int32_t alr_kept_ref_groups(int32_t V);
 
 /*
  * alr_slot_loss_fwd, which also writes the logits z_d = H_d W and z_t = H_t W:
- *   Zd, Zt  [N, V] row-major, fp16 for ALR_BF16 inputs (rounded to nearest from the fp32
- *           accumulators; |z| must stay below 65504, the fp16 range), fp32 for ALR_F32 inputs;
- *           caller-owned, 16-byte aligned, not overlapping any input or output.
+ *   Zd, Zt          [N, V] row-major: fp16 relative to the group references for ALR_BF16
+ *                   inputs, fp32 for ALR_F32 inputs;
+ *   Zd_ref, Zt_ref  [alr_kept_ref_groups(V), N] fp16 group references (ALR_BF16 inputs);
+ *   all caller-owned, 16-byte aligned, not overlapping any input or output.
  * Every other argument, output and error is that of alr_slot_loss_fwd (same workspace size),
  * and the forward outputs are bit-identical to it.
  */
 int alr_slot_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* Ht,
                                   const void* W, const float* row_mask, const int32_t* corpus_tok,
-                                  void* Zd, void* Zt, const alr_fwd_outputs* out, void* workspace,
-                                  size_t ws_bytes, void* stream);
+                                  void* Zd, void* Zt, uint16_t* Zd_ref, uint16_t* Zt_ref,
+                                  const alr_fwd_outputs* out, void* workspace, size_t ws_bytes,
+                                  void* stream);
 
 /*
- * G[r, v] = lambda * omega_r / sum omega * (exp(Zd[r, v] - lse_d[r]) - exp(Zt[r, v] - lse_t[r]))
- * from kept logits (element types as in alr_slot_loss_fwd_keep_logits) and the forward's
- * weight, weight_sum, lse_d, lse_t; G [N, V] has the element type of p->dtype (bf16 / fp32).
- * G may be Zd itself (the gradient then overwrites z_d in place); it must not otherwise
- * overlap Zd or Zt.  Rows with omega_r = 0 (or sum omega = 0) get G = 0.  No workspace.
+ * G[r, v] = lambda * omega_r / sum omega * (exp(z_d[r, v] - lse_d[r]) - exp(z_t[r, v] - lse_t[r]))
+ * from kept logits (Zd, Zt and, for bf16 inputs, Zd_ref, Zt_ref as written by
+ * alr_slot_loss_fwd_keep_logits) and the forward's weight, weight_sum, lse_d, lse_t; G [N, V]
+ * has the element type of p->dtype (bf16 / fp32).  G may be Zd itself (the gradient then
+ * overwrites z_d in place); it must not otherwise overlap Zd, Zt or the references.  Rows with
+ * omega_r = 0 (or sum omega = 0) get G = 0.  No workspace.
  */
 int alr_logit_grad_from_logits(const alr_params* p, const void* Zd, const void* Zt,
+                               const uint16_t* Zd_ref, const uint16_t* Zt_ref,
                                const float* weight, const float* weight_sum, const float* lse_d,
                                const float* lse_t, void* G, void* stream);
 
@@ -273,7 +296,8 @@ size_t alr_bwd_from_logits_workspace_size(const alr_params* p);
  * dW += H_d^T G (dW [d, V] fp32).  Errors as in alr_slot_loss_bwd.
  */
 int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
-                                  const void* Zd, const void* Zt, const float* weight,
+                                  const void* Zd, const void* Zt, const uint16_t* Zd_ref,
+                                  const uint16_t* Zt_ref, const float* weight,
                                   const float* weight_sum, const float* lse_d, const float* lse_t,
                                   void* G, float* dHd, float* dW, void* workspace,
                                   size_t ws_bytes, void* stream);
@@ -367,24 +391,26 @@ int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const 
  * product.
  *
  * alr_topk_loss_fwd_keep_logits: alr_topk_loss_fwd (same arguments, outputs, workspace and
- * errors, bit-identical outputs) that also writes Zd [N, V] row-major, fp16 for ALR_BF16 inputs
- * (|z| < 65504), fp32 for ALR_F32; caller-owned, 16-byte aligned, overlapping nothing else.
+ * errors, bit-identical outputs) that also writes Zd [N, V] and, for ALR_BF16 inputs, its group
+ * references Zd_ref [alr_kept_ref_groups(V), N] in the kept-logit storage described above;
+ * caller-owned, 16-byte aligned, overlapping nothing else.
  */
 int alr_topk_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* W,
                                   const int32_t* top_idx, const float* top_prob, const float* tail,
                                   const float* row_mask, const float* weight_in, void* Zd,
-                                  const alr_topk_fwd_outputs* out, void* workspace,
-                                  size_t ws_bytes, void* stream);
+                                  uint16_t* Zd_ref, const alr_topk_fwd_outputs* out,
+                                  void* workspace, size_t ws_bytes, void* stream);
 
 /*
- * G of the top-k + tail loss from kept z_d (types as above) and the forward's weight,
- * weight_sum, lse_d, tail_q: G = c_r beta_r q outside the row's label tokens and
+ * G of the top-k + tail loss from kept z_d (Zd and, for bf16 inputs, Zd_ref) and the
+ * forward's weight, weight_sum, lse_d, tail_q: G = c_r beta_r q outside the row's label tokens and
  * c_r (q - top_prob) at them, q = exp(z_d - lse_d), c_r = lambda omega_r / sum omega,
  * beta_r = 1 - tail_r / tail_q_r.  G [N, V] (bf16 / fp32) may be Zd itself (in place); it must
  * not otherwise overlap Zd.  A row's label tokens must be distinct.  No workspace.
  */
-int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const int32_t* top_idx,
-                                    const float* top_prob, const float* tail, const float* weight,
+int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const uint16_t* Zd_ref,
+                                    const int32_t* top_idx, const float* top_prob,
+                                    const float* tail, const float* weight,
                                     const float* weight_sum, const float* lse_d,
                                     const float* tail_q, void* G, void* stream);
 
@@ -394,7 +420,8 @@ int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const i
  * Workspace: alr_bwd_from_logits_workspace_size.
  */
 int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
-                                  const void* Zd, const int32_t* top_idx, const float* top_prob,
+                                  const void* Zd, const uint16_t* Zd_ref,
+                                  const int32_t* top_idx, const float* top_prob,
                                   const float* tail, const float* weight, const float* weight_sum,
                                   const float* lse_d, const float* tail_q, void* G, float* dHd,
                                   float* dW, void* workspace, size_t ws_bytes, void* stream);

@@ -68,15 +68,16 @@ SIGNATURES = {
     "alr_logit_grad_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_logit_grad": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_sz, _c_p]),
+    "alr_kept_ref_groups": (_c_i32, [_c_i32]),
     "alr_slot_loss_fwd_keep_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p,
-                                               _c_p, _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                                ctypes.POINTER(AlrFwdOutputs), _c_p, _c_sz, _c_p]),
     "alr_logit_grad_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
-                                            _c_p, _c_p, _c_p, _c_p]),
+                                            _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]),
     "alr_bwd_from_logits_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_slot_loss_bwd_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
                                                _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
-                                               _c_sz, _c_p]),
+                                               _c_p, _c_p, _c_sz, _c_p]),
     "alr_readout_workspace_size": (_c_sz, [ctypes.POINTER(AlrParams)]),
     "alr_label_readout": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
@@ -88,14 +89,14 @@ SIGNATURES = {
     "alr_topk_loss_bwd": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                    _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_topk_loss_fwd_keep_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
-                                               _c_p, _c_p, _c_p, _c_p,
+                                               _c_p, _c_p, _c_p, _c_p, _c_p,
                                                ctypes.POINTER(AlrTopkFwdOutputs), _c_p, _c_sz,
                                                _c_p]),
     "alr_topk_logit_grad_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
-                                                 _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]),
+                                                 _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]),
     "alr_topk_loss_bwd_from_logits": (_c_int, [ctypes.POINTER(AlrParams), _c_p, _c_p, _c_p, _c_p,
                                                _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
-                                               _c_p, _c_p, _c_sz, _c_p]),
+                                               _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_ira_blocks": (_c_int, [_c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
@@ -325,8 +326,22 @@ def _logits(params, Z, name):
     return _ptr(Z, name, params.N * params.V, _logit_dtype(params))
 
 
-def alr_slot_loss_fwd_keep_logits(params, Hd, Ht, W, Zd, Zt, out: dict, workspace, row_mask=None,
-                                  corpus_tok=None, stream=None):
+def alr_kept_ref_groups(V) -> int:
+    """16-column groups of a row of V logits: the leading dimension of a kept-logit
+    group-reference array [groups, N]."""
+    return lib().alr_kept_ref_groups(int(V))
+
+
+def _refs(params, R, name):
+    """Group references of kept fp16 logits: [alr_kept_ref_groups(V), N] float16 (bf16 inputs);
+    fp32 inputs keep plain logits and pass None."""
+    if params.dtype != ALR_BF16:
+        return _ptr(R, name)
+    return _ptr(R, name, params.N * alr_kept_ref_groups(params.V), torch.float16)
+
+
+def alr_slot_loss_fwd_keep_logits(params, Hd, Ht, W, Zd, Zt, Zd_ref, Zt_ref, out: dict,
+                                  workspace, row_mask=None, corpus_tok=None, stream=None):
     N = params.N
     hd, ht, w = _heads(params, Hd, Ht, W)
     o = _fwd_outputs(params, out)
@@ -334,14 +349,19 @@ def alr_slot_loss_fwd_keep_logits(params, Hd, Ht, W, Zd, Zt, out: dict, workspac
                                                _ptr(row_mask, "row_mask", N, _F32),
                                                _ptr(corpus_tok, "corpus_tok", N, _I32),
                                                _logits(params, Zd, "Zd"), _logits(params, Zt, "Zt"),
+                                               _refs(params, Zd_ref, "Zd_ref"),
+                                               _refs(params, Zt_ref, "Zt_ref"),
                                                ctypes.byref(o), _ws(workspace),
                                                _nbytes(workspace), _stream(stream)))
 
 
-def alr_logit_grad_from_logits(params, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, stream=None):
+def alr_logit_grad_from_logits(params, Zd, Zt, Zd_ref, Zt_ref, weight, weight_sum, lse_d, lse_t, G,
+                               stream=None):
     wt, ws_, ld, lt = _row_stats(params, weight, weight_sum, lse_d, lse_t)
     _check(lib().alr_logit_grad_from_logits(ctypes.byref(params), _logits(params, Zd, "Zd"),
-                                            _logits(params, Zt, "Zt"), wt, ws_, ld, lt,
+                                            _logits(params, Zt, "Zt"),
+                                            _refs(params, Zd_ref, "Zd_ref"),
+                                            _refs(params, Zt_ref, "Zt_ref"), wt, ws_, ld, lt,
                                             _grad_matrix(params, G), _stream(stream)))
 
 
@@ -349,14 +369,16 @@ def alr_bwd_from_logits_workspace_size(params) -> int:
     return lib().alr_bwd_from_logits_workspace_size(ctypes.byref(params))
 
 
-def alr_slot_loss_bwd_from_logits(params, Hd, W, Zd, Zt, weight, weight_sum, lse_d, lse_t, G, dHd,
-                                  dW, workspace=None, stream=None):
+def alr_slot_loss_bwd_from_logits(params, Hd, W, Zd, Zt, Zd_ref, Zt_ref, weight, weight_sum, lse_d,
+                                  lse_t, G, dHd, dW, workspace=None, stream=None):
     hd, _, w = _heads(params, Hd, None, W)
     wt, ws_, ld, lt = _row_stats(params, weight, weight_sum, lse_d, lse_t)
     dh, dw = _head_grads(params, dHd, dW)
     _check(lib().alr_slot_loss_bwd_from_logits(ctypes.byref(params), hd, w,
                                                _logits(params, Zd, "Zd"),
-                                               _logits(params, Zt, "Zt"), wt, ws_, ld, lt,
+                                               _logits(params, Zt, "Zt"),
+                                               _refs(params, Zd_ref, "Zd_ref"),
+                                               _refs(params, Zt_ref, "Zt_ref"), wt, ws_, ld, lt,
                                                _grad_matrix(params, G), dh, dw, _ws(workspace),
                                                _nbytes(workspace), _stream(stream)))
 
@@ -424,7 +446,7 @@ def alr_topk_loss_bwd(params, Hd, W, top_idx, top_prob, tail, weight, weight_sum
                                    dh, dw, _ws(workspace), _nbytes(workspace), _stream(stream)))
 
 
-def alr_topk_loss_fwd_keep_logits(params, Hd, W, top_idx, top_prob, tail, Zd, out: dict,
+def alr_topk_loss_fwd_keep_logits(params, Hd, W, top_idx, top_prob, tail, Zd, Zd_ref, out: dict,
                                   workspace, row_mask=None, weight_in=None, stream=None):
     N = params.N
     hd, _, w = _heads(params, Hd, None, W)
@@ -433,27 +455,31 @@ def alr_topk_loss_fwd_keep_logits(params, Hd, W, top_idx, top_prob, tail, Zd, ou
                                                *_labels(params, top_idx, top_prob, tail),
                                                _ptr(row_mask, "row_mask", N, _F32),
                                                _ptr(weight_in, "weight_in", N, _F32),
-                                               _logits(params, Zd, "Zd"), ctypes.byref(o),
+                                               _logits(params, Zd, "Zd"),
+                                               _refs(params, Zd_ref, "Zd_ref"), ctypes.byref(o),
                                                _ws(workspace), _nbytes(workspace),
                                                _stream(stream)))
 
 
-def alr_topk_logit_grad_from_logits(params, Zd, top_idx, top_prob, tail, weight, weight_sum,
-                                    lse_d, tail_q, G, stream=None):
+def alr_topk_logit_grad_from_logits(params, Zd, Zd_ref, top_idx, top_prob, tail, weight,
+                                    weight_sum, lse_d, tail_q, G, stream=None):
     wt, ws_, ld, tq = _row_stats(params, weight, weight_sum, lse_d, tail_q, "tail_q")
     _check(lib().alr_topk_logit_grad_from_logits(ctypes.byref(params), _logits(params, Zd, "Zd"),
+                                                 _refs(params, Zd_ref, "Zd_ref"),
                                                  *_labels(params, top_idx, top_prob, tail),
                                                  wt, ws_, ld, tq, _grad_matrix(params, G),
                                                  _stream(stream)))
 
 
-def alr_topk_loss_bwd_from_logits(params, Hd, W, Zd, top_idx, top_prob, tail, weight, weight_sum,
-                                  lse_d, tail_q, G, dHd, dW, workspace=None, stream=None):
+def alr_topk_loss_bwd_from_logits(params, Hd, W, Zd, Zd_ref, top_idx, top_prob, tail, weight,
+                                  weight_sum, lse_d, tail_q, G, dHd, dW, workspace=None,
+                                  stream=None):
     hd, _, w = _heads(params, Hd, None, W)
     wt, ws_, ld, tq = _row_stats(params, weight, weight_sum, lse_d, tail_q, "tail_q")
     dh, dw = _head_grads(params, dHd, dW)
     _check(lib().alr_topk_loss_bwd_from_logits(ctypes.byref(params), hd, w,
                                                _logits(params, Zd, "Zd"),
+                                               _refs(params, Zd_ref, "Zd_ref"),
                                                *_labels(params, top_idx, top_prob, tail),
                                                wt, ws_, ld, tq, _grad_matrix(params, G), dh, dw,
                                                _ws(workspace), _nbytes(workspace),
@@ -519,9 +545,10 @@ def alr_gemm(A, B, C, M, Nc, K, a_mn=False, b_mn=False, accumulate=False, stream
 class SlotLoss:
     """Owns the outputs and workspaces of the slot-loss calls for one problem size.
 
-    keep_logits: the forward also writes z_d and z_t (``self.Zd``, ``self.Zt``) and the
-    backward computes G from them in place of z_d instead of recomputing the head products;
-    each forward then allows one backward."""
+    keep_logits: the forward also writes z_d and z_t (``self.Zd``, ``self.Zt``, with their
+    fp16 group references ``self.Zd_ref``, ``self.Zt_ref`` for bf16 inputs) and the backward
+    computes G from them in place of z_d instead of recomputing the head products; each
+    forward then allows one backward."""
     N: int
     d: int
     V: int
@@ -546,11 +573,15 @@ class SlotLoss:
         self.ws_fwd = torch.empty(max(alr_fwd_workspace_size(self.params), 16), dtype=torch.uint8,
                                   device=dev)
         self._ws_bwd = None
-        self.Zd = self.Zt = None
+        self.Zd = self.Zt = self.Zd_ref = self.Zt_ref = None
         if self.keep_logits:
             lt = logits_dtype(self.dtype)
             self.Zd = torch.empty(N, self.V, dtype=lt, device=dev)
             self.Zt = torch.empty(N, self.V, dtype=lt, device=dev)
+            if self.dtype == torch.bfloat16:
+                ng = alr_kept_ref_groups(self.V)
+                self.Zd_ref = torch.empty(ng, N, dtype=torch.float16, device=dev)
+                self.Zt_ref = torch.empty(ng, N, dtype=torch.float16, device=dev)
         self.acc_len = torch.empty(N // self.B, dtype=torch.int32, device=dev)
         self.hist = torch.empty(self.B + 1, dtype=torch.int64, device=dev)
 
@@ -563,9 +594,9 @@ class SlotLoss:
 
     def forward(self, Hd, Ht, W, row_mask=None, corpus_tok=None, stream=None):
         if self.keep_logits:
-            alr_slot_loss_fwd_keep_logits(self.params, Hd, Ht, W, self.Zd, self.Zt, self.out,
-                                          self.ws_fwd, row_mask=row_mask, corpus_tok=corpus_tok,
-                                          stream=stream)
+            alr_slot_loss_fwd_keep_logits(self.params, Hd, Ht, W, self.Zd, self.Zt, self.Zd_ref,
+                                          self.Zt_ref, self.out, self.ws_fwd, row_mask=row_mask,
+                                          corpus_tok=corpus_tok, stream=stream)
         else:
             alr_slot_loss_fwd(self.params, Hd, Ht, W, self.out, self.ws_fwd, row_mask=row_mask,
                               corpus_tok=corpus_tok, stream=stream)
@@ -582,9 +613,10 @@ class SlotLoss:
             if self._ws_bwd is None:
                 n = alr_bwd_from_logits_workspace_size(self.params)
                 self._ws_bwd = torch.empty(max(n, 16), dtype=torch.uint8, device=self.device)
-            alr_slot_loss_bwd_from_logits(self.params, Hd, W, self.Zd, self.Zt, o["weight"],
-                                          o["weight_sum"], o["lse_d"], o["lse_t"], self.G, dHd,
-                                          dW, self._ws_bwd, stream=stream)
+            alr_slot_loss_bwd_from_logits(self.params, Hd, W, self.Zd, self.Zt, self.Zd_ref,
+                                          self.Zt_ref, o["weight"], o["weight_sum"], o["lse_d"],
+                                          o["lse_t"], self.G, dHd, dW, self._ws_bwd,
+                                          stream=stream)
             return
         alr_slot_loss_bwd(self.params, Hd, Ht, W, o["weight"], o["weight_sum"], o["lse_d"],
                           o["lse_t"], dHd, dW, self.ws_bwd, stream=stream)

@@ -151,6 +151,19 @@ int check_params(const alr_params* p) {
   return ALR_OK;
 }
 
+// A kept logit matrix and its group references: both needed (and 16-byte aligned) for bf16
+// inputs, whose logits are kept as fp16 relative to the references; fp32 inputs keep plain
+// fp32 logits and ignore `ref`.
+int check_kept(const alr_params* p, const void* Z, const void* ref, const char* name) {
+  if (Z == nullptr || !aligned16(Z))
+    return fail(ALR_ERR_INVALID_ARG, "%s must be non-NULL and 16-byte aligned", name);
+  if (p->dtype == ALR_BF16 && (ref == nullptr || !aligned16(ref)))
+    return fail(ALR_ERR_INVALID_ARG,
+                "%s_ref (the fp16 group references of bf16 inputs) must be non-NULL and "
+                "16-byte aligned", name);
+  return ALR_OK;
+}
+
 // Vocabulary tile width of the fused loss kernels (columns of z_d and of z_t per tile).
 #ifndef ALR_LOSS_BN
 #define ALR_LOSS_BN 256
@@ -371,7 +384,8 @@ int head_map(CUtensorMap* m, const alr_params* p, const void* W, void* wt, cudaS
 // matrices (kModeFwdKeep).
 int fwd_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
              const float* row_mask, const int32_t* corpus_tok, void* Zd, void* Zt,
-             const alr_fwd_outputs* out, void* workspace, size_t ws_bytes, void* stream) {
+             uint16_t* Zd_ref, uint16_t* Zt_ref, const alr_fwd_outputs* out, void* workspace,
+             size_t ws_bytes, void* stream) {
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if (Hd == nullptr || Ht == nullptr || W == nullptr || out == nullptr)
@@ -413,6 +427,8 @@ int fwd_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
   args.zd_out = Zd;
   args.zt_out = Zt;
+  args.zd_ref = Zd_ref;
+  args.zt_ref = Zt_ref;
   // bf16 inputs keep fp16 logits through TMA stores of 16-column x 32-row boxes
   CUtensorMap m_zd = m_w, m_zt = m_w;
   if (Zd != nullptr && dt == ALR_BF16) {
@@ -510,20 +526,26 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
                       const float* row_mask, const int32_t* corpus_tok, const alr_fwd_outputs* out,
                       void* workspace, size_t ws_bytes, void* stream) {
   ALR_RANGE();
-  return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, nullptr, nullptr, out, workspace, ws_bytes,
-                  stream);
+  return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, nullptr, nullptr, nullptr, nullptr, out,
+                  workspace, ws_bytes, stream);
 }
 
 int alr_slot_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* Ht,
                                   const void* W, const float* row_mask, const int32_t* corpus_tok,
-                                  void* Zd, void* Zt, const alr_fwd_outputs* out, void* workspace,
-                                  size_t ws_bytes, void* stream) {
+                                  void* Zd, void* Zt, uint16_t* Zd_ref, uint16_t* Zt_ref,
+                                  const alr_fwd_outputs* out, void* workspace, size_t ws_bytes,
+                                  void* stream) {
   ALR_RANGE();
-  if (Zd == nullptr || Zt == nullptr)
-    return fail(ALR_ERR_INVALID_ARG, "Zd and Zt must be non-NULL");
-  if (!aligned16(Zd) || !aligned16(Zt))
-    return fail(ALR_ERR_INVALID_ARG, "Zd and Zt must be 16-byte aligned");
-  return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, Zd, Zt, out, workspace, ws_bytes, stream);
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if ((rc = check_kept(p, Zd, Zd_ref, "Zd")) != ALR_OK) return rc;
+  if ((rc = check_kept(p, Zt, Zt_ref, "Zt")) != ALR_OK) return rc;
+  return fwd_impl(p, Hd, Ht, W, row_mask, corpus_tok, Zd, Zt, Zd_ref, Zt_ref, out, workspace,
+                  ws_bytes, stream);
+}
+
+int32_t alr_kept_ref_groups(int32_t V) {
+  return V < 1 ? 0 : (V + alr::kKeepGroup - 1) / alr::kKeepGroup;
 }
 
 size_t alr_bwd_workspace_size(const alr_params* p) {
@@ -723,20 +745,22 @@ int alr_slot_loss_bwd(const alr_params* p, const void* Hd, const void* Ht, const
 }
 
 int alr_logit_grad_from_logits(const alr_params* p, const void* Zd, const void* Zt,
+                               const uint16_t* Zd_ref, const uint16_t* Zt_ref,
                                const float* weight, const float* weight_sum, const float* lse_d,
                                const float* lse_t, void* G, void* stream) {
   ALR_RANGE();
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
-  if (Zd == nullptr || Zt == nullptr || G == nullptr || weight == nullptr ||
-      weight_sum == nullptr || lse_d == nullptr || lse_t == nullptr)
+  if ((rc = check_kept(p, Zd, Zd_ref, "Zd")) != ALR_OK) return rc;
+  if ((rc = check_kept(p, Zt, Zt_ref, "Zt")) != ALR_OK) return rc;
+  if (G == nullptr || weight == nullptr || weight_sum == nullptr || lse_d == nullptr ||
+      lse_t == nullptr)
     return fail(ALR_ERR_INVALID_ARG, "a required pointer is NULL");
-  if (!aligned16(Zd) || !aligned16(Zt) || !aligned16(G))
-    return fail(ALR_ERR_INVALID_ARG, "Zd, Zt and G must be 16-byte aligned");
+  if (!aligned16(G)) return fail(ALR_ERR_INVALID_ARG, "G must be 16-byte aligned");
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  cudaError_t e = alr::launch_logits_grad(p->dtype, Zd, Zt, lse_d, lse_t, weight, weight_sum,
-                                          p->lambda, int(p->N), p->V, G,
+  cudaError_t e = alr::launch_logits_grad(p->dtype, Zd, Zt, Zd_ref, Zt_ref, lse_d, lse_t, weight,
+                                          weight_sum, p->lambda, int(p->N), p->V, G,
                                           static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "logit-gradient launch");
   return ALR_OK;
@@ -748,7 +772,8 @@ size_t alr_bwd_from_logits_workspace_size(const alr_params* p) {
 }
 
 int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
-                                  const void* Zd, const void* Zt, const float* weight,
+                                  const void* Zd, const void* Zt, const uint16_t* Zd_ref,
+                                  const uint16_t* Zt_ref, const float* weight,
                                   const float* weight_sum, const float* lse_d, const float* lse_t,
                                   void* G, float* dHd, float* dW, void* workspace,
                                   size_t ws_bytes, void* stream) {
@@ -756,8 +781,8 @@ int alr_slot_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
   // everything is validated before the gradient kernel overwrites anything
   int rc = check_head_grad_args(p, Hd, W, dHd, dW, workspace, ws_bytes);
   if (rc != ALR_OK) return rc;
-  if ((rc = alr_logit_grad_from_logits(p, Zd, Zt, weight, weight_sum, lse_d, lse_t, G,
-                                       stream)) != ALR_OK)
+  if ((rc = alr_logit_grad_from_logits(p, Zd, Zt, Zd_ref, Zt_ref, weight, weight_sum, lse_d,
+                                       lse_t, G, stream)) != ALR_OK)
     return rc;
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
@@ -824,8 +849,9 @@ namespace {
 // The top-k + tail forward; with Zd given the fused kernel also writes z_d (kModeTopkFwdKeep).
 int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
                   const float* top_prob, const float* tail, const float* row_mask,
-                  const float* weight_in, void* Zd, const alr_topk_fwd_outputs* out,
-                  void* workspace, size_t ws_bytes, void* stream) {
+                  const float* weight_in, void* Zd, uint16_t* Zd_ref,
+                  const alr_topk_fwd_outputs* out, void* workspace, size_t ws_bytes,
+                  void* stream) {
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
@@ -851,6 +877,7 @@ int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int3
   args.part = reinterpret_cast<float*>(ws + lay.part_off);
   args.top_idx = top_idx;
   args.zd_out = Zd;
+  args.zd_ref = Zd_ref;
   args.status = alr::device_status_ptr();
   if (args.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
   CUtensorMap m_zd = m_w;
@@ -880,46 +907,50 @@ int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const 
                       const float* weight_in, const alr_topk_fwd_outputs* out, void* workspace,
                       size_t ws_bytes, void* stream) {
   ALR_RANGE();
-  return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, nullptr, out,
-                       workspace, ws_bytes, stream);
+  return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, nullptr, nullptr,
+                       out, workspace, ws_bytes, stream);
 }
 
 int alr_topk_loss_fwd_keep_logits(const alr_params* p, const void* Hd, const void* W,
                                   const int32_t* top_idx, const float* top_prob, const float* tail,
                                   const float* row_mask, const float* weight_in, void* Zd,
-                                  const alr_topk_fwd_outputs* out, void* workspace,
-                                  size_t ws_bytes, void* stream) {
+                                  uint16_t* Zd_ref, const alr_topk_fwd_outputs* out,
+                                  void* workspace, size_t ws_bytes, void* stream) {
   ALR_RANGE();
-  if (Zd == nullptr || !aligned16(Zd))
-    return fail(ALR_ERR_INVALID_ARG, "Zd must be non-NULL and 16-byte aligned");
-  return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, Zd, out,
+  int rc = check_params(p);
+  if (rc != ALR_OK) return rc;
+  if ((rc = check_kept(p, Zd, Zd_ref, "Zd")) != ALR_OK) return rc;
+  return topk_fwd_impl(p, Hd, W, top_idx, top_prob, tail, row_mask, weight_in, Zd, Zd_ref, out,
                        workspace, ws_bytes, stream);
 }
 
-int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const int32_t* top_idx,
-                                    const float* top_prob, const float* tail, const float* weight,
+int alr_topk_logit_grad_from_logits(const alr_params* p, const void* Zd, const uint16_t* Zd_ref,
+                                    const int32_t* top_idx, const float* top_prob,
+                                    const float* tail, const float* weight,
                                     const float* weight_sum, const float* lse_d,
                                     const float* tail_q, void* G, void* stream) {
   ALR_RANGE();
   int rc = check_params(p);
   if (rc != ALR_OK) return rc;
   if ((rc = check_topk_labels(p, top_idx, top_prob, tail)) != ALR_OK) return rc;
-  if (Zd == nullptr || G == nullptr || weight == nullptr || weight_sum == nullptr ||
-      lse_d == nullptr || tail_q == nullptr)
+  if ((rc = check_kept(p, Zd, Zd_ref, "Zd")) != ALR_OK) return rc;
+  if (G == nullptr || weight == nullptr || weight_sum == nullptr || lse_d == nullptr ||
+      tail_q == nullptr)
     return fail(ALR_ERR_INVALID_ARG, "a required pointer is NULL");
-  if (!aligned16(Zd) || !aligned16(G))
-    return fail(ALR_ERR_INVALID_ARG, "Zd and G must be 16-byte aligned");
+  if (!aligned16(G)) return fail(ALR_ERR_INVALID_ARG, "G must be 16-byte aligned");
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;
-  cudaError_t e = alr::launch_topk_logits_grad(p->dtype, Zd, top_idx, top_prob, tail, tail_q,
-                                               lse_d, weight, weight_sum, p->lambda, int(p->N),
-                                               p->V, G, static_cast<cudaStream_t>(stream));
+  cudaError_t e = alr::launch_topk_logits_grad(p->dtype, Zd, Zd_ref, top_idx, top_prob, tail,
+                                               tail_q, lse_d, weight, weight_sum, p->lambda,
+                                               int(p->N), p->V, G,
+                                               static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "top-k logit-gradient launch");
   return ALR_OK;
 }
 
 int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const void* W,
-                                  const void* Zd, const int32_t* top_idx, const float* top_prob,
+                                  const void* Zd, const uint16_t* Zd_ref,
+                                  const int32_t* top_idx, const float* top_prob,
                                   const float* tail, const float* weight, const float* weight_sum,
                                   const float* lse_d, const float* tail_q, void* G, float* dHd,
                                   float* dW, void* workspace, size_t ws_bytes, void* stream) {
@@ -927,8 +958,8 @@ int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
   // everything is validated before the gradient kernel overwrites anything
   int rc = check_head_grad_args(p, Hd, W, dHd, dW, workspace, ws_bytes);
   if (rc != ALR_OK) return rc;
-  if ((rc = alr_topk_logit_grad_from_logits(p, Zd, top_idx, top_prob, tail, weight, weight_sum,
-                                            lse_d, tail_q, G, stream)) != ALR_OK)
+  if ((rc = alr_topk_logit_grad_from_logits(p, Zd, Zd_ref, top_idx, top_prob, tail, weight,
+                                            weight_sum, lse_d, tail_q, G, stream)) != ALR_OK)
     return rc;
   DevInfo info;
   if ((rc = require_sm103(&info)) != ALR_OK) return rc;

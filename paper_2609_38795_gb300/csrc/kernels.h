@@ -31,11 +31,12 @@ struct LossPlan {
 // epilogue thread (structure of arrays, field-major: part[f * n_parts * N + part * N + row]).
 enum PartField {
   kPMd = 0,   // running max of z_d
-  kPSd,       // sum exp(z_d - m_d)
+  kPSd,       // sum exp(z_d - m_d) over the part's columns other than its leader (whose
+              // own term is the exact 1 left out)
   kPMt,       // running max of z_t
-  kPSt,       // sum exp(z_t - m_t)
-  kPU,        // sum exp(z_t - m_t) * z_d
-  kPW,        // sum exp(z_t - m_t) * z_t
+  kPSt,       // same for z_t
+  kPU,        // sum exp(z_t - m_t) * (z_d - m_d)
+  kPW,        // sum exp(z_t - m_t) * (z_t - m_t)
   kPBd,       // best z_d
   kPId,       // its index (int bits)
   kPSecd,     // second-best z_d (any other index)
@@ -86,7 +87,16 @@ struct LossArgs {
   const float* tail_q;        // top-k backward: drafter mass outside the label tokens [N]
   void* zd_out;               // keep modes: z_d (and z_t) [N, V] (fp16 for bf16 inputs, else fp32)
   void* zt_out;
+  uint16_t* zd_ref;           // keep modes, bf16 inputs: fp16 reference of each 16-column group
+  uint16_t* zt_ref;           // of z_d / z_t, group-major [ceil(V / 16), N] (see kKeepGroup)
 };
+
+// Kept fp16 logits are stored relative to a per-group reference: the columns of a row go in
+// groups of kKeepGroup, whose reference R is the group's maximum rounded up to fp16, and each
+// logit is kept as fp16(z - R).  The rounding error then scales with R - z, which is small
+// exactly where exp(z - lse) is large.  The references are stored group-major,
+// R[v / 16, r] at (v / 16) * N + r, so that one warp's 32 rows of a group are contiguous.
+constexpr int kKeepGroup = 16;
 
 // Fused loss kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
 //   a0: the first hidden-state operand (H_d; H_t for the readout), a1: H_t (dual modes).
@@ -155,15 +165,18 @@ cudaError_t launch_topk_combine(const LossPlan& plan, const float* part, const f
                                 int32_t* argmax_d, float* gap_d, float* weight,
                                 double* anchor_part, cudaStream_t s);
 // G = lambda omega_r / sum omega (exp(z_d - lse_d) - exp(z_t - lse_t)) from kept logits
-// (fp16 for dtype 0, fp32 for dtype 1) into G [N, V] (bf16 / fp32); G may be zd itself.
-cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const float* lse_d,
-                               const float* lse_t, const float* weight, const float* weight_sum,
-                               float lam, int N, int V, void* G, cudaStream_t s);
-// Gradient of the top-k + tail soft CE from kept z_d (fp16 for dtype 0, fp32 for dtype 1):
+// (dtype 0: fp16 values plus the group references zd_ref / zt_ref [ceil(V / 16), N];
+// dtype 1: fp32, references unused) into G [N, V] (bf16 / fp32); G may be zd itself.
+cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const uint16_t* zd_ref,
+                               const uint16_t* zt_ref, const float* lse_d, const float* lse_t,
+                               const float* weight, const float* weight_sum, float lam, int N,
+                               int V, void* G, cudaStream_t s);
+// Gradient of the top-k + tail soft CE from kept z_d (as in launch_logits_grad):
 // G = c_r beta_r q outside the row's label tokens, c_r (q - prob_i) at label token i, with
 // q = exp(z_d - lse_d), c_r = lambda omega_r / sum omega, beta_r = 1 - tail_r / tail_q_r (1 when
 // tail_r = 0).  G (bf16 / fp32) may be zd itself.
-cudaError_t launch_topk_logits_grad(int dtype, const void* zd, const int32_t* top_idx,
+cudaError_t launch_topk_logits_grad(int dtype, const void* zd, const uint16_t* zd_ref,
+                                    const int32_t* top_idx,
                                     const float* top_prob, const float* tail, const float* tail_q,
                                     const float* lse_d, const float* weight,
                                     const float* weight_sum, float lam, int N, int V, void* G,

@@ -8,9 +8,9 @@
 //                the soft cross-entropy of Eq. 1, greedy top-2 with lowest-index ties, z_t at
 //                the corpus token), one partial record per row, vocabulary split and 64-column
 //                group;
-//   kModeFwdKeep the same, and both logit tiles are also written to global memory (fp16 for
-//                bf16 inputs, fp32 for fp32 inputs) so that the backward need not recompute
-//                them;
+//   kModeFwdKeep the same, and both logit tiles are also written to global memory (fp16
+//                relative to per-16-column-group references for bf16 inputs, fp32 for fp32
+//                inputs) so that the backward need not recompute them;
 //   kModeBwd     the same two tiles recomputed: G = lambda omega_r / sum omega (q - p), the
 //                gradient of Eq. 1 with respect to z_d;
 //   kModeReadout z_t only: log-sum-exp and the k most probable tokens (the label a rollout
@@ -18,7 +18,7 @@
 //   kModeTopkFwd z_d only: log-sum-exp, greedy top-2 and z_d at the row's k label tokens (the
 //                top-k + tail-bin soft CE of Sec. 3.1);
 //   kModeTopkBwd z_d only, recomputed: the gradient of that loss;
-//   kModeTopkFwdKeep  kModeTopkFwd that also writes z_d (fp16 for bf16 inputs, fp32 else).
+//   kModeTopkFwdKeep  kModeTopkFwd that also writes z_d (as kModeFwdKeep).
 //
 // Accumulators: 2 x kBN TMEM columns per tile (single-buffered at kBN = 256).  The dual modes
 // hold z_d and z_t of one 128-row block; the single-operand modes (readout, top-k) hold one
@@ -175,20 +175,28 @@ ALR_DEV void lse_update(float& m, float& s, const float (&z)[16], float cm) {
 
 // Greedy top-2 with lowest-index ties, given the sub-chunk maximum cm.  Columns reach a
 // thread in increasing order, so an equal later value never takes the lead.
+ALR_DEV int first_at(const float (&z)[16], float cm) {
+  int jj = kSub - 1;
+#pragma unroll
+  for (int j = kSub - 1; j >= 0; --j) jj = (z[j] == cm) ? j : jj;
+  return jj;
+}
+
+// top2_update for a sub-chunk whose new leader (cm > best) sits at column jj.
+ALR_DEV void top2_lead(float& best, float& sec, int& idx, const float (&z)[16], float cm, int jj,
+                       int v0) {
+  float c2 = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < kSub; ++j) c2 = fmaxf(c2, j == jj ? -INFINITY : z[j]);
+  sec = fmaxf(best, c2);
+  best = cm;
+  idx = v0 + jj;
+}
+
 ALR_DEV void top2_update(float& best, float& sec, int& idx, const float (&z)[16], float cm,
                          int v0) {
   sec = fmaxf(sec, fminf(cm, best));
-  if (cm > best) {  // a new leader in this sub-chunk: find its first position and runner-up
-    int jj = kSub - 1;
-#pragma unroll
-    for (int j = kSub - 1; j >= 0; --j) jj = (z[j] == cm) ? j : jj;
-    float c2 = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < kSub; ++j) c2 = fmaxf(c2, j == jj ? -INFINITY : z[j]);
-    sec = fmaxf(best, c2);
-    best = cm;
-    idx = v0 + jj;
-  }
+  if (cm > best) top2_lead(best, sec, idx, z, cm, first_at(z, cm), v0);  // a new leader
 }
 
 // Insert (v, i) into a list sorted by value descending; an equal value stays below the
@@ -209,74 +217,111 @@ ALR_DEV void topk_insert(float (&t)[kTopK], int (&ti)[kTopK], float v, int i) {
 }
 
 // Running statistics of one row over the columns one thread sees (full-vocabulary forward).
-// best_x is both the greedy top-1 and the online-softmax reference of side x; s_x sums
-// exp(z_x - best_x); u and w sum exp(z_t - best_t) * z_d and * z_t.
+// best_x is both the greedy top-1 (the leader) and the online-softmax reference of side x.
+// r_x sums exp(z_x - best_x) over the columns other than the leader, whose own term is the
+// exact 1 (the whole sum is 1 + r_x): once the row's maximum is in, a plain running sum sits at
+// 1 + small and every added term would lose up to half a unit of 1, while r_x keeps the small
+// part, which is what a near-zero loss or entropy is made of, at full relative precision.
+// u and w sum exp(z_t - best_t) * (z_d - best_d) and * (z_t - best_t): measured from the
+// running maxima, the terms that carry weight are near zero, so these sums stay small and
+// precise when the logits are large, and the soft CE comes out as log(1 + r_d) - u / (1 + r_t),
+// a sum of two non-negative terms, instead of a difference of two numbers of the logits' size.
 struct RowStats {
-  float best_d, sec_d, s_d, best_t, sec_t, s_t, u, w, zx;
+  float best_d, sec_d, r_d, best_t, sec_t, r_t, u, w, zx;
   int i_d, i_t;
 };
 
 ALR_DEV void stats_init(RowStats& st) {
   st.best_d = st.sec_d = st.best_t = st.sec_t = -INFINITY;
-  st.s_d = st.s_t = st.u = st.w = 0.f;
+  st.r_d = st.r_t = st.u = st.w = 0.f;
   st.i_d = st.i_t = 0x7fffffff;
   st.zx = qnan();
 }
 
+// Sum of 2^(z_j log2 e + b) over the sub-chunk's columns other than jj (masked columns are -inf
+// and add 0): the rest-sum of a sub-chunk that brings a new leader at jj.
+ALR_DEV float sum_except(const float (&z)[16], float b, int jj) {
+  float e = 0.f;
+#pragma unroll
+  for (int j = 0; j < kSub; ++j) e += (j == jj) ? 0.f : ex2(fmaf(z[j], kLog2e, b));
+  return e;
+}
+
 // Fold one 16-column sub-chunk (nv valid columns) into the full-vocabulary statistics.
+// cd, ct: the sub-chunk's maxima of z_d and z_t (over its valid columns), returned.
 template <bool kFull>
 ALR_DEV void stats_sub(RowStats& st, const uint32_t (&rd)[16], const uint32_t (&rt)[16], int v0,
-                       int nv, int x) {
+                       int nv, int x, float& cd, float& ct) {
   float zd[16], zt[16];
   load_masked<kFull>(zd, rd, nv);
   load_masked<kFull>(zt, rt, nv);
-  const float cd = max16(zd), ct = max16(zt);
-  // target side: rescale to the new running maximum, then add this sub-chunk
-  const float nbt = fmaxf(st.best_t, ct);
-  const float sct = ex2((st.best_t - nbt) * kLog2e);
-  const float bt = -nbt * kLog2e;
-  float s0 = 0.f, s1 = 0.f, u0 = 0.f, u1 = 0.f, w0 = 0.f, w1 = 0.f;
+  cd = max16(zd);
+  ct = max16(zt);
+  const float nbt = fmaxf(st.best_t, ct), nbd = fmaxf(st.best_d, cd);
+  const float bt = -nbt * kLog2e, bd = -nbd * kLog2e;
+  // per column: T = (z_t - nbt) log2 e, D = (z_d - nbd) log2 e, E = 2^T; sums of E, 2^D,
+  // E D and E T (the last two in log2 units, converted once below)
+  float s0 = 0.f, s1 = 0.f, d0 = 0.f, d1 = 0.f, u0 = 0.f, u1 = 0.f, w0 = 0.f, w1 = 0.f;
   if constexpr (kFull) {
-    // even / odd columns in the two lanes of packed registers (same sums as the scalar loop)
-    const uint64_t l2e = f2_pack(kLog2e, kLog2e), b2 = f2_pack(bt, bt);
-    uint64_t S = f2_pack(0.f, 0.f), U = S, Wt = S;
+    // even / odd columns in the two lanes of packed registers
+    const uint64_t l2e = f2_pack(kLog2e, kLog2e), bt2 = f2_pack(bt, bt), bd2 = f2_pack(bd, bd);
+    uint64_t S = f2_pack(0.f, 0.f), SD = S, U = S, Wt = S;
 #pragma unroll
     for (int j = 0; j < kSub; j += 2) {
-      const uint64_t ZT = f2_pack(zt[j], zt[j + 1]), ZD = f2_pack(zd[j], zd[j + 1]);
-      const uint64_t E = f2_ex2(f2_fma(ZT, l2e, b2));
+      const uint64_t T = f2_fma(f2_pack(zt[j], zt[j + 1]), l2e, bt2);
+      const uint64_t D = f2_fma(f2_pack(zd[j], zd[j + 1]), l2e, bd2);
+      const uint64_t E = f2_ex2(T);
       S = f2_add(S, E);
-      U = f2_fma(E, ZD, U);
-      Wt = f2_fma(E, ZT, Wt);
+      SD = f2_add(SD, f2_ex2(D));
+      U = f2_fma(E, D, U);
+      Wt = f2_fma(E, T, Wt);
     }
     f2_unpack(S, s0, s1);
+    f2_unpack(SD, d0, d1);
     f2_unpack(U, u0, u1);
     f2_unpack(Wt, w0, w1);
   } else {
 #pragma unroll
-    for (int j = 0; j < kSub; j += 2) {
+    for (int j = 0; j < kSub; ++j) {
       if (j < nv) {
-        const float e = ex2(fmaf(zt[j], kLog2e, bt));
+        const float T = fmaf(zt[j], kLog2e, bt), D = fmaf(zd[j], kLog2e, bd);
+        const float e = ex2(T);
         s0 += e;
-        u0 = fmaf(e, zd[j], u0);
-        w0 = fmaf(e, zt[j], w0);
-      }
-      if (j + 1 < nv) {
-        const float e = ex2(fmaf(zt[j + 1], kLog2e, bt));
-        s1 += e;
-        u1 = fmaf(e, zd[j + 1], u1);
-        w1 = fmaf(e, zt[j + 1], w1);
+        d0 += ex2(D);
+        u0 = fmaf(e, D, u0);
+        w0 = fmaf(e, T, w0);
       }
     }
   }
-  st.s_t = fmaf(st.s_t, sct, s0 + s1);
-  st.u = fmaf(st.u, sct, u0 + u1);
-  st.w = fmaf(st.w, sct, w0 + w1);
-  // drafter side
-  float m_d = st.best_d;
-  lse_update(m_d, st.s_d, zd, cd);
-  // greedy top-2 of both sides (moves best_d / best_t to the new maxima)
-  top2_update(st.best_d, st.sec_d, st.i_d, zd, cd, v0);
-  top2_update(st.best_t, st.sec_t, st.i_t, zt, ct, v0);
+  // u, w: move to the new references (skipped while nothing has been summed: the old
+  // reference is still -inf), rescale, add this sub-chunk
+  const bool any = st.best_t > -INFINITY;
+  const float u_sh = any ? fmaf(st.best_d - nbd, 1.f + st.r_t, st.u) : 0.f;
+  const float w_sh = any ? fmaf(st.best_t - nbt, 1.f + st.r_t, st.w) : 0.f;
+  const float sct = ex2((st.best_t - nbt) * kLog2e);
+  st.u = fmaf(u_sh, sct, (u0 + u1) * kLn2);
+  st.w = fmaf(w_sh, sct, (w0 + w1) * kLn2);
+  // rest-sums and greedy top-2.  Without a new leader all of the sub-chunk's terms join the
+  // rest.  A new leader (rare: a few times per thread) leaves the sub-chunk's sum, and the old
+  // leader's exact 1 joins the rest, both rescaled to the new reference.
+  if (ct > st.best_t) {
+    const int jj = first_at(zt, ct);
+    const float e = sum_except(zt, bt, jj);
+    st.r_t = any ? fmaf(st.r_t + 1.f, sct, e) : e;
+    top2_lead(st.best_t, st.sec_t, st.i_t, zt, ct, jj, v0);
+  } else {
+    st.r_t += s0 + s1;
+    st.sec_t = fmaxf(st.sec_t, ct);
+  }
+  if (cd > st.best_d) {
+    const int jj = first_at(zd, cd);
+    const float e = sum_except(zd, bd, jj);
+    st.r_d = st.best_d > -INFINITY ? fmaf(st.r_d + 1.f, ex2((st.best_d - nbd) * kLog2e), e) : e;
+    top2_lead(st.best_d, st.sec_d, st.i_d, zd, cd, jj, v0);
+  } else {
+    st.r_d += d0 + d1;
+    st.sec_d = fmaxf(st.sec_d, cd);
+  }
   const int xr = x - v0;
   if (xr >= 0 && xr < (kFull ? kSub : nv)) {
 #pragma unroll
@@ -290,30 +335,45 @@ ALR_DEV uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-ALR_DEV uint32_t pack_f16x2(uint32_t a, uint32_t b) {
-  __half2 h = __floats2half2_rn(f32(a), f32(b));
+// fp16 pair of (a - ref, b - ref), rounded to nearest (one packed subtraction for the pair).
+ALR_DEV uint32_t pack_f16x2(uint32_t a, uint32_t b, uint64_t ref2) {
+  float x, y;
+  f2_unpack(f2_sub(f2_pack(f32(a), f32(b)), ref2), x, y);
+  __half2 h = __floats2half2_rn(x, y);
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// Keep one warp's 32 x 16 sub-chunk of z_d and z_t, fp16 (bf16 inputs): each lane packs its
-// row into the warp's two staging buffers, then one lane issues a TMA store per matrix (rows
-// past N and columns past V are clipped by the tensor maps).  The stores of the previous
-// sub-chunk must have finished reading the buffers first.
-ALR_DEV void keep_logits_staged(const uint32_t (&rd)[16], const uint32_t (&rt)[16],
-                                uint8_t* my_stage, const CUtensorMap* tm_zd,
+// Reference of a kept 16-column group from its maximum cm: cm rounded up to fp16, so that every
+// kept value z - ref is at most 0 and its fp16 rounding error, at most 2^-11 (ref - z), is small
+// exactly for the logits that dominate the softmax.
+ALR_DEV __half group_ref(float cm) { return __float2half_ru(cm); }
+
+// Store the reference of the group at columns v0.. of `row`: references are group-major,
+// [groups, N], so the 32 lanes of a warp (32 consecutive rows) write 64 contiguous bytes.
+ALR_DEV void store_ref(uint16_t* ref, int n, int row, int v0, __half h) {
+  ref[size_t(v0 / kSub) * size_t(n) + size_t(row)] = __half_as_ushort(h);
+}
+
+// One lane's 16 logits relative to `ref`, as two 16-byte fp16 vectors.
+ALR_DEV void pack_rel(uint4* b, const uint32_t (&r)[16], float ref_value) {
+  const uint64_t ref = f2_pack(ref_value, ref_value);
+  b[0] = make_uint4(pack_f16x2(r[0], r[1], ref), pack_f16x2(r[2], r[3], ref),
+                    pack_f16x2(r[4], r[5], ref), pack_f16x2(r[6], r[7], ref));
+  b[1] = make_uint4(pack_f16x2(r[8], r[9], ref), pack_f16x2(r[10], r[11], ref),
+                    pack_f16x2(r[12], r[13], ref), pack_f16x2(r[14], r[15], ref));
+}
+
+// Keep one warp's 32 x 16 sub-chunk of z_d and z_t, fp16 relative to each row's group
+// references (bf16 inputs): each lane packs its row into the warp's two staging buffers, then
+// one lane issues a TMA store per matrix (rows past N and columns past V are clipped by the
+// tensor maps).  The stores of the previous sub-chunk must have finished reading the buffers.
+ALR_DEV void keep_logits_staged(const uint32_t (&rd)[16], const uint32_t (&rt)[16], float ref_d,
+                                float ref_t, uint8_t* my_stage, const CUtensorMap* tm_zd,
                                 const CUtensorMap* tm_zt, int v0, int row0, int lane) {
   if (lane == 0) tma_store_wait_read_all();
   __syncwarp();
-  uint4* bd = reinterpret_cast<uint4*>(my_stage + lane * 32);
-  uint4* bt = reinterpret_cast<uint4*>(my_stage + kGStageBytes + lane * 32);
-  bd[0] = make_uint4(pack_f16x2(rd[0], rd[1]), pack_f16x2(rd[2], rd[3]), pack_f16x2(rd[4], rd[5]),
-                     pack_f16x2(rd[6], rd[7]));
-  bd[1] = make_uint4(pack_f16x2(rd[8], rd[9]), pack_f16x2(rd[10], rd[11]),
-                     pack_f16x2(rd[12], rd[13]), pack_f16x2(rd[14], rd[15]));
-  bt[0] = make_uint4(pack_f16x2(rt[0], rt[1]), pack_f16x2(rt[2], rt[3]), pack_f16x2(rt[4], rt[5]),
-                     pack_f16x2(rt[6], rt[7]));
-  bt[1] = make_uint4(pack_f16x2(rt[8], rt[9]), pack_f16x2(rt[10], rt[11]),
-                     pack_f16x2(rt[12], rt[13]), pack_f16x2(rt[14], rt[15]));
+  pack_rel(reinterpret_cast<uint4*>(my_stage + lane * 32), rd, ref_d);
+  pack_rel(reinterpret_cast<uint4*>(my_stage + kGStageBytes + lane * 32), rt, ref_t);
   fence_proxy_async_smem();
   __syncwarp();
   if (lane == 0) {
@@ -323,18 +383,16 @@ ALR_DEV void keep_logits_staged(const uint32_t (&rd)[16], const uint32_t (&rt)[1
   }
 }
 
-// Keep one warp's 32 x 16 sub-chunk of z_d alone, fp16 (bf16 inputs), through the warp's two
-// staging buffers in turn (the store issued from a buffer two sub-chunks ago must have read it).
-ALR_DEV void keep_one_staged(const uint32_t (&r)[16], uint8_t* my_stage, uint32_t& n_stores,
-                             const CUtensorMap* tm, int v0, int row0, int lane) {
+// Keep one warp's 32 x 16 sub-chunk of z_d alone, fp16 relative to the group references (bf16
+// inputs), through the warp's two staging buffers in turn (the store issued from a buffer two
+// sub-chunks ago must have read it).
+ALR_DEV void keep_one_staged(const uint32_t (&r)[16], float ref, uint8_t* my_stage,
+                             uint32_t& n_stores, const CUtensorMap* tm, int v0, int row0,
+                             int lane) {
   uint8_t* buf = my_stage + (n_stores & 1u) * kGStageBytes;
   if (lane == 0) tma_store_wait_read_le1();
   __syncwarp();
-  uint4* b = reinterpret_cast<uint4*>(buf + lane * 32);
-  b[0] = make_uint4(pack_f16x2(r[0], r[1]), pack_f16x2(r[2], r[3]), pack_f16x2(r[4], r[5]),
-                    pack_f16x2(r[6], r[7]));
-  b[1] = make_uint4(pack_f16x2(r[8], r[9]), pack_f16x2(r[10], r[11]), pack_f16x2(r[12], r[13]),
-                    pack_f16x2(r[14], r[15]));
+  pack_rel(reinterpret_cast<uint4*>(buf + lane * 32), r, ref);
   fence_proxy_async_smem();
   __syncwarp();
   if (lane == 0) {
@@ -701,30 +759,39 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
           const int nv = min(kSub, P.V - v0);
 
           if constexpr (is_fwd(kMode)) {
-            // kept logits first: their packed copies die before the statistics need registers
+            float cd, ct;   // the sub-chunk's maxima, which also give the kept references
+            if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x, cd, ct);
+            else stats_sub<false>(st, r0, r1, v0, nv, x, cd, ct);
             if constexpr (kMode == kModeFwdKeep) {
               if constexpr (kStaged) {
-                keep_logits_staged(r0, r1, my_stage, &tm_g, &tm_g2, v0, rb * kBM + q * 32, lane);
+                const __half hd = group_ref(cd), ht = group_ref(ct);
+                if (row_ok) {
+                  store_ref(args.zd_ref, P.N, row, v0, hd);
+                  store_ref(args.zt_ref, P.N, row, v0, ht);
+                }
+                keep_logits_staged(r0, r1, __half2float(hd), __half2float(ht), my_stage, &tm_g,
+                                   &tm_g2, v0, rb * kBM + q * 32, lane);
               } else if (row_ok) {
                 const size_t off = size_t(row) * size_t(P.V) + size_t(v0);
                 keep_logits_f32(r0, args.zd_out, off, nv);
                 keep_logits_f32(r1, args.zt_out, off, nv);
               }
             }
-            if (nv == kSub) stats_sub<true>(st, r0, r1, v0, kSub, x);
-            else stats_sub<false>(st, r0, r1, v0, nv, x);
           } else if constexpr (kMode == kModeReadout || is_topk_fwd(kMode)) {
-            if constexpr (kMode == kModeTopkFwdKeep) {
-              if constexpr (kStaged) {
-                keep_one_staged(r0, my_stage, n_stores, &tm_g, v0, rb * kBM + q * 32, lane);
-              } else if (row_ok) {
-                keep_logits_f32(r0, args.zd_out, size_t(row) * size_t(P.V) + size_t(v0), nv);
-              }
-            }
             float z[16];
             if (nv == kSub) load_masked<true>(z, r0, nv);
             else load_masked<false>(z, r0, nv);
             const float cm = max16(z);
+            if constexpr (kMode == kModeTopkFwdKeep) {
+              if constexpr (kStaged) {
+                const __half h = group_ref(cm);
+                if (row_ok) store_ref(args.zd_ref, P.N, row, v0, h);
+                keep_one_staged(r0, __half2float(h), my_stage, n_stores, &tm_g, v0,
+                                rb * kBM + q * 32, lane);
+              } else if (row_ok) {
+                keep_logits_f32(r0, args.zd_out, size_t(row) * size_t(P.V) + size_t(v0), nv);
+              }
+            }
             lse_update(m, s, z, cm);
             if constexpr (kMode == kModeReadout) {
               const int xr = x - v0;
@@ -814,9 +881,9 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
         float* o = args.part + part * P.N + row;
         if constexpr (is_fwd(kMode)) {
           o[kPMd * fs] = st.best_d;
-          o[kPSd * fs] = st.s_d;
+          o[kPSd * fs] = st.r_d;
           o[kPMt * fs] = st.best_t;
-          o[kPSt * fs] = st.s_t;
+          o[kPSt * fs] = st.r_t;
           o[kPU * fs] = st.u;
           o[kPW * fs] = st.w;
           o[kPBd * fs] = st.best_d;

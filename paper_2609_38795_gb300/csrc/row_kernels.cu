@@ -97,22 +97,34 @@ __global__ void __launch_bounds__(256) combine_kernel(
   const int r = a * P.B + (active ? lane : 0);
   const size_t fs = size_t(P.n_parts) * P.N;
 
-  float Md = -INFINITY, Sd = 0.f, Mt = -INFINITY, St = 0.f, U = 0.f, Wt = 0.f;
+  // the sums of exponentials are merged in fp64: their logarithms are the near-zero parts of
+  // the loss and the entropy when the softmax is sharp
+  float Md = -INFINITY, Mt = -INFINITY, U = 0.f, Wt = 0.f;
+  double Sd = 0.0, St = 0.0;
   float bd = -INFINITY, secd = -INFINITY, bt = -INFINITY, sect = -INFINITY, zx = quiet_nan();
   int id = 0x7fffffff, it = 0x7fffffff;
   if (active) {
     for (int k = 0; k < P.n_parts; ++k) {
       const float* p = part + size_t(k) * P.N + r;
-      const float md = p[kPMd * fs], sd = p[kPSd * fs];
-      const float nmd = fmaxf(Md, md);
-      Sd = Sd * ex2((Md - nmd) * kLog2e) + sd * ex2((md - nmd) * kLog2e);
-      Md = nmd;
-      const float mt = p[kPMt * fs];
-      const float nmt = fmaxf(Mt, mt);
+      // a part's sum of exponentials is its leader's exact 1 plus the rest it kept
+      const float md = p[kPMd * fs], mt = p[kPMt * fs];
+      const double sd = 1.0 + double(p[kPSd * fs]), st = 1.0 + double(p[kPSt * fs]);
+      const float nmd = fmaxf(Md, md), nmt = fmaxf(Mt, mt);
       const float so = ex2((Mt - nmt) * kLog2e), sn = ex2((mt - nmt) * kLog2e);
-      St = St * so + p[kPSt * fs] * sn;
-      U = U * so + p[kPU * fs] * sn;
-      Wt = Wt * so + p[kPW * fs] * sn;
+      // U, Wt and the parts' u, w are measured from their own maxima (z_d - M_d, z_t - M_t):
+      // move both to the merged references before adding.  A side with no columns yet (its
+      // maximum still -inf: the merge's start, or a part past the vocabulary) adds nothing.
+      const bool have = Mt > -INFINITY, part_has = mt > -INFINITY;
+      const float Uo = have ? fmaf(Md - nmd, float(St), U) : 0.f;
+      const float Wo = have ? fmaf(Mt - nmt, float(St), Wt) : 0.f;
+      const float un = part_has ? fmaf(md - nmd, float(st), p[kPU * fs]) : 0.f;
+      const float wn = part_has ? fmaf(mt - nmt, float(st), p[kPW * fs]) : 0.f;
+      U = Uo * so + un * sn;
+      Wt = Wo * so + wn * sn;
+      Sd = (have ? Sd * double(ex2((Md - nmd) * kLog2e)) : 0.0) +
+           (part_has ? sd * double(ex2((md - nmd) * kLog2e)) : 0.0);
+      St = (have ? St * double(so) : 0.0) + (part_has ? st * double(sn) : 0.0);
+      Md = nmd;
       Mt = nmt;
       // top-2 merge; equal leaders go to the lower token id
       const float b2 = p[kPBd * fs], s2 = p[kPSecd * fs];
@@ -137,9 +149,11 @@ __global__ void __launch_bounds__(256) combine_kernel(
       if (z == z) zx = z;
     }
   }
-  const float lse_d = Md + logf(Sd);
-  const float lse_t = Mt + logf(St);
-  const float loss = lse_d - U / St;
+  const double lsd = log(Sd), lst = log(St);
+  const float lse_d = Md + float(lsd);
+  const float lse_t = Mt + float(lst);
+  // l = lse_d - E_p[z_d] = log S_d - E_p[z_d - M_d]: two non-negative terms, no cancellation
+  const float loss = float(lsd - double(U) / St);
   const float logp = zx - lse_t;
   const bool erase = mode != 0;
   const int x = (erase && active) ? corpus_tok[r] : -1;
@@ -149,7 +163,7 @@ __global__ void __launch_bounds__(256) combine_kernel(
     w = expf(-float(lane) / gamma) * gate;
     if (row_mask != nullptr) w *= row_mask[r];
     loss_row[r] = loss;
-    if (ent_row) ent_row[r] = lse_t - Wt / St;
+    if (ent_row) ent_row[r] = float(lst - double(Wt) / St);
     lse_d_out[r] = lse_d;
     lse_t_out[r] = lse_t;
     argmax_d[r] = id;
@@ -472,12 +486,20 @@ __global__ void __launch_bounds__(256) transpose32_kernel(const float* __restric
 
 // ------------------------------------------------ logit gradient from kept logits ---
 // G[r, v] = c_r (exp(z_d - lse_d) - exp(z_t - lse_t)) with c_r = lambda omega_r / sum omega:
-// the gradient of Eq. 1 with respect to z_d, from the logits the forward wrote.  One block per
-// row, 8 columns per vector (V is a multiple of 8), kLogitsUnroll vectors of each matrix in
-// flight per thread, held raw until all of them have arrived.  G may be the z_d buffer itself:
-// each element is read before the thread that read it overwrites it, and no other thread
-// touches it.  Masked rows (c_r = 0) read nothing.
+// the gradient of Eq. 1 with respect to z_d, from the logits the forward wrote (fp16 values
+// plus their 16-column group references for bf16 inputs: z = value + reference).
+// A block takes 32 rows x 2048 columns: the rows' constants are staged in shared memory, then
+// each pass of the 256 threads streams one row's 2048 columns (an 8-column vector per thread),
+// with kLogitsUnroll rows' loads in flight.  (Blocks of 32 x 2048 measured 6.5 TB/s; staging
+// the block's group references in shared memory first ran at 5.8 TB/s, whole rows per block
+// with the same direct reference loads at 5.4, and tiles of 16 x 4096 or 8 x 8192 slower.)  G may be the z_d buffer itself: each element is read
+// before the thread that read it overwrites it, and no other thread touches it.  Masked rows
+// (c_r = 0) read nothing.
 constexpr int kLogitsUnroll = 4;
+constexpr int kGradRows = 32;
+constexpr int kGradCols = 2048;
+constexpr int kGradGroups = kGradCols / kKeepGroup;
+constexpr int kGradThreads = kGradCols / 8;
 
 // 8 kept logits as loaded: fp16 (bf16 inputs) or fp32 (fp32 inputs).
 template <typename Z>
@@ -528,142 +550,196 @@ __device__ __forceinline__ void store8(float* p, const float (&g)[8]) {
   reinterpret_cast<float4*>(p)[1] = make_float4(g[4], g[5], g[6], g[7]);
 }
 
-template <typename Z, typename Gt>
-__global__ void __launch_bounds__(256, sizeof(Z) == 2 ? 4 : 2) logits_grad_kernel(const Z* zd, const Z* zt,
-                                                             const float* __restrict__ lse_d,
-                                                             const float* __restrict__ lse_t,
-                                                             const float* __restrict__ weight,
-                                                             const float* __restrict__ weight_sum,
-                                                             float lam, int V, Gt* G) {
-  const int row = blockIdx.x;
-  const float ws = *weight_sum;
-  const float c = ws > 0.f ? lam * weight[row] / ws : 0.f;
-  const size_t base = size_t(row) * size_t(V);
-  const int n8 = V / 8;
-  if (c == 0.f) {
-    const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int i = threadIdx.x; i < n8; i += blockDim.x) store8(G + base + 8 * size_t(i), z);
-    return;
-  }
-  const float ad = -lse_d[row] * kLog2e, at = -lse_t[row] * kLog2e;
-  for (int i0 = threadIdx.x; i0 < n8; i0 += kLogitsUnroll * blockDim.x) {
-    Raw8<Z> a[kLogitsUnroll], b[kLogitsUnroll];
-#pragma unroll
-    for (int u = 0; u < kLogitsUnroll; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i < n8) {
-        a[u].load(zd + base + 8 * size_t(i));
-        b[u].load(zt + base + 8 * size_t(i));
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kLogitsUnroll; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i < n8) {
-        float x[8], y[8], g[8];
-        a[u].to_float(x);
-        b[u].to_float(y);
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          g[j] = c * (ex2(fmaf(x[j], kLog2e, ad)) - ex2(fmaf(y[j], kLog2e, at)));
-        store8(G + base + 8 * size_t(i), g);
-      }
-    }
-  }
-}
-
 __device__ __forceinline__ float load1(const __half* p) { return __half2float(*p); }
 __device__ __forceinline__ float load1(const float* p) { return *p; }
 __device__ __forceinline__ void store1(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
 __device__ __forceinline__ void store1(float* p, float v) { *p = v; }
 
-// Gradient of the top-k + tail soft CE from the kept z_d: c beta q over the whole row, then
-// c (q - prob_i) at the row's label tokens, whose logits are read before the row is
-// overwritten (G may be the z_d buffer).  The label tokens of a row are distinct.
-template <typename Z, typename Gt>
-__global__ void __launch_bounds__(256, sizeof(Z) == 2 ? 4 : 2) topk_logits_grad_kernel(
-    const Z* zd, const int32_t* __restrict__ top_idx, const float* __restrict__ top_prob,
-    const float* __restrict__ tail, const float* __restrict__ tail_q,
-    const float* __restrict__ lse_d, const float* __restrict__ weight,
-    const float* __restrict__ weight_sum, float lam, int V, Gt* G) {
-  __shared__ float lab_g[kTopK];
-  __shared__ int lab_v[kTopK];
-  const int row = blockIdx.x;
+// Reference of the group that holds vector i (8 columns; two vectors per 16-column group) of
+// row r, from the group-major array, scaled by log2 e: a warp's 32 vectors of one row read 16
+// groups, and the next rows of the block read the same sectors again (32 rows of a group are
+// 64 contiguous bytes), so the loads go through the read-only cache.  fp32 logits have none.
+template <typename Z>
+__device__ __forceinline__ float ref_l2e(const uint16_t* ref, int N, int g, int r) {
+  if constexpr (sizeof(Z) == 2)
+    return __half2float(__ushort_as_half(__ldg(ref + size_t(g) * size_t(N) + r))) * kLog2e;
+  else
+    return 0.f;
+}
+
+// Row factor c_r = lambda omega_r / sum omega (0 when sum omega = 0).
+__device__ __forceinline__ float row_factor(const float* weight, const float* weight_sum, float lam,
+                                            int r) {
   const float ws = *weight_sum;
-  const float c = ws > 0.f ? lam * weight[row] / ws : 0.f;
-  const size_t base = size_t(row) * size_t(V);
-  const int n8 = V / 8;
-  if (c == 0.f) {
-    const float z[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int i = threadIdx.x; i < n8; i += blockDim.x) store8(G + base + 8 * size_t(i), z);
-    return;
-  }
-  const float ad = -lse_d[row] * kLog2e;
-  const float tl = tail[row];
-  const float cb = c * (tl > 0.f ? 1.f - tl / tail_q[row] : 1.f);
-  if (threadIdx.x < kTopK) {
-    const int v = top_idx[size_t(row) * kTopK + threadIdx.x];
-    lab_v[threadIdx.x] = v;
-    if (v >= 0 && v < V)
-      lab_g[threadIdx.x] = c * (ex2(fmaf(load1(zd + base + v), kLog2e, ad)) -
-                                top_prob[size_t(row) * kTopK + threadIdx.x]);
+  return ws > 0.f ? lam * weight[r] / ws : 0.f;
+}
+
+template <typename Z, typename Gt>
+__global__ void __launch_bounds__(kGradThreads) logits_grad_kernel(
+    const Z* zd, const Z* zt, const uint16_t* __restrict__ zd_ref,
+    const uint16_t* __restrict__ zt_ref, const float* __restrict__ lse_d,
+    const float* __restrict__ lse_t, const float* __restrict__ weight,
+    const float* __restrict__ weight_sum, float lam, int N, int V, Gt* G) {
+  __shared__ float s_c[kGradRows], s_ad[kGradRows], s_at[kGradRows];
+  const int r0 = blockIdx.x * kGradRows, c0 = blockIdx.y * kGradCols;
+  const int nr = min(kGradRows, N - r0), nc = min(kGradCols, V - c0);
+  if (threadIdx.x < nr) {
+    const int r = r0 + threadIdx.x;
+    s_c[threadIdx.x] = row_factor(weight, weight_sum, lam, r);
+    s_ad[threadIdx.x] = -lse_d[r] * kLog2e;
+    s_at[threadIdx.x] = -lse_t[r] * kLog2e;
   }
   __syncthreads();
-  for (int i0 = threadIdx.x; i0 < n8; i0 += kLogitsUnroll * blockDim.x) {
-    Raw8<Z> a[kLogitsUnroll];
+  const int i = threadIdx.x;                   // this thread's 8-column vector of every row
+  if (8 * i >= nc) return;
+  const size_t col = size_t(c0) + 8 * size_t(i);
+  const int g = c0 / kKeepGroup + (i >> 1);
+  for (int rr0 = 0; rr0 < nr; rr0 += kLogitsUnroll) {
+    Raw8<Z> a[kLogitsUnroll], b[kLogitsUnroll];
+    float oa[kLogitsUnroll], ob[kLogitsUnroll];
 #pragma unroll
     for (int u = 0; u < kLogitsUnroll; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i < n8) a[u].load(zd + base + 8 * size_t(i));
+      const int rr = rr0 + u;
+      if (rr < nr && s_c[rr] != 0.f) {
+        const size_t e = size_t(r0 + rr) * size_t(V) + col;
+        a[u].load(zd + e);
+        b[u].load(zt + e);
+        oa[u] = ref_l2e<Z>(zd_ref, N, g, r0 + rr) + s_ad[rr];
+        ob[u] = ref_l2e<Z>(zt_ref, N, g, r0 + rr) + s_at[rr];
+      }
     }
 #pragma unroll
     for (int u = 0; u < kLogitsUnroll; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i < n8) {
-        float x[8], g[8];
-        a[u].to_float(x);
+      const int rr = rr0 + u;
+      if (rr < nr) {
+        const float c = s_c[rr];
+        float gv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (c != 0.f) {
+          float x[8], y[8];
+          a[u].to_float(x);
+          b[u].to_float(y);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) g[j] = cb * ex2(fmaf(x[j], kLog2e, ad));
-        store8(G + base + 8 * size_t(i), g);
+          for (int j = 0; j < 8; ++j)
+            gv[j] = c * (ex2(fmaf(x[j], kLog2e, oa[u])) - ex2(fmaf(y[j], kLog2e, ob[u])));
+        }
+        store8(G + size_t(r0 + rr) * size_t(V) + col, gv);
+      }
+    }
+  }
+}
+
+// Gradient of the top-k + tail soft CE from the kept z_d, tiled like logits_grad_kernel:
+// c beta q over the whole row, then c (q - prob_i) at the row's label tokens inside the block's
+// columns, whose logits are read before the streaming pass overwrites them (G may be the z_d
+// buffer).  The label tokens of a row are distinct.
+template <typename Z, typename Gt>
+__global__ void __launch_bounds__(kGradThreads) topk_logits_grad_kernel(
+    const Z* zd, const uint16_t* __restrict__ zd_ref, const int32_t* __restrict__ top_idx,
+    const float* __restrict__ top_prob, const float* __restrict__ tail,
+    const float* __restrict__ tail_q, const float* __restrict__ lse_d,
+    const float* __restrict__ weight, const float* __restrict__ weight_sum, float lam, int N,
+    int V, Gt* G) {
+  static_assert(kGradRows * kTopK <= kGradThreads, "one thread per label of the block's rows");
+  __shared__ float s_c[kGradRows], s_cb[kGradRows], s_ad[kGradRows];
+  __shared__ float lab_g[kGradRows * kTopK];
+  __shared__ int lab_v[kGradRows * kTopK];
+  const int r0 = blockIdx.x * kGradRows, c0 = blockIdx.y * kGradCols;
+  const int nr = min(kGradRows, N - r0), nc = min(kGradCols, V - c0);
+  if (threadIdx.x < nr) {
+    const int r = r0 + threadIdx.x;
+    const float c = row_factor(weight, weight_sum, lam, r);
+    const float tl = tail[r];
+    s_c[threadIdx.x] = c;
+    s_cb[threadIdx.x] = c * (tl > 0.f ? 1.f - tl / tail_q[r] : 1.f);
+    s_ad[threadIdx.x] = -lse_d[r] * kLog2e;
+  }
+  __syncthreads();
+  {  // the label tokens of the block's rows that fall in its columns, before any overwrite
+    const int rr = threadIdx.x / kTopK, k = threadIdx.x % kTopK;
+    int v = -1;
+    if (rr < nr) {
+      const int r = r0 + rr;
+      v = top_idx[size_t(r) * kTopK + k];
+      if (v >= c0 && v < c0 + nc) {
+        const float z = load1(zd + size_t(r) * size_t(V) + v);
+        const float o = ref_l2e<Z>(zd_ref, N, v / kKeepGroup, r) + s_ad[rr];
+        lab_g[threadIdx.x] = s_c[rr] * (ex2(fmaf(z, kLog2e, o)) - top_prob[size_t(r) * kTopK + k]);
+      } else {
+        v = -1;
+      }
+    }
+    lab_v[threadIdx.x] = v;
+  }
+  __syncthreads();
+  const int i = threadIdx.x;
+  if (8 * i < nc) {
+    const size_t col = size_t(c0) + 8 * size_t(i);
+    const int g = c0 / kKeepGroup + (i >> 1);
+    for (int rr0 = 0; rr0 < nr; rr0 += kLogitsUnroll) {
+      Raw8<Z> a[kLogitsUnroll];
+      float oa[kLogitsUnroll];
+#pragma unroll
+      for (int u = 0; u < kLogitsUnroll; ++u) {
+        const int rr = rr0 + u;
+        if (rr < nr && s_c[rr] != 0.f) {
+          a[u].load(zd + size_t(r0 + rr) * size_t(V) + col);
+          oa[u] = ref_l2e<Z>(zd_ref, N, g, r0 + rr) + s_ad[rr];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kLogitsUnroll; ++u) {
+        const int rr = rr0 + u;
+        if (rr < nr) {
+          const float cb = s_cb[rr];
+          float gv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+          if (s_c[rr] != 0.f) {
+            float x[8];
+            a[u].to_float(x);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) gv[j] = cb * ex2(fmaf(x[j], kLog2e, oa[u]));
+          }
+          store8(G + size_t(r0 + rr) * size_t(V) + col, gv);
+        }
       }
     }
   }
   __syncthreads();
-  if (threadIdx.x < kTopK) {
-    const int v = lab_v[threadIdx.x];
-    if (v >= 0 && v < V) store1(G + base + v, lab_g[threadIdx.x]);
-  }
+  const int v = lab_v[threadIdx.x];
+  if (v >= 0) store1(G + size_t(r0 + threadIdx.x / kTopK) * size_t(V) + v, lab_g[threadIdx.x]);
 }
 
 }  // namespace
 
-cudaError_t launch_topk_logits_grad(int dtype, const void* zd, const int32_t* top_idx,
-                                    const float* top_prob, const float* tail, const float* tail_q,
-                                    const float* lse_d, const float* weight,
-                                    const float* weight_sum, float lam, int N, int V, void* G,
-                                    cudaStream_t s) {
+cudaError_t launch_topk_logits_grad(int dtype, const void* zd, const uint16_t* zd_ref,
+                                    const int32_t* top_idx, const float* top_prob,
+                                    const float* tail, const float* tail_q, const float* lse_d,
+                                    const float* weight, const float* weight_sum, float lam, int N,
+                                    int V, void* G, cudaStream_t s) {
+  const dim3 grid(unsigned((N + kGradRows - 1) / kGradRows), unsigned((V + kGradCols - 1) / kGradCols));
   if (dtype == 0)
-    topk_logits_grad_kernel<__half, __nv_bfloat16><<<N, 256, 0, s>>>(
-        static_cast<const __half*>(zd), top_idx, top_prob, tail, tail_q, lse_d, weight,
-        weight_sum, lam, V, static_cast<__nv_bfloat16*>(G));
+    topk_logits_grad_kernel<__half, __nv_bfloat16><<<grid, kGradThreads, 0, s>>>(
+        static_cast<const __half*>(zd), zd_ref, top_idx, top_prob, tail, tail_q, lse_d, weight,
+        weight_sum, lam, N, V, static_cast<__nv_bfloat16*>(G));
   else
-    topk_logits_grad_kernel<float, float><<<N, 256, 0, s>>>(
-        static_cast<const float*>(zd), top_idx, top_prob, tail, tail_q, lse_d, weight,
-        weight_sum, lam, V, static_cast<float*>(G));
+    topk_logits_grad_kernel<float, float><<<grid, kGradThreads, 0, s>>>(
+        static_cast<const float*>(zd), nullptr, top_idx, top_prob, tail, tail_q, lse_d, weight,
+        weight_sum, lam, N, V, static_cast<float*>(G));
   return cudaGetLastError();
 }
 
-cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const float* lse_d,
-                               const float* lse_t, const float* weight, const float* weight_sum,
-                               float lam, int N, int V, void* G, cudaStream_t s) {
+cudaError_t launch_logits_grad(int dtype, const void* zd, const void* zt, const uint16_t* zd_ref,
+                               const uint16_t* zt_ref, const float* lse_d, const float* lse_t,
+                               const float* weight, const float* weight_sum, float lam, int N,
+                               int V, void* G, cudaStream_t s) {
+  const dim3 grid(unsigned((N + kGradRows - 1) / kGradRows), unsigned((V + kGradCols - 1) / kGradCols));
   if (dtype == 0)
-    logits_grad_kernel<__half, __nv_bfloat16><<<N, 256, 0, s>>>(
-        static_cast<const __half*>(zd), static_cast<const __half*>(zt), lse_d, lse_t, weight,
-        weight_sum, lam, V, static_cast<__nv_bfloat16*>(G));
+    logits_grad_kernel<__half, __nv_bfloat16><<<grid, kGradThreads, 0, s>>>(
+        static_cast<const __half*>(zd), static_cast<const __half*>(zt), zd_ref, zt_ref, lse_d,
+        lse_t, weight, weight_sum, lam, N, V, static_cast<__nv_bfloat16*>(G));
   else
-    logits_grad_kernel<float, float><<<N, 256, 0, s>>>(
-        static_cast<const float*>(zd), static_cast<const float*>(zt), lse_d, lse_t, weight,
-        weight_sum, lam, V, static_cast<float*>(G));
+    logits_grad_kernel<float, float><<<grid, kGradThreads, 0, s>>>(
+        static_cast<const float*>(zd), static_cast<const float*>(zt), nullptr, nullptr, lse_d,
+        lse_t, weight, weight_sum, lam, N, V, static_cast<float*>(G));
   return cudaGetLastError();
 }
 

@@ -14,6 +14,8 @@ Workloads (the paper's head shapes; its corpora are not available, so these stan
                                                 {0.25, 0.5, 1.0}
   erase  bf16  as text8b with sigma 0.5; corpus token = greedy target token, replaced by a
                uniform random token with probability 0.2 per position
+  sharp  any of the above through ``sharpen``: the head scaled so that the logits reach a
+         trained head's magnitude (|z| up to 30-40) instead of the random head's (|z| < 7)
 """
 
 from __future__ import annotations
@@ -124,3 +126,12 @@ def corpus_replacement(N, V, rate, *, device="cpu", seed=0):
 def corpus_tokens(greedy_tok, mask, tok):
     """Corpus token per row: the greedy target token, or the random one where replaced."""
     return torch.where(mask, tok, greedy_tok.to(torch.int32))
+
+
+
+def sharpen(batch, scale=6.0):
+    """A head whose logits reach a trained head's magnitude: W scaled by ``scale`` (rounded
+    once to the input dtype), so that with d = 4096 the logits spread to |z| of 30-40 instead
+    of the random head's |z| < 7.  Returns a new dict; the input dict is untouched."""
+    W = batch["W"]
+    return dict(batch, W=(W.float() * scale).to(W.dtype))

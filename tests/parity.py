@@ -18,6 +18,10 @@ from paper_2609_38795_gb300 import alr
 LOSS_RTOL = 1e-3
 GRAD_RTOL = 2e-2
 NEAR_TIE = 1e-2
+# Elementwise gradient checks: values below fp32's normal range (2^-126 = 1.2e-38), which bf16
+# shares, are flushed to zero by the fp32 exponentials; after the row factor c < 1 anything under
+# about 1e-36 may read 0.
+FLUSH_FLOOR = 1e-36
 
 
 def np64(t):
@@ -98,3 +102,64 @@ def compare_accept(acc_g, hist_g, acc_r, gaps_d, gaps_t, B):
             assert np.array_equal(hist_g, np.bincount(acc_r, minlength=B + 1))
         assert hist_g.sum() == A
     return int((~ok).sum())
+
+
+# ------------------------------------------------------------------ kept logits ---
+KEEP_GROUP = 16
+
+
+def _refs_per_column(R, V):
+    """Group references [groups, rows] spread to one per logit: [rows, V] fp64."""
+    return np.repeat(np64(R).T, KEEP_GROUP, axis=1)[:, :V]
+
+
+def kept_logits(Z, R=None):
+    """Logits a kept matrix holds, in fp64: fp32 values as they are, or fp16 values plus their
+    16-column group references (bf16 inputs, group-major R[g, r]): z[r, v] = Z[r, v] +
+    R[v // 16, r]."""
+    z = np64(Z)
+    return z if R is None else z + _refs_per_column(R, z.shape[1])
+
+
+def fp16_round_up(x):
+    """The smallest fp16 value >= x (elementwise, fp64 in, fp16 out)."""
+    h = x.astype(np.float16)
+    low = h.astype(np.float64) < x
+    h[low] = np.nextafter(h[low], np.float16(np.inf))
+    return h
+
+
+def _group_max(z):
+    rows, V = z.shape
+    n_grp = (V + KEEP_GROUP - 1) // KEEP_GROUP
+    pad = np.full((rows, n_grp * KEEP_GROUP), -np.inf)
+    pad[:, :V] = z
+    return pad.reshape(rows, n_grp, KEEP_GROUP).max(axis=2)
+
+
+def encode_kept(z):
+    """(Z, R) torch fp16 tensors holding fp64 logits z [rows, V] in the kept-logit storage of
+    bf16 inputs: R [groups, rows] = each 16-column group's maximum rounded up to fp16,
+    Z = fp16(z - R)."""
+    R = np.ascontiguousarray(fp16_round_up(_group_max(z)).T)
+    Z = (z - _refs_per_column(torch.from_numpy(R), z.shape[1])).astype(np.float16)
+    return torch.from_numpy(Z), torch.from_numpy(R)
+
+
+def check_kept(Z, R, z_ref):
+    """Kept logits of bf16 inputs (Z [rows, V], R [groups, rows]) against the oracle's fp64
+    logits z_ref:
+      - every stored value is <= 0 (its group reference bounds the group from above);
+      - each reference is the group maximum rounded up to fp16, up to the accumulation error;
+      - |kept - z_ref| <= 2^-11 (R - z_ref) (the fp16 rounding of z - R) plus the fp32
+        accumulation over d of exact bf16 products (1e-4 + 2^-16 |z|, far above its size)."""
+    zs = np64(Z)
+    assert np.all(zs <= 0.0)
+    gmax, gref = _group_max(z_ref), np64(R).T
+    ulp = np.abs(gmax) * 2.0 ** -10 + 2.0 ** -24
+    tol_g = 1e-4 + 2.0 ** -16 * np.abs(gmax)
+    assert np.all(gref >= gmax - tol_g) and np.all(gref <= gmax + ulp + tol_g)
+    ref = _refs_per_column(R, z_ref.shape[1])
+    acc = 1e-4 + 2.0 ** -16 * np.abs(z_ref)
+    err = np.abs(zs + ref - z_ref)
+    assert np.all(err <= 2.0 ** -11 * np.abs(ref - z_ref) + acc), err.max()

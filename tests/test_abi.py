@@ -73,14 +73,26 @@ def test_argument_errors_are_reported_without_a_launch(libalr):
     good = alr.make_params(N=32, d=64, V=128, B=16)
     fake = ctypes.c_void_p(1 << 20)                        # never dereferenced on this path
     rc = lib.alr_slot_loss_bwd_from_logits(ctypes.byref(good), fake, fake, fake, fake, fake,
-                                           fake, fake, fake, fake, None, None, None, 0, None)
+                                           fake, fake, fake, fake, fake, fake, None, None, None,
+                                           0, None)
     assert rc == alr.ALR_ERR_INVALID_ARG
     assert "dHd" in lib.alr_last_error().decode()
     rc = lib.alr_topk_loss_bwd_from_logits(ctypes.byref(good), fake, fake, fake, fake, fake,
-                                           fake, fake, fake, fake, fake, fake, None, None,
+                                           fake, fake, fake, fake, fake, fake, fake, None, None,
                                            None, 0, None)
     assert rc == alr.ALR_ERR_INVALID_ARG
     assert "dHd" in lib.alr_last_error().decode()
+    # kept fp16 logits of bf16 inputs are unreadable without their group references
+    rc = lib.alr_logit_grad_from_logits(ctypes.byref(good), fake, fake, None, fake, fake, fake,
+                                        fake, fake, fake, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    assert "Zd_ref" in lib.alr_last_error().decode()
+    rc = lib.alr_topk_logit_grad_from_logits(ctypes.byref(good), fake, None, fake, fake, fake,
+                                             fake, fake, fake, fake, fake, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
+    assert "Zd_ref" in lib.alr_last_error().decode()
+    # group references: one per 16 logits of a row (the last group may be partial)
+    assert [lib.alr_kept_ref_groups(v) for v in (8, 256, 264, 151936)] == [1, 16, 17, 9496]
 
 
 def test_binding_refuses_host_and_malformed_tensors_before_any_call(libalr):
