@@ -7,6 +7,7 @@
 // runs the very same forward kernels with their scratch placed in a fixed array in device
 // global memory that is part of this library image, so it calls no allocator at all.
 #include <cstdio>
+#include <cuda.h>
 #include <mutex>
 
 #include "alr.h"
@@ -19,8 +20,30 @@ namespace {
 // device address comes from cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char g_fwd_scratch[ALR_NOALLOC_SCRATCH_BYTES];
 
+// The array's device address per device, with the context it was looked up in: a device
+// reset or a new primary context loads the module again at another address, so a cached
+// address is used only while the current context is the one it came from.
 std::mutex g_scratch_mu;
 void* g_scratch_ptr[64] = {nullptr};
+CUcontext g_scratch_ctx[64] = {nullptr};
+
+// The current context of the calling thread (nullptr when it cannot be read: the address is
+// then looked up on every call).
+CUcontext current_context() {
+  using Fn = CUresult (*)(CUcontext*);
+  static Fn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    return (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+               ? reinterpret_cast<Fn>(p)
+               : nullptr;
+  }();
+  CUcontext c = nullptr;
+  if (fn == nullptr || fn(&c) != CUDA_SUCCESS) return nullptr;
+  return c;
+}
 
 }  // namespace
 
@@ -43,7 +66,8 @@ extern "C" int alr_slot_loss_fwd_noalloc(const alr_params* p, const void* Hd, co
              need, size_t(ALR_NOALLOC_SCRATCH_BYTES));
     return alr::set_last_error(ALR_ERR_INVALID_ARG, msg);
   }
-  // Set-up, once per device, with that device current: look up the array's device address.
+  // Set-up, once per device and context, with that device current: look up the array's
+  // device address (cudaGetSymbolAddress also makes sure the module is loaded there).
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess || dev < 0 || dev >= 64) {
@@ -55,7 +79,8 @@ extern "C" int alr_slot_loss_fwd_noalloc(const alr_params* p, const void* Hd, co
   void* scratch = nullptr;
   {
     std::lock_guard<std::mutex> lk(g_scratch_mu);
-    if (g_scratch_ptr[dev] == nullptr) {
+    const CUcontext ctx = current_context();
+    if (g_scratch_ptr[dev] == nullptr || ctx == nullptr || ctx != g_scratch_ctx[dev]) {
       void* ptr = nullptr;
       e = cudaGetSymbolAddress(&ptr, g_fwd_scratch);
       if (e != cudaSuccess || ptr == nullptr) {
@@ -66,6 +91,7 @@ extern "C" int alr_slot_loss_fwd_noalloc(const alr_params* p, const void* Hd, co
         return alr::set_last_error(ALR_ERR_CUDA, msg);
       }
       g_scratch_ptr[dev] = ptr;
+      g_scratch_ctx[dev] = current_context();   // current now, after the runtime call
     }
     scratch = g_scratch_ptr[dev];
   }
