@@ -67,6 +67,8 @@ def parse_args():
                          "result (no step, a little over 2 GB of device memory)")
     ap.add_argument("--anchors", type=int, default=0,
                     help="profiling only: fewer anchors than the workload (config says so)")
+    ap.add_argument("--oracle-rates", action="store_true",
+                    help="internal: print the CPU oracle's rows/s at each workload and exit")
     return ap.parse_args()
 
 
@@ -262,6 +264,54 @@ def time_oracle_single_thread(sigma, n_anchors):
                 "seconds": j["ms_per_step"] / 1e3}
     except (subprocess.SubprocessError, IndexError, ValueError, KeyError) as e:
         return {"unavailable": f"{type(e).__name__}"}
+
+
+ORACLE_WORKLOADS = ("small", "vl7b", "text8b")
+
+
+def oracle_rates(n_anchors, reps=2):
+    """The oracle's forward-only and forward+backward rows/s at each workload's d and V, on
+    n_anchors anchors of seeded CPU inputs (the workload's recipe without a feature buffer);
+    the best of `reps` timings each.  Runs in whatever thread budget the process has."""
+    import numpy as np
+    import torch
+    from oracle import alr_oracle as orc
+    from paper_2609_38795_gb300 import synthetic
+    out = {}
+    for name in ORACLE_WORKLOADS:
+        wl = synthetic.WORKLOADS[name]
+        b = synthetic.slot_batch(wl.d, wl.V, n_anchors, wl.B, wl.sigma, dtype=torch.bfloat16, seed=0)
+        Hd, Ht, W = (b[k].float().numpy() for k in ("Hd", "Ht", "W"))
+        mask = np.ones(n_anchors * wl.B)
+        rows = n_anchors * wl.B
+        t_f, t_s = [], []
+        for _ in range(reps):
+            t0 = time.perf_counter()
+            orc.slot_loss_forward(Hd, Ht, W, wl.B, row_mask=mask)
+            t_f.append(time.perf_counter() - t0)
+            t0 = time.perf_counter()
+            oracle_step(wl, Hd, Ht, W, mask)
+            t_s.append(time.perf_counter() - t0)
+        out[name] = {"fwd": rows / min(t_f), "fwd_bwd": rows / min(t_s)}
+    return out
+
+
+def oracle_rates_child(n_anchors, threads=None):
+    """oracle_rates in a fresh interpreter (never a fork of this CUDA process); threads=1 limits
+    its BLAS and OpenMP pools to one thread.  Returns flat keys for the cpu_baseline record."""
+    env = dict(os.environ, RANK="0", WORLD_SIZE="1")
+    if threads is not None:
+        env.update(OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
+                   MKL_NUM_THREADS=str(threads))
+    cmd = [sys.executable, os.path.abspath(__file__), "--oracle-rates",
+           "--cpu-sample-anchors", str(n_anchors)]
+    suffix = "" if threads is None else f"_{threads}core"
+    try:
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=600)
+        j = json.loads([ln for ln in r.stdout.splitlines() if ln.startswith("{")][-1])
+    except (subprocess.SubprocessError, IndexError, ValueError) as e:
+        return {f"oracle_rates{suffix}": f"unavailable: {type(e).__name__}"}
+    return {f"{kind}_rows_per_s_{wl}{suffix}": v[kind] for wl, v in j.items() for kind in v}
 
 
 # ------------------------------------------------------------- gather bandwidth ---
@@ -750,6 +800,13 @@ def run_gpu(args, rank, world, local_rank):
                          f"workload, full d={wl.d} and V={wl.V}, fwd+bwd in fp64, "
                          f"{len(ts)} repetition(s), {sum(ts):.1f} s",
                "single_thread": time_oracle_single_thread(args.sigma, args.cpu_sample_anchors)}
+        # flat keys: forward-only and forward+backward oracle rates at every workload's d and V,
+        # on all host cores and on one
+        cpu["rates_sample"] = (f"{args.cpu_sample_anchors} anchor(s) x B rows of seeded CPU "
+                               f"inputs per workload, best of 2")
+        cpu.update(oracle_rates_child(args.cpu_sample_anchors))
+        cpu.update(oracle_rates_child(args.cpu_sample_anchors, threads=1))
+        cpu["single_thread_rows_per_s"] = cpu["single_thread"].get("value")
     if rank != 0:
         return None
 
@@ -798,7 +855,8 @@ def run_gpu(args, rank, world, local_rank):
         "logit_grad_hbm": ({"bytes": g_bytes, "GB/s": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9,
                             "frac_of_hbm": g_bytes / (phase_ms["logit_grad"] / 1e3) / 1e9 / pk["hbm"],
                             "traffic": kernel_traffic("logit_grad")} if keep else None),
-        "step": "forward keeps the logits" if keep else "backward recomputes the logits",
+        "step": ("forward keeps the logits (fp16 with group references), the backward reads "
+                 "them" if keep else "backward recomputes the logits"),
         ("recompute" if keep else "keep"): other,
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
@@ -813,6 +871,28 @@ def run_gpu(args, rank, world, local_rank):
         "clocks": clk,
         "cpu_baseline": cpu,
     }
+    # The step the hot path's outline describes (logits never stored; the backward recomputes
+    # its logit tiles), with its own roofline record: timed here as `recompute` beside the
+    # default kept-logits step, or as the main step under --step recompute.
+    ns = other if keep else {"ms_per_step": ms_step, "rows_per_s": rows_per_s, "phase_ms": phase_ms}
+    if ns is not None:
+        ns_flops = {"fwd": 4 * NdV, "logit_grad": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
+        ns_dom = max(ns_flops, key=lambda ph: ns["phase_ms"][ph])
+        ns_ach = ns_flops[ns_dom] / (ns["phase_ms"][ns_dom] / 1e3) / 1e12
+        out["north_star_rows_per_s"] = ns["rows_per_s"]
+        out["north_star"] = {
+            "what": "logits never stored: the forward reduces both logit tiles on chip, the "
+                    "backward recomputes them (12 NdV tensor flops per step)",
+            "rows_per_s": ns["rows_per_s"], "ms_per_step": ns["ms_per_step"],
+            "executed_tflops_12NdV": 12 * NdV / (ns["ms_per_step"] / 1e3) / 1e12,
+            "algorithmic_tflops_8NdV": 8 * NdV / (ns["ms_per_step"] / 1e3) / 1e12,
+            "roofline": {"bound": "tensor", "kernel": ns_dom, "achieved": ns_ach,
+                         "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+                         "frac": ns_ach / pk["bf16_sustained"],
+                         "frac_of_burst_peak": ns_ach / pk["bf16"],
+                         "traffic": kernel_traffic(ns_dom + "_recompute"),
+                         "flops_per_launch": ns_flops[ns_dom],
+                         "peak_note": f"{pk['source']} sustained bf16"}}
     if e2e is not None:
         out["e2e"] = {"value": job_rows_per_s(world, wl.N, K, e2e_ms), "unit": UNIT,
                       "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
@@ -860,6 +940,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.oracle_rates:
+        print(json.dumps(oracle_rates(args.cpu_sample_anchors)), flush=True)
+        return
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args)), flush=True)

@@ -84,6 +84,8 @@ typedef struct {
     float* weight;       /* omega_r, the final slot weight (required)                          */
     float* loss_total;   /* [1] L = lambda * sum omega l / sum omega, 0 when sum omega = 0     */
     float* weight_sum;   /* [1] sum omega (the backward's normaliser)                          */
+    float* wl_sum;       /* [1] sum omega l, the numerator of Eq. 1 (nullable; for sums across
+                            the shards of a batch, see alr_loss_from_sums)                      */
 } alr_fwd_outputs;
 
 /* Library version string (static storage). */
@@ -191,7 +193,9 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
  *     B=16 on a 152-SM GB300: about 16 900 rows).
  *   - Memory: every device that loads the library holds the array until the process exits.
  *   - Set-up: the first call on a device (with that device current) looks up the array's
- *     device address; make that first call before any stream capture.
+ *     device address; make that first call before any stream capture.  The address is kept
+ *     per device and context, so after a device reset or a new primary context the next call
+ *     looks it up again (again, before any capture).
  *   - Sharing: all calls on a device share the one array and it keeps the last call's
  *     contents.  Nothing in it needs clearing (the kernels overwrite what they read), but
  *     calls whose work overlaps on the GPU (different streams, or different host threads
@@ -343,6 +347,7 @@ typedef struct {
     float* weight;       /* omega_r used (required)                                            */
     float* loss_total;   /* [1] L of Eq. 1 times lambda                                        */
     float* weight_sum;   /* [1] sum omega                                                      */
+    float* wl_sum;       /* [1] sum omega l (nullable; as in alr_fwd_outputs)                  */
 } alr_topk_fwd_outputs;
 
 /* Workspace bytes alr_topk_loss_fwd needs for `p` (0 on invalid params). */
@@ -425,6 +430,29 @@ int alr_topk_loss_bwd_from_logits(const alr_params* p, const void* Hd, const voi
                                   const float* tail, const float* weight, const float* weight_sum,
                                   const float* lse_d, const float* tail_q, void* G, float* dHd,
                                   float* dW, void* workspace, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------------
+ * Row-sharded (data-parallel) batches.  Eq. 1 normalises over the whole batch, so when the
+ * anchors of one batch are spread over several ranks (App. A: FSDP data parallelism), each
+ * rank:
+ *   1. runs its forward on its own anchors, with out->wl_sum and out->weight_sum giving its
+ *      partial sums (sum omega l, sum omega);
+ *   2. sums both scalars over the ranks (an all-reduce of 2 floats, by the caller);
+ *   3. calls alr_loss_from_sums on the reduced sums for the batch's L;
+ *   4. runs its backward with weight_sum pointing at the REDUCED sum omega (every backward
+ *      entry point takes it as a device pointer), so that its G = lambda omega_r / sum omega
+ *      (q - p) is its rows' share of the batch gradient;
+ *   5. sums dW over the ranks (dW = H_d^T G is a sum over rows: an all-reduce, or a
+ *      reduce-scatter when the head is sharded), while each rank keeps its own rows of dH.
+ * Accepted-length histograms add up over ranks the same way.
+ * ------------------------------------------------------------------------------------- */
+
+/*
+ * L = lambda * wl_sum / weight_sum, or 0 when weight_sum = 0 (Eq. 1, from sums the caller
+ * reduced over the shards of a batch).  All three are device pointers to one float.
+ */
+int alr_loss_from_sums(const float* wl_sum, const float* weight_sum, float lambda,
+                       float* loss_total, void* stream);
 
 /*
  * Greedy accepted length per anchor (Sec. 3.2: slot k counts only when slots 1..k-1 were

@@ -32,7 +32,7 @@ class AlrParams(ctypes.Structure):
 
 
 _FWD_FIELDS = ("loss_row", "ent_row", "lse_d", "lse_t", "argmax_d", "argmax_t", "gap_d", "gap_t",
-               "logp_x", "weight", "loss_total", "weight_sum")
+               "logp_x", "weight", "loss_total", "weight_sum", "wl_sum")
 
 
 class AlrFwdOutputs(ctypes.Structure):
@@ -40,7 +40,7 @@ class AlrFwdOutputs(ctypes.Structure):
 
 
 _TOPK_FIELDS = ("loss_row", "lse_d", "tail_q", "argmax_d", "gap_d", "weight", "loss_total",
-                "weight_sum")
+                "weight_sum", "wl_sum")
 ALR_TOPK = 8
 
 
@@ -99,6 +99,7 @@ SIGNATURES = {
                                                _c_p, _c_p, _c_p, _c_sz, _c_p]),
     "alr_ira_blocks": (_c_int, [_c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_p]),
+    "alr_loss_from_sums": (_c_int, [_c_p, _c_p, _c_f, _c_p, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
     "alr_erase_weights": (_c_int, [_c_p, _c_p, _c_p, _c_p, _c_i32, _c_i32, _c_f, _c_i32, _c_p,
                                    _c_p]),
@@ -171,14 +172,16 @@ def _fwd_outputs(params, out):
     N = params.N
     spec = dict(loss_row=(N, _F32), ent_row=(N, _F32), lse_d=(N, _F32), lse_t=(N, _F32),
                 argmax_d=(N, _I32), argmax_t=(N, _I32), gap_d=(N, _F32), gap_t=(N, _F32),
-                logp_x=(N, _F32), weight=(N, _F32), loss_total=(1, _F32), weight_sum=(1, _F32))
+                logp_x=(N, _F32), weight=(N, _F32), loss_total=(1, _F32), weight_sum=(1, _F32),
+                wl_sum=(1, _F32))
     return AlrFwdOutputs(**{f: _ptr(out.get(f), f, *spec[f]) for f in _FWD_FIELDS})
 
 
 def _topk_outputs(params, out):
     N = params.N
     spec = dict(loss_row=(N, _F32), lse_d=(N, _F32), tail_q=(N, _F32), argmax_d=(N, _I32),
-                gap_d=(N, _F32), weight=(N, _F32), loss_total=(1, _F32), weight_sum=(1, _F32))
+                gap_d=(N, _F32), weight=(N, _F32), loss_total=(1, _F32), weight_sum=(1, _F32),
+                wl_sum=(1, _F32))
     return AlrTopkFwdOutputs(**{f: _ptr(out.get(f), f, *spec[f]) for f in _TOPK_FIELDS})
 
 
@@ -505,6 +508,14 @@ def alr_ira_blocks(K, max_blocks, valid_anchors, rollout_len, offsets, out: dict
                                 _stream(stream)))
 
 
+def alr_loss_from_sums(wl_sum, weight_sum, lam, loss_total, stream=None):
+    """L = lambda * wl_sum / weight_sum (0 when weight_sum = 0) from reduced sums (one float
+    each, on the device)."""
+    _check(lib().alr_loss_from_sums(_ptr(wl_sum, "wl_sum", 1, _F32),
+                                    _ptr(weight_sum, "weight_sum", 1, _F32), float(lam),
+                                    _ptr(loss_total, "loss_total", 1, _F32), _stream(stream)))
+
+
 def _anchors(t, B, name):
     """Anchor count of a per-row tensor of A*B entries."""
     if B < 1 or t.numel() % B != 0:
@@ -569,7 +580,8 @@ class SlotLoss:
         self.out = dict(loss_row=f(), ent_row=f(), lse_d=f(), lse_t=f(), argmax_d=i(),
                         argmax_t=i(), gap_d=f(), gap_t=f(), logp_x=f(), weight=f(),
                         loss_total=torch.zeros(1, dtype=torch.float32, device=dev),
-                        weight_sum=torch.zeros(1, dtype=torch.float32, device=dev))
+                        weight_sum=torch.zeros(1, dtype=torch.float32, device=dev),
+                        wl_sum=torch.zeros(1, dtype=torch.float32, device=dev))
         self.ws_fwd = torch.empty(max(alr_fwd_workspace_size(self.params), 16), dtype=torch.uint8,
                                   device=dev)
         self._ws_bwd = None
@@ -607,8 +619,12 @@ class SlotLoss:
                        self.hist, active=active, stream=stream)
         return self.acc_len, self.hist
 
-    def backward(self, Hd, Ht, W, dHd, dW=None, stream=None):
-        o = self.out
+    def backward(self, Hd, Ht, W, dHd, dW=None, weight_sum=None, stream=None):
+        """weight_sum: the normaliser sum omega of Eq. 1 (default: this forward's own; a
+        row-sharded batch passes the sum over all its shards)."""
+        o = dict(self.out)
+        if weight_sum is not None:
+            o["weight_sum"] = weight_sum
         if self.keep_logits:
             if self._ws_bwd is None:
                 n = alr_bwd_from_logits_workspace_size(self.params)

@@ -448,7 +448,8 @@ int fwd_impl(const alr_params* p, const void* Hd, const void* Ht, const void* W,
                           out->argmax_t, out->gap_d, out->gap_t, out->logp_x, out->weight, anchor,
                           s);
   if (e != cudaSuccess) return cuda_fail(e, "combine launch");
-  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
+  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum,
+                          out->wl_sum, s);
   if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
   return ALR_OK;
 }
@@ -893,7 +894,8 @@ int topk_fwd_impl(const alr_params* p, const void* Hd, const void* W, const int3
                                out->loss_row, out->lse_d, out->tail_q, out->argmax_d, out->gap_d,
                                out->weight, anchor, s);
   if (e != cudaSuccess) return cuda_fail(e, "top-k combine launch");
-  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum, s);
+  e = alr::launch_finalize(anchor, int(p->N / p->B), p->lambda, out->loss_total, out->weight_sum,
+                          out->wl_sum, s);
   if (e != cudaSuccess) return cuda_fail(e, "finalize launch");
   return ALR_OK;
 }
@@ -1015,6 +1017,21 @@ int alr_topk_loss_bwd(const alr_params* p, const void* Hd, const void* W, const 
                        ws + lay.wt_off, info, s);
   if (rc != ALR_OK) return rc;
   return head_grads_impl(p, Hd, W, G, dHd, dW, ws, lay, info, s);
+}
+
+int alr_loss_from_sums(const float* wl_sum, const float* weight_sum, float lambda,
+                       float* loss_total, void* stream) {
+  ALR_RANGE();
+  if (wl_sum == nullptr || weight_sum == nullptr || loss_total == nullptr)
+    return fail(ALR_ERR_INVALID_ARG, "wl_sum, weight_sum and loss_total must be non-NULL");
+  if (!(lambda == lambda)) return fail(ALR_ERR_INVALID_ARG, "lambda is NaN");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  cudaError_t e = alr::launch_loss_from_sums(wl_sum, weight_sum, lambda, loss_total,
+                                             static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loss-from-sums launch");
+  return ALR_OK;
 }
 
 int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* valid_anchors,

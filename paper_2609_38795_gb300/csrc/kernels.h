@@ -154,7 +154,10 @@ cudaError_t launch_combine(const LossPlan& plan, const float* part, int mode, fl
                            int32_t* argmax_t, float* gap_d, float* gap_t, float* logp_x,
                            float* weight, double* anchor_part, cudaStream_t s);
 cudaError_t launch_finalize(const double* anchor_part, int A, float lam, float* loss_total,
-                            float* weight_sum, cudaStream_t s);
+                            float* weight_sum, float* wl_sum, cudaStream_t s);
+// loss_total = lambda * wl_sum / weight_sum (0 when weight_sum = 0), from reduced sums.
+cudaError_t launch_loss_from_sums(const float* wl_sum, const float* weight_sum, float lam,
+                                  float* loss_total, cudaStream_t s);
 cudaError_t launch_readout_combine(const LossPlan& plan, const float* part, bool has_corpus,
                                    int32_t* top_idx, float* top_prob, float* tail, float* lse_t,
                                    int32_t* argmax_t, float* gap_t, float* logp_x,

@@ -186,11 +186,13 @@ __global__ void __launch_bounds__(256) combine_kernel(
   }
 }
 
-// Batch reduction of Eq. 1 in a fixed order (one block, deterministic).
+// Batch reduction of Eq. 1 in a fixed order (one block, deterministic).  wl_sum (nullable)
+// receives the numerator sum omega l itself, for a sum across the shards of a batch.
 __global__ void __launch_bounds__(1024) finalize_kernel(const double* __restrict__ anchor_part,
                                                         int A, float lam,
                                                         float* __restrict__ loss_total,
-                                                        float* __restrict__ weight_sum) {
+                                                        float* __restrict__ weight_sum,
+                                                        float* __restrict__ wl_sum) {
   __shared__ double s_wl[32], s_ws[32];
   double wl = 0.0, ws = 0.0;
   for (int a = threadIdx.x; a < A; a += blockDim.x) {
@@ -219,8 +221,18 @@ __global__ void __launch_bounds__(1024) finalize_kernel(const double* __restrict
     if (lane == 0) {
       *loss_total = ws > 0.0 ? float(double(lam) * wl / ws) : 0.f;
       *weight_sum = float(ws);
+      if (wl_sum != nullptr) *wl_sum = float(wl);
     }
   }
+}
+
+// Eq. 1 from sums that the caller reduced over the shards of a batch: L = lambda * wl / ws,
+// 0 when ws = 0 (no supervised slot anywhere in the batch).
+__global__ void loss_from_sums_kernel(const float* __restrict__ wl_sum,
+                                      const float* __restrict__ weight_sum, float lam,
+                                      float* __restrict__ loss_total) {
+  const double ws = *weight_sum;
+  *loss_total = ws > 0.0 ? float(double(lam) * double(*wl_sum) / ws) : 0.f;
 }
 
 // ------------------------------------------------------------- accepted length ---
@@ -809,8 +821,14 @@ cudaError_t launch_topk_combine(const LossPlan& plan, const float* part, const f
 }
 
 cudaError_t launch_finalize(const double* anchor_part, int A, float lam, float* loss_total,
-                            float* weight_sum, cudaStream_t s) {
-  finalize_kernel<<<1, 1024, 0, s>>>(anchor_part, A, lam, loss_total, weight_sum);
+                            float* weight_sum, float* wl_sum, cudaStream_t s) {
+  finalize_kernel<<<1, 1024, 0, s>>>(anchor_part, A, lam, loss_total, weight_sum, wl_sum);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_loss_from_sums(const float* wl_sum, const float* weight_sum, float lam,
+                                  float* loss_total, cudaStream_t s) {
+  loss_from_sums_kernel<<<1, 1, 0, s>>>(wl_sum, weight_sum, lam, loss_total);
   return cudaGetLastError();
 }
 

@@ -45,7 +45,8 @@ def test_struct_layouts_match_the_header():
     # alr_params: int64 N, five int32, two floats -> 8 + 20 + 8 = 36, padded to 40
     assert ctypes.sizeof(alr.AlrParams) == 40
     assert alr.AlrParams.lam.offset == 28 and alr.AlrParams.gamma.offset == 32
-    assert ctypes.sizeof(alr.AlrFwdOutputs) == 12 * 8
+    assert ctypes.sizeof(alr.AlrFwdOutputs) == 13 * 8          # 13 pointers
+    assert ctypes.sizeof(alr.AlrTopkFwdOutputs) == 9 * 8
 
 
 def test_argument_errors_are_reported_without_a_launch(libalr):
@@ -91,6 +92,8 @@ def test_argument_errors_are_reported_without_a_launch(libalr):
                                              fake, fake, fake, fake, fake, None)
     assert rc == alr.ALR_ERR_INVALID_ARG
     assert "Zd_ref" in lib.alr_last_error().decode()
+    rc = lib.alr_loss_from_sums(None, fake, ctypes.c_float(1.0), fake, None)
+    assert rc == alr.ALR_ERR_INVALID_ARG
     # group references: one per 16 logits of a row (the last group may be partial)
     assert [lib.alr_kept_ref_groups(v) for v in (8, 256, 264, 151936)] == [1, 16, 17, 9496]
 

@@ -1,8 +1,9 @@
 """Multi-rank host logic on CPU ranks (gloo, world size 2-4).
 
 - Row sharding (data parallelism over anchors): with Eq. 1 normalised over the global batch,
-  all-reducing sum omega l, sum omega and the per-rank H_d^T G reproduces the unsharded loss
-  and head gradient.
+  the product's collective steps (all-reduce of sum omega l and sum omega, backward with the
+  batch's sum omega, all-reduce of the per-rank H_d^T G and of the histograms) reproduce the
+  unsharded loss, dH, dW and accepted-length histogram.
 - Vocabulary sharding: per-shard partial statistics (running max / sum-exp of both sides,
   label-weighted sums, greedy top-2) merged in rank order give the unsharded log-sum-exps,
   losses, entropies, argmaxes and gaps — the same merge the forward kernel applies across
@@ -62,32 +63,49 @@ def _problem(seed=0, d=12, V=37, A=6, B=4):
 
 
 def _row_shard(rank, world):
+    """One rank of a row-sharded batch: the product's sequence of collective steps
+    (paper_2609_38795_gb300.sharded), with the oracle standing in for the library's compute on
+    this CPU rank (the forward's partial sums, L from the reduced sums, the backward with the
+    batch's sum omega, the accepted lengths)."""
+    from paper_2609_38795_gb300 import sharded
+    lam = 1.013441
     Hd, Ht, W, mask, B = _problem()
     A = Hd.shape[0] // B
     anchors = np.arange(rank, A, world)
     rows = (anchors[:, None] * B + np.arange(B)).reshape(-1)
-    out = orc.slot_loss_forward(Hd[rows], Ht[rows], W, B, lam=1.013441, row_mask=mask[rows])
+    out = orc.slot_loss_forward(Hd[rows], Ht[rows], W, B, lam=lam, row_mask=mask[rows])   # 1
     sums = torch.tensor([(out["weight"] * out["loss_row"]).sum(), out["weight"].sum()],
                         dtype=torch.float64)
-    dist.all_reduce(sums)
-    G = orc.logit_grad(out["z_d"], out["z_t"], out["weight"], 1.013441,
-                       weight_sum=float(sums[1]))
-    _, dW = orc.slot_loss_backward(Hd[rows], W, G)
+    sharded.reduce_sums(sums)                                                             # 2
+    L = lam * float(sums[0]) / float(sums[1])                                             # 3
+    G = orc.logit_grad(out["z_d"], out["z_t"], out["weight"], lam, weight_sum=float(sums[1]))
+    dH, dW = orc.slot_loss_backward(Hd[rows], W, G)                                       # 4
     dW = torch.from_numpy(dW)
-    dist.all_reduce(dW)
-    return float(1.013441 * sums[0] / sums[1]), dW.numpy()
+    sharded.reduce_weight_grad(dW)                                                        # 5
+    _, hist = orc.accept_len(out["argmax_d"], out["argmax_t"], B, active=mask[rows])
+    hist = torch.from_numpy(np.asarray(hist, dtype=np.int64))
+    sharded.reduce_hist(hist)
+    return L, dW.numpy(), rows, dH, hist.numpy()
 
 
-@pytest.mark.parametrize("world", [2, 3])
-def test_row_sharded_loss_and_head_gradient_match_unsharded(world):
+@pytest.mark.parametrize("world", [2, 3, 4])
+def test_row_sharded_loss_and_gradients_match_unsharded(world):
+    """Every rank ends with the batch's L and dW; the ranks' dH rows together are the batch's
+    dH; the reduced histogram counts every anchor of the batch."""
     res = _run(_row_shard, world)
     Hd, Ht, W, mask, B = _problem()
-    full = orc.slot_loss_forward(Hd, Ht, W, B, lam=1.013441, row_mask=mask)
-    G = orc.logit_grad(full["z_d"], full["z_t"], full["weight"], 1.013441)
-    _, dW = orc.slot_loss_backward(Hd, W, G)
-    for L, dW_r in res:
+    lam = 1.013441
+    full = orc.slot_loss_forward(Hd, Ht, W, B, lam=lam, row_mask=mask)
+    G = orc.logit_grad(full["z_d"], full["z_t"], full["weight"], lam)
+    dH, dW = orc.slot_loss_backward(Hd, W, G)
+    _, hist = orc.accept_len(full["argmax_d"], full["argmax_t"], B, active=mask)
+    dH_sharded = np.zeros_like(dH)
+    for L, dW_r, rows, dH_r, hist_r in res:
         np.testing.assert_allclose(L, full["loss_total"], rtol=1e-13)
         np.testing.assert_allclose(dW_r, dW, rtol=1e-11, atol=1e-14)
+        assert np.array_equal(hist_r, hist)
+        dH_sharded[rows] = dH_r
+    np.testing.assert_allclose(dH_sharded, dH, rtol=1e-12, atol=1e-15)
 
 
 def _vocab_shard(rank, world):
