@@ -348,7 +348,8 @@ def ira_blocks(valid_anchors, rollout_len, offsets, K, max_blocks=128, rollout_t
     first ceil(m/2) are primary (they run the target rollout), the next floor(m/2) secondary;
     slots past m are unused.  Secondary block i sits in primary block i's rollout at offset
     j = offsets[s, i] in {2..K-1}.  Primary block p's stored rollout holds rollout_len[s, p]
-    label rows (K, or fewer after early termination).
+    label rows (K, or fewer after early termination); a secondary whose offset lies past them
+    (j > rollout_len) has no anchor token y*_j and stays unused.
 
     Per block (s, b), with P = max_blocks - max_blocks // 2 primary slots per sample, the
     gather of label rows from the primary label buffer viewed as [S * P, K, d]:
@@ -375,7 +376,9 @@ def ira_blocks(valid_anchors, rollout_len, offsets, K, max_blocks=128, rollout_t
                 p, j = b, 0
             else:
                 p, j = b - n_prim, int(offsets[s][b - n_prim])
-                if j < 1 or j > K - 1:
+                # an offset outside the rollout leaves the block unused: past K - 1, or past
+                # the end of a primary rollout that terminated early, y*_j does not exist
+                if j < 1 or j > K - 1 or j > int(rollout_len[s][p]):
                     continue
             seq[s, b] = s * P + p
             pos[s, b] = j
@@ -386,3 +389,66 @@ def ira_blocks(valid_anchors, rollout_len, offsets, K, max_blocks=128, rollout_t
             if j > 0 and rollout_tok is not None:
                 tok[s, b] = int(rollout_tok[s][p][j - 1])      # y*_j is rollout step j
     return dict(seq=seq, pos=pos, valid_len=vlen, ctx_len=ctx, anchor_tok=tok)
+
+
+def ira_draw(anchor_ok, keys, offset_u, K, max_blocks=128):
+    """The random draws of IRA (Sec. 3.2, In-rollout anchors; App. A: 128 anchors per sample,
+    j ~ U{2, ..., K-1}), from uniform random numbers given as inputs.
+
+    Anchors: sample s has v_s valid positions (anchor_ok[s, a] != 0); m_s = min(v_s,
+    max_blocks) of them are drawn uniformly without replacement, as the valid positions in
+    increasing order of their keys (uniform 32-bit integers; equal keys in position order),
+    the first m_s taken, in that order.  Offsets: j = 2 + floor(u (K - 2) / 2^32) for a
+    uniform 32-bit u, one per secondary slot.
+
+    Returns n_valid [S], anchor_pos [S, max_blocks] (-1 past m_s), offsets [S, max_blocks // 2].
+    """
+    anchor_ok = np.asarray(anchor_ok)
+    keys = np.asarray(keys, dtype=np.int64)
+    S, L = anchor_ok.shape
+    n_valid = np.zeros(S, dtype=np.int64)
+    anchor_pos = np.full((S, max_blocks), -1, dtype=np.int64)
+    for s in range(S):
+        valid = [a for a in range(L) if anchor_ok[s, a]]
+        n_valid[s] = len(valid)
+        order = sorted(valid, key=lambda a: (int(keys[s, a]), a))
+        for i, a in enumerate(order[:max_blocks]):
+            anchor_pos[s, i] = a
+    u = np.asarray(offset_u, dtype=np.int64).reshape(S, max_blocks // 2)
+    offsets = 2 + (u * (K - 2)) // (1 << 32)
+    return n_valid, anchor_pos, offsets
+
+
+def ira_context(store, n_valid, rollout_len, offsets, anchor_pos, K, max_blocks=128):
+    """Context of every secondary block (Sec. 3.2: the target representations of the corpus
+    prefix up to the anchor a, then those stored for y*_1..y*_{j-1}; App. A: the rollout
+    stores the outputs of the five target layers the drafter reads for y*_1..y*_13).
+
+    store [S * P, C, F]: primary block p of sample s keeps C rows of F features (the five
+    layers' outputs side by side), row r for rollout token y*_{r+1}.  Secondary i of sample s
+    (i < floor(m_s / 2)) sits in primary i at offset j = offsets[s, i]; when 1 <= j <= K - 1
+    and j <= rollout_len[s, i] it exists, its context takes the j - 1 rows of y*_1..y*_{j-1}
+    and the corpus prefix ends at primary i's anchor anchor_pos[s, i].
+
+    Returns ctx [S, H, C, F] (rows past the context zero), ctx_len [S, H], prefix_end [S, H]
+    (-1 for a secondary slot without a block), with H = max_blocks // 2.
+    """
+    store = np.asarray(store)
+    S = len(n_valid)
+    P, H = max_blocks - max_blocks // 2, max_blocks // 2
+    _, C, F = store.shape
+    assert C >= K - 2, "the store must hold the rows of y*_1..y*_{K-2}"
+    ctx = np.zeros((S, H, C, F), dtype=store.dtype)
+    ctx_len = np.zeros((S, H), dtype=np.int64)
+    prefix_end = np.full((S, H), -1, dtype=np.int64)
+    for s in range(S):
+        m = min(int(n_valid[s]), max_blocks)
+        for i in range(m // 2):
+            j = int(offsets[s][i])
+            if j < 1 or j > K - 1 or j > int(rollout_len[s][i]):
+                continue
+            n = j - 1
+            ctx[s, i, :n] = store[s * P + i, :n]
+            ctx_len[s, i] = n
+            prefix_end[s, i] = int(anchor_pos[s][i])
+    return ctx, ctx_len, prefix_end

@@ -314,6 +314,9 @@ def test_ira_block_split_and_inheritance():
     offsets = rng.integers(2, K, size=(len(valid), P))
     rlen = np.full((len(valid), P), K)
     rlen[3, 1] = 9                                        # an early-terminated rollout
+    offsets[3, 1] = 12                                    # ... whose secondary lies past it
+    rlen[5, 2] = 11                                       # ... and one whose secondary fits
+    offsets[5, 2] = 6
     roll_tok = rng.integers(0, 1000, size=(len(valid), P, K))
     corp_tok = rng.integers(0, 1000, size=(len(valid), max_b))
     out = orc.ira_blocks(valid, rlen, offsets, K, max_b, rollout_tok=roll_tok,
@@ -327,8 +330,12 @@ def test_ira_block_split_and_inheritance():
                 assert out["seq"][s, b] == -1
                 continue
             p = b if kind == "P" else b - (m + 1) // 2
-            assert out["seq"][s, b] == s * P + p
             j = 0 if kind == "P" else offsets[s, p]
+            if j > rlen[s, p]:                            # y*_j was never generated
+                assert out["seq"][s, b] == -1 and out["anchor_tok"][s, b] == -1
+                assert out["ctx_len"][s, b] == 0
+                continue
+            assert out["seq"][s, b] == s * P + p
             assert out["pos"][s, b] == j and out["valid_len"][s, b] == rlen[s, p]
             assert out["ctx_len"][s, b] == max(j - 1, 0)
             assert out["anchor_tok"][s, b] == (corp_tok[s, b] if kind == "P" else roll_tok[s, p, j - 1])
