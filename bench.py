@@ -371,6 +371,77 @@ def gather_bandwidth(device, reps=24, warmup=4, n_sets=4):
             "reps": reps, "timing": "one CUDA graph of reps launches, replayed"}
 
 
+def ira_context_bandwidth(device, reps=24, warmup=4, n_sets=3):
+    """Context rows of the IRA secondary blocks at the paper's shape (App. A: 6 samples per
+    GPU, 128 anchors per sample, K = 15, the five target layers' outputs stored for
+    y*_1..y*_13, d = 4096 bf16): 64 secondaries per sample, each a [13, 5 d] context buffer
+    filled from its primary's store (j - 1 rows copied, the rest zeroed).  The draws come from
+    seeded random integers; the algorithmic bytes are the copied rows read and written plus the
+    zero rows written, from the actual offsets.  Rotating input/output sets larger than L2; a
+    CUDA graph of reps launches replayed, as for the gather."""
+    import numpy as np
+    import torch
+    from paper_2609_38795_gb300 import alr
+    S, L, K, max_b, C, F = 6, 4096, 15, 128, 13, 5 * 4096
+    H, P = max_b // 2, max_b - max_b // 2
+    g = torch.Generator(device=device).manual_seed(11)
+    sets = []
+    for _ in range(n_sets):
+        ok = torch.ones(S, L, dtype=torch.uint8, device=device)
+        keys = torch.randint(-(1 << 31), 1 << 31, (S, L), generator=g, device=device,
+                             dtype=torch.int64).to(torch.int32)
+        off_u = torch.randint(-(1 << 31), 1 << 31, (S, H), generator=g, device=device,
+                              dtype=torch.int64).to(torch.int32)
+        d = dict(n_valid=torch.empty(S, dtype=torch.int32, device=device),
+                 anchor_pos=torch.empty(S, max_b, dtype=torch.int32, device=device),
+                 offsets=torch.empty(S, H, dtype=torch.int32, device=device))
+        alr.alr_ira_draw(K, max_b, ok, keys, off_u, d)
+        store = torch.randn(S * P, C, F, generator=g, device=device).to(torch.bfloat16)
+        rlen = torch.full((S * P,), K, dtype=torch.int32, device=device)
+        ctx = torch.empty(S, H, C, F, dtype=torch.bfloat16, device=device)
+        sets.append((store, d, rlen, ctx))
+
+    def launch(i):
+        store, d, rlen, ctx = sets[i % n_sets]
+        alr.alr_ira_context(K, max_b, store, d["n_valid"], rlen, d["offsets"], d["anchor_pos"], ctx)
+
+    for i in range(warmup):
+        launch(i)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for i in range(reps):
+        launch(i)
+    b.record()
+    torch.cuda.synchronize()
+    ms_stream = a.elapsed_time(b) / reps
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for i in range(reps):
+            launch(i)
+    graph.replay()
+    torch.cuda.synchronize()
+    a.record()
+    graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / reps
+    check_device_status("IRA context")
+    row = F * 2
+    nbytes = []
+    for _, d, _, _ in sets:                         # mean over the rotating sets' offsets
+        copied = int((d["offsets"].cpu().numpy().astype(np.int64) - 1).sum())
+        nbytes.append(2 * copied * row + (S * H * C - copied) * row)
+    nb = sum(nbytes) / len(nbytes)
+    return {"workload": f"{S} samples x {H} secondary blocks, {C} stored rows of 5 x 4096 bf16 "
+                        f"features (K={K}, 128 anchors, length {L})",
+            "bytes": nb, "us_per_launch": ms * 1e3, "GB/s": nb / (ms / 1e3) / 1e9,
+            "us_per_launch_stream": ms_stream * 1e3,
+            "GB/s_stream": nb / (ms_stream / 1e3) / 1e9,
+            "l2": f"inputs larger than L2 ({n_sets} rotating input/output sets)",
+            "reps": reps, "timing": "one CUDA graph of reps launches, replayed"}
+
+
 # ------------------------------------------------------------------------ GPU arm ---
 def make_inputs(wl, sigma, device, seed):
     import torch
@@ -780,6 +851,7 @@ def run_gpu(args, rank, world, local_rank):
     total_ms, e2e_ms = max_over_ranks([total_ms, e2e["ms"] if e2e else 0.0], device)
 
     gather = gather_bandwidth(device) if rank == 0 else None
+    ira_ctx = ira_context_bandwidth(device) if rank == 0 else None
     topk = time_topk(step, K, args.warmup) if (rank == 0 and not args.no_topk) else None
     other = (time_variant(wl, x, device, K, args.warmup, keep=not keep)
              if (rank == 0 and not args.no_recompute) else None)
@@ -860,6 +932,7 @@ def run_gpu(args, rank, world, local_rank):
         ("recompute" if keep else "keep"): other,
         "gpu_launches": Step.KERNELS_PER_STEP * K,
         "ira_gather": dict(gather, frac_of_hbm=gather["GB/s"] / pk["hbm"], hbm_peak_gbs=pk["hbm"]),
+        "ira_context": dict(ira_ctx, frac_of_hbm=ira_ctx["GB/s"] / pk["hbm"]),
         "compact_labels": topk,
         "loss": loss, "acc_hist": acc_hist, "acc_hist_by_sigma": hist_sigma,
         # mean accepted length per anchor + 1: the tokens a verification round yields (MAT)
@@ -955,9 +1028,12 @@ def main():
         alr.lib()
         if rank == 0:
             g = gather_bandwidth(f"cuda:{local_rank}")
+            c = ira_context_bandwidth(f"cuda:{local_rank}")
             pk = peaks()
             print(json.dumps({"ira_gather": dict(g, frac_of_hbm=g["GB/s"] / pk["hbm"],
-                                                  hbm_peak_gbs=pk["hbm"])}), flush=True)
+                                                  hbm_peak_gbs=pk["hbm"]),
+                              "ira_context": dict(c, frac_of_hbm=c["GB/s"] / pk["hbm"])}),
+                  flush=True)
         return
     if world > 1:
         import torch

@@ -143,7 +143,8 @@ int alr_gather_ira_blocks(const void* feat, int32_t S, int32_t L, int32_t d, int
  * j = offsets[s * (max_blocks/2) + i] (the method draws j ~ U{2..K-1}; the caller passes the
  * draws; j outside [1, K-1] leaves the block unused).  Primary block p of sample s owns rows
  * [s*P + p] of a label buffer [S*P, K, ...] with P = max_blocks - max_blocks/2, of which
- * rollout_len[s*P + p] are valid (K, fewer after early termination).
+ * rollout_len[s*P + p] are valid (K, fewer after early termination); a secondary block whose
+ * offset lies past them (j > rollout_len: y*_j was never generated) is unused.
  * Outputs per block slot t = s*max_blocks + b (int32 [S*max_blocks]):
  *   seq, pos, valid_len - the alr_gather_ira_blocks arguments that read the block's K label
  *             rows from that buffer: a secondary block's row k reads primary row j + k - 1 and
@@ -156,6 +157,49 @@ int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* vali
                    const int32_t* rollout_len, const int32_t* offsets, const int32_t* rollout_tok,
                    const int32_t* corpus_anchor_tok, int32_t* seq, int32_t* pos,
                    int32_t* valid_len, int32_t* ctx_len, int32_t* anchor_tok, void* stream);
+
+/*
+ * IRA draws (Sec. 3.2, In-rollout anchors: m = min(v, max_blocks) blocks from the v valid
+ * anchor positions of a sample, secondary offsets j ~ U{2, ..., K-1}; App. A: 128 anchors per
+ * sample, j in {2..14}).  The random numbers are inputs, so that a run is reproducible from
+ * the caller's generator:
+ *   anchor_ok [S, L] uint8: nonzero where position a of sample s may anchor a block.
+ *   keys      [S, L] uint32: independent uniform random integers, one per position.  The draw
+ *             (uniform, without replacement) is the valid positions in increasing order of
+ *             their keys, equal keys in position order, the first m taken.
+ *   offset_u  [S, max_blocks/2] uint32 uniform: j = 2 + floor(u * (K - 2) / 2^32).
+ * Outputs: n_valid [S] (v); anchor_pos [S, max_blocks] the drawn positions in draw order, -1
+ * past m (the first ceil(m/2) anchor the primary blocks, see alr_ira_blocks); offsets
+ * [S, max_blocks/2] (j, the offsets argument of alr_ira_blocks and alr_ira_context).
+ * Requires 1 <= L <= ALR_IRA_MAX_LEN (L * 8 bytes of shared memory per sample) and K >= 3.
+ */
+#define ALR_IRA_MAX_LEN 16384
+int alr_ira_draw(int32_t S, int32_t L, int32_t K, int32_t max_blocks, const uint8_t* anchor_ok,
+                 const uint32_t* keys, const uint32_t* offset_u, int32_t* n_valid,
+                 int32_t* anchor_pos, int32_t* offsets, void* stream);
+
+/*
+ * Context of the IRA secondary blocks (Sec. 3.2: the target representations of the corpus
+ * prefix up to the anchor a, concatenated with those stored for y*_1..y*_{j-1}; App. A: the
+ * rollout stores the outputs of the five target layers the drafter reads for y*_1..y*_13).
+ *   store [S*P, C, F] (dtype), P = max_blocks - max_blocks/2: primary block p of sample s
+ *         keeps C >= K-2 rows of F features (e.g. the five layers' d-vectors side by side,
+ *         F = 5 d), row r for rollout token y*_{r+1}.
+ *   n_valid [S], offsets [S, max_blocks/2], anchor_pos [S, max_blocks]: from alr_ira_draw;
+ *   rollout_len [S*P]: label rows of each primary rollout (K, fewer after early termination).
+ * Secondary i of sample s (i < floor(m/2)) sits in primary i at offset j; it exists when
+ * 1 <= j <= K-1 and j <= rollout_len (as in alr_ira_blocks).  Outputs:
+ *   ctx [S, max_blocks/2, C, F]: rows r < j-1 are store[s*P + i, r] (y*_1..y*_{j-1}), the
+ *       other rows, and every row of a slot without a block, are zero;
+ *   ctx_len [S, max_blocks/2] (nullable): j - 1, or 0;
+ *   prefix_end [S, max_blocks/2] (nullable): the corpus position a whose prefix x_0..x_a the
+ *       context starts with (primary i's anchor), -1 without a block.
+ * Requires F * elemsize % 16 == 0, 16-byte aligned store and ctx.
+ */
+int alr_ira_context(const void* store, int32_t C, int32_t F, int32_t dtype, int32_t S, int32_t K,
+                    int32_t max_blocks, const int32_t* n_valid, const int32_t* rollout_len,
+                    const int32_t* offsets, const int32_t* anchor_pos, void* ctx,
+                    int32_t* ctx_len, int32_t* prefix_end, void* stream);
 
 /* Workspace bytes alr_slot_loss_fwd needs for `p` (0 on invalid params). */
 size_t alr_fwd_workspace_size(const alr_params* p);

@@ -100,6 +100,10 @@ SIGNATURES = {
     "alr_ira_blocks": (_c_int, [_c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
                                 _c_p, _c_p, _c_p, _c_p]),
     "alr_loss_from_sums": (_c_int, [_c_p, _c_p, _c_f, _c_p, _c_p]),
+    "alr_ira_draw": (_c_int, [_c_i32, _c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p, _c_p, _c_p, _c_p,
+                              _c_p]),
+    "alr_ira_context": (_c_int, [_c_p, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _c_p, _c_p,
+                                 _c_p, _c_p, _c_p, _c_p, _c_p, _c_p]),
     "alr_accept_len": (_c_int, [_c_p, _c_p, _c_p, _c_i32, _c_i32, _c_p, _c_p, _c_p]),
     "alr_erase_weights": (_c_int, [_c_p, _c_p, _c_p, _c_p, _c_i32, _c_i32, _c_f, _c_i32, _c_p,
                                    _c_p]),
@@ -514,6 +518,37 @@ def alr_loss_from_sums(wl_sum, weight_sum, lam, loss_total, stream=None):
     _check(lib().alr_loss_from_sums(_ptr(wl_sum, "wl_sum", 1, _F32),
                                     _ptr(weight_sum, "weight_sum", 1, _F32), float(lam),
                                     _ptr(loss_total, "loss_total", 1, _F32), _stream(stream)))
+
+
+def alr_ira_draw(K, max_blocks, anchor_ok, keys, offset_u, out: dict, stream=None):
+    """anchor_ok [S, L] uint8, keys [S, L] and offset_u [S, max_blocks // 2] random integers
+    (int32 tensors holding the uint32 bits); out: n_valid [S], anchor_pos [S, max_blocks],
+    offsets [S, max_blocks // 2] (int32)."""
+    S, L = anchor_ok.shape
+    H = max_blocks // 2
+    _check(lib().alr_ira_draw(S, L, K, max_blocks, _ptr(anchor_ok, "anchor_ok", S * L, torch.uint8),
+                              _ptr(keys, "keys", S * L, _I32),
+                              _ptr(offset_u, "offset_u", S * H, _I32),
+                              _ptr(out["n_valid"], "n_valid", S, _I32),
+                              _ptr(out["anchor_pos"], "anchor_pos", S * max_blocks, _I32),
+                              _ptr(out["offsets"], "offsets", S * H, _I32), _stream(stream)))
+
+
+def alr_ira_context(K, max_blocks, store, n_valid, rollout_len, offsets, anchor_pos, ctx,
+                    ctx_len=None, prefix_end=None, stream=None):
+    """store [S * P, C, F]; ctx [S, max_blocks // 2, C, F] (same dtype)."""
+    SP, C, F = store.shape
+    H, P = max_blocks // 2, max_blocks - max_blocks // 2
+    S = SP // P
+    dt = store.dtype
+    _check(lib().alr_ira_context(_ptr(store, "store", SP * C * F, dt), C, F, dtype_code(dt), S, K,
+                                 max_blocks, _ptr(n_valid, "n_valid", S, _I32),
+                                 _ptr(rollout_len, "rollout_len", S * P, _I32),
+                                 _ptr(offsets, "offsets", S * H, _I32),
+                                 _ptr(anchor_pos, "anchor_pos", S * max_blocks, _I32),
+                                 _ptr(ctx, "ctx", S * H * C * F, dt),
+                                 _ptr(ctx_len, "ctx_len", S * H, _I32),
+                                 _ptr(prefix_end, "prefix_end", S * H, _I32), _stream(stream)))
 
 
 def _anchors(t, B, name):

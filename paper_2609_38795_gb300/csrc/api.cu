@@ -1056,6 +1056,56 @@ int alr_ira_blocks(int32_t S, int32_t K, int32_t max_blocks, const int32_t* vali
   return ALR_OK;
 }
 
+int alr_ira_draw(int32_t S, int32_t L, int32_t K, int32_t max_blocks, const uint8_t* anchor_ok,
+                 const uint32_t* keys, const uint32_t* offset_u, int32_t* n_valid,
+                 int32_t* anchor_pos, int32_t* offsets, void* stream) {
+  ALR_RANGE();
+  if (S < 0 || L < 1 || L > ALR_IRA_MAX_LEN || K < 3 || max_blocks < 1)
+    return fail(ALR_ERR_INVALID_ARG, "bad sizes S=%d L=%d (at most %d) K=%d max_blocks=%d", S, L,
+                ALR_IRA_MAX_LEN, K, max_blocks);
+  if (S == 0) return ALR_OK;
+  if (anchor_ok == nullptr || keys == nullptr || n_valid == nullptr || anchor_pos == nullptr ||
+      (max_blocks > 1 && (offset_u == nullptr || offsets == nullptr)))
+    return fail(ALR_ERR_INVALID_ARG,
+                "anchor_ok, keys, offset_u, n_valid, anchor_pos and offsets must be non-NULL");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  cudaError_t e = alr::launch_ira_draw(S, L, K, max_blocks, anchor_ok, keys, offset_u, n_valid,
+                                       anchor_pos, offsets, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "IRA draw launch");
+  return ALR_OK;
+}
+
+int alr_ira_context(const void* store, int32_t C, int32_t F, int32_t dtype, int32_t S, int32_t K,
+                    int32_t max_blocks, const int32_t* n_valid, const int32_t* rollout_len,
+                    const int32_t* offsets, const int32_t* anchor_pos, void* ctx,
+                    int32_t* ctx_len, int32_t* prefix_end, void* stream) {
+  ALR_RANGE();
+  if (dtype != ALR_BF16 && dtype != ALR_F32) return fail(ALR_ERR_UNSUPPORTED, "dtype %d", dtype);
+  if (S < 0 || K < 3 || max_blocks < 2 || C < K - 2 || F < 1)
+    return fail(ALR_ERR_INVALID_ARG,
+                "bad sizes S=%d K=%d max_blocks=%d C=%d (at least K-2) F=%d", S, K, max_blocks, C,
+                F);
+  if ((size_t(F) * elem_size(dtype)) % 16 != 0)
+    return fail(ALR_ERR_INVALID_ARG, "F * element size must be a multiple of 16 bytes");
+  if (S == 0) return ALR_OK;
+  if (store == nullptr || n_valid == nullptr || rollout_len == nullptr || offsets == nullptr ||
+      anchor_pos == nullptr || ctx == nullptr)
+    return fail(ALR_ERR_INVALID_ARG,
+                "store, n_valid, rollout_len, offsets, anchor_pos and ctx must be non-NULL");
+  if (!aligned16(store) || !aligned16(ctx))
+    return fail(ALR_ERR_INVALID_ARG, "store and ctx must be 16-byte aligned");
+  DevInfo info;
+  int rc = require_sm103(&info);
+  if (rc != ALR_OK) return rc;
+  cudaError_t e = alr::launch_ira_context(store, C, F, int(elem_size(dtype)), S, K, max_blocks,
+                                          n_valid, rollout_len, offsets, anchor_pos, ctx, ctx_len,
+                                          prefix_end, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "IRA context launch");
+  return ALR_OK;
+}
+
 int alr_accept_len(const int32_t* argmax_d, const int32_t* argmax_t, const float* active,
                    int32_t A, int32_t B, int32_t* acc_len, int64_t* hist, void* stream) {
   ALR_RANGE();

@@ -196,6 +196,18 @@ cudaError_t launch_ira_blocks(int S, int K, int max_blocks, const int32_t* valid
                               int32_t* seq, int32_t* pos, int32_t* vlen, int32_t* ctx_len,
                               int32_t* anchor_tok, cudaStream_t s);
 
+// IRA draws (one block per sample, L * 8 bytes of shared memory): n_valid [S], anchor_pos
+// [S, max_blocks] (draw order, -1 past m), offsets [S, max_blocks / 2].
+cudaError_t launch_ira_draw(int S, int L, int K, int max_blocks, const uint8_t* anchor_ok,
+                            const uint32_t* keys, const uint32_t* offset_u, int32_t* n_valid,
+                            int32_t* anchor_pos, int32_t* offsets, cudaStream_t s);
+// Context rows of the secondary blocks: ctx [S, max_blocks / 2, C, F] from the primaries'
+// stored rollout features [S * P, C, F]; ctx_len, prefix_end [S, max_blocks / 2] (nullable).
+cudaError_t launch_ira_context(const void* store, int C, int F, int elem_bytes, int S, int K,
+                               int max_blocks, const int32_t* n_valid, const int32_t* rollout_len,
+                               const int32_t* offsets, const int32_t* anchor_pos, void* ctx,
+                               int32_t* ctx_len, int32_t* prefix_end, cudaStream_t s);
+
 // out[c, r] = in[r, c] for an fp32 [R, C] matrix; out rows are ld_out elements apart.
 cudaError_t launch_transpose32(const float* in, float* out, int R, int C, int ld_out,
                                cudaStream_t s);

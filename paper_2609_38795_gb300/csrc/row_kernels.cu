@@ -455,7 +455,9 @@ __global__ void __launch_bounds__(256) ira_blocks_kernel(
   } else if (b < m) {
     p = b - n_prim;
     j = offsets[size_t(s) * Q + p];
-    if (j < 1 || j > K - 1) p = -1;   // an offset outside the rollout leaves the block unused
+    // an offset outside the rollout leaves the block unused: past K - 1, or past the end of
+    // a primary rollout that terminated early (y*_j, the block's anchor token, never existed)
+    if (j < 1 || j > K - 1 || j > rollout_len[size_t(s) * P + p]) p = -1;
   }
   if (p < 0) {
     seq[t] = -1;
@@ -475,6 +477,99 @@ __global__ void __launch_bounds__(256) ira_blocks_kernel(
     if (j == 0 && corpus_anchor_tok) tok = corpus_anchor_tok[t];
     if (j > 0 && rollout_tok) tok = rollout_tok[prim * K + (j - 1)];   // y*_j
     anchor_tok[t] = tok;
+  }
+}
+
+// ------------------------------------------------------------------ IRA draws ---
+// One block per sample.  The anchor draw is the sample's valid positions in increasing
+// (key, position) order; each valid position's rank in that order is the number of smaller
+// (key, position) pairs, counted over the sample's pairs held in shared memory (invalid
+// positions hold the largest value and are never counted or drawn).  Ranks below m =
+// min(v, max_blocks) are the draw.  Offsets: j = 2 + floor(u (K - 2) / 2^32).
+__global__ void __launch_bounds__(1024) ira_draw_kernel(int L, int K, int max_blocks,
+                                                        const uint8_t* __restrict__ anchor_ok,
+                                                        const uint32_t* __restrict__ keys,
+                                                        const uint32_t* __restrict__ offset_u,
+                                                        int32_t* __restrict__ n_valid,
+                                                        int32_t* __restrict__ anchor_pos,
+                                                        int32_t* __restrict__ offsets) {
+  extern __shared__ unsigned long long pair[];   // [L] (key << 32 | position), or ~0
+  __shared__ int s_count;
+  const int s = blockIdx.x;
+  const size_t row = size_t(s) * size_t(L);
+  if (threadIdx.x == 0) s_count = 0;
+  __syncthreads();
+  int mine = 0;
+  for (int a = threadIdx.x; a < L; a += blockDim.x) {
+    const bool ok = anchor_ok[row + a] != 0;
+    pair[a] = ok ? ((static_cast<unsigned long long>(keys[row + a]) << 32) | unsigned(a))
+                 : ~0ull;
+    mine += ok ? 1 : 0;
+  }
+  atomicAdd(&s_count, mine);
+  __syncthreads();
+  const int v = s_count, m = min(v, max_blocks);
+  int32_t* out = anchor_pos + size_t(s) * size_t(max_blocks);
+  for (int i = m + threadIdx.x; i < max_blocks; i += blockDim.x) out[i] = -1;
+  for (int a = threadIdx.x; a < L; a += blockDim.x) {
+    const unsigned long long c = pair[a];
+    if (c == ~0ull) continue;
+    int rank = 0;
+    for (int q = 0; q < L; ++q) rank += pair[q] < c ? 1 : 0;
+    if (rank < m) out[rank] = a;
+  }
+  const int H = max_blocks / 2;
+  for (int i = threadIdx.x; i < H; i += blockDim.x) {
+    const unsigned long long u = offset_u[size_t(s) * H + i];
+    offsets[size_t(s) * H + i] = 2 + int((u * unsigned(K - 2)) >> 32);
+  }
+  if (threadIdx.x == 0) n_valid[s] = v;
+}
+
+// ------------------------------------------------------------------ IRA context ---
+// Context rows of the secondary blocks: output row (s, i, r) of [S, H, C, F] is row r of
+// primary i's stored rollout features when secondary i of sample s exists and r < j - 1,
+// zero otherwise.  One warp per output row, 16-byte vectors in batches as in the gather.
+__global__ void __launch_bounds__(256) ira_context_kernel(
+    const uint4* __restrict__ store, int C, int vec_per_row, int S, int K, int max_blocks,
+    const int32_t* __restrict__ n_valid, const int32_t* __restrict__ rollout_len,
+    const int32_t* __restrict__ offsets, const int32_t* __restrict__ anchor_pos,
+    uint4* __restrict__ ctx, int32_t* __restrict__ ctx_len, int32_t* __restrict__ prefix_end) {
+  const int H = max_blocks / 2, P = max_blocks - H;
+  const long long t = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (t >= (long long)S * H * C) return;
+  const int r = int(t % C);
+  const long long si = t / C;
+  const int s = int(si / H), i = int(si - (long long)s * H);
+  const int m = max(0, min(n_valid[s], max_blocks));
+  const int j = offsets[si];
+  const size_t prim = size_t(s) * P + i;
+  const bool exists = i < m / 2 && j >= 1 && j <= K - 1 && j <= rollout_len[prim];
+  const int n = exists ? j - 1 : 0;
+  if (r == 0 && lane == 0) {
+    if (ctx_len) ctx_len[si] = n;
+    if (prefix_end) prefix_end[si] = exists ? anchor_pos[size_t(s) * max_blocks + i] : -1;
+  }
+  uint4* dst = ctx + t * vec_per_row;
+  if (r >= n) {
+    const uint4 z = make_uint4(0, 0, 0, 0);
+    for (int k = lane; k < vec_per_row; k += 32) __stcs(dst + k, z);
+    return;
+  }
+  const uint4* src = store + ((long long)prim * C + r) * vec_per_row;
+  for (int base = 0; base < vec_per_row; base += 32 * kGatherBatch) {
+    uint4 v[kGatherBatch];
+#pragma unroll
+    for (int k = 0; k < kGatherBatch; ++k) {
+      const int e = base + k * 32 + lane;
+      if (e < vec_per_row) v[k] = __ldg(src + e);
+    }
+#pragma unroll
+    for (int k = 0; k < kGatherBatch; ++k) {
+      const int e = base + k * 32 + lane;
+      if (e < vec_per_row) __stcs(dst + e, v[k]);
+    }
   }
 }
 
@@ -764,6 +859,30 @@ cudaError_t launch_ira_blocks(int S, int K, int max_blocks, const int32_t* valid
   ira_blocks_kernel<<<unsigned((n + 255) / 256), 256, 0, s>>>(
       S, K, max_blocks, valid_anchors, rollout_len, offsets, rollout_tok, corpus_anchor_tok, seq,
       pos, vlen, ctx_len, anchor_tok);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ira_draw(int S, int L, int K, int max_blocks, const uint8_t* anchor_ok,
+                            const uint32_t* keys, const uint32_t* offset_u, int32_t* n_valid,
+                            int32_t* anchor_pos, int32_t* offsets, cudaStream_t s) {
+  const size_t smem = size_t(L) * sizeof(unsigned long long);
+  cudaError_t e = cudaFuncSetAttribute(ira_draw_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       int(smem));
+  if (e != cudaSuccess) return e;
+  ira_draw_kernel<<<S, 1024, smem, s>>>(L, K, max_blocks, anchor_ok, keys, offset_u, n_valid,
+                                        anchor_pos, offsets);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ira_context(const void* store, int C, int F, int elem_bytes, int S, int K,
+                               int max_blocks, const int32_t* n_valid, const int32_t* rollout_len,
+                               const int32_t* offsets, const int32_t* anchor_pos, void* ctx,
+                               int32_t* ctx_len, int32_t* prefix_end, cudaStream_t s) {
+  const long long rows = (long long)S * (max_blocks / 2) * C;
+  const int vec = int((long long)F * elem_bytes / 16);
+  ira_context_kernel<<<unsigned((rows + 7) / 8), 256, 0, s>>>(
+      static_cast<const uint4*>(store), C, vec, S, K, max_blocks, n_valid, rollout_len, offsets,
+      anchor_pos, static_cast<uint4*>(ctx), ctx_len, prefix_end);
   return cudaGetLastError();
 }
 
