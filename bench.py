@@ -903,6 +903,7 @@ def run_gpu(args, rank, world, local_rank):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{WORKLOAD}{' PROFILING SUBSET' if args.anchors else ''}: d={wl.d} V={wl.V} B={wl.B} A={wl.A} rows={wl.N} "
                                f"sigma={args.sigma} feature buffer {wl.S}x{wl.L}",
+                   "kernel_forms": dict(zip(("gemm", "loss"), alr.alr_kernel_forms())),
                    "global_batch_rows": world * wl.N, "l2": "inputs larger than L2 "
                    "(W 1.24 GB, H 268 MB each, kept logits 2 x 10 GB)", "parallelism": f"replicas{world}"},
         "tensor_tflops": {"executed": exec_tf, "algorithmic_8NdV": algo_tf,

@@ -31,6 +31,9 @@
  *              multicast) | single | mcast4 | pair (CTA pairs with M = 256 tcgen05 products)
  *              selects the bf16 GEMM kernel; ALR_LOSS_FORM = single (default) | mcast selects
  *              the fused loss kernels' form.  fp32 (tf32) products always run on single CTAs.
+ *              A process launched as one rank of several (environment WORLD_SIZE > 1) never
+ *              uses the multicast forms: mcast and mcast4 run as single there, so TMA multicast
+ *              loads stay in single-GPU runs.  alr_kernel_forms() reports the choice.
  */
 #ifndef ALR_H
 #define ALR_H
@@ -103,6 +106,14 @@ int alr_device_supported(void);
  * clear != 0 resets the word to ALR_OK.
  */
 int alr_device_status(void* stream, int clear);
+
+/*
+ * The kernel forms the next bf16 call will use in this process (no device needed):
+ *   *gemm: 0 single CTAs, 1 clusters of two sharing B tiles by TMA multicast, 2 CTA pairs
+ *          (cta_group::2), 3 clusters of four with multicast;
+ *   *loss: 0 single CTAs, 1 clusters of two sharing head tiles by TMA multicast.
+ */
+int alr_kernel_forms(int32_t* gemm, int32_t* loss);
 
 /*
  * Test hook for the failure-detection path (the paper has no counterpart).  With enable != 0,

@@ -54,6 +54,7 @@ SIGNATURES = {
     "alr_last_error": (ctypes.c_char_p, []),
     "alr_device_supported": (_c_int, []),
     "alr_device_status": (_c_int, [_c_p, _c_int]),
+    "alr_kernel_forms": (_c_int, [_c_p, _c_p]),
     "alr_debug_withhold_next_stage": (_c_int, [_c_int]),
     "alr_gather_ira_blocks": (_c_int, [_c_p, _c_i32, _c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p,
                                        _c_i32, _c_i32, _c_p, _c_p, _c_p]),
@@ -226,6 +227,17 @@ def alr_device_supported() -> int:
 
 def alr_device_status(clear=True, stream=None) -> int:
     return lib().alr_device_status(_stream(stream), int(clear))
+
+
+GEMM_FORMS = ("single", "mcast", "pair", "mcast4")
+LOSS_FORMS = ("single", "mcast")
+
+
+def alr_kernel_forms():
+    """(GEMM form, loss-kernel form) names the next bf16 call will use in this process."""
+    g, l = ctypes.c_int32(), ctypes.c_int32()
+    _check(lib().alr_kernel_forms(ctypes.byref(g), ctypes.byref(l)))
+    return GEMM_FORMS[g.value], LOSS_FORMS[l.value]
 
 
 def alr_debug_withhold_next_stage(enable=True) -> int:

@@ -169,13 +169,22 @@ int check_kept(const alr_params* p, const void* Z, const void* ref, const char* 
 #define ALR_LOSS_BN 256
 #endif
 
+// True in a process launched as one rank of several (WORLD_SIZE > 1, as torchrun and
+// torch.distributed set it): such a process uses no kernel form with TMA multicast loads, so
+// that multicast reads of device memory stay in single-GPU runs.
+bool multi_rank_process() {
+  const char* w = getenv("WORLD_SIZE");
+  return w != nullptr && atoi(w) > 1;
+}
+
 // The fused loss kernels run on single CTAs unless the environment variable ALR_LOSS_FORM is
-// "mcast" (bf16 inputs): clusters of two CTAs sharing every head tile by TMA multicast.  The
+// "mcast" (bf16 inputs, single-GPU runs): clusters of two CTAs sharing every head tile by TMA
+// multicast.  The
 // dual-product modes already share each head tile between z_d and z_t, and at the power cap
 // the multicast form settles ~4 % lower in clock for ~1 % fewer L2 bytes per product: it is
 // not faster, so it is not the default.  Both forms give bit-identical results.
 bool loss_multicast(const alr_params* p) {
-  if (p->dtype != ALR_BF16 || ALR_LOSS_BN != 256) return false;
+  if (p->dtype != ALR_BF16 || ALR_LOSS_BN != 256 || multi_rank_process()) return false;
   const char* v = getenv("ALR_LOSS_FORM");
   return v != nullptr && strcmp(v, "mcast") == 0;
 }
@@ -277,15 +286,16 @@ BwdLayout bwd_layout(const alr_params* p, bool with_g = true) {
 // same clock and power.  The pair form issues more products per clock but draws more power
 // per product and settles at a clock ~20 % lower.  tf32 products always run on single CTAs.
 //   "mcast4"  as "mcast" with clusters of four CTAs, each loading a quarter of the B tile.
+// One rank of a multi-rank launch never takes the multicast forms: "mcast", "mcast4" and the
+// default run as "single" there.
 enum GemmForm { kGemmSingle = 0, kGemmMcast = 1, kGemmPair = 2, kGemmMcast4 = 3 };
 
 GemmForm gemm_form(int dtype) {
   if (dtype != ALR_BF16) return kGemmSingle;
   const char* v = getenv("ALR_GEMM_FORM");
-  if (v == nullptr) return kGemmMcast;
-  if (strcmp(v, "single") == 0) return kGemmSingle;
-  if (strcmp(v, "pair") == 0) return kGemmPair;
-  if (strcmp(v, "mcast4") == 0) return kGemmMcast4;
+  if (v != nullptr && strcmp(v, "pair") == 0) return kGemmPair;
+  if (multi_rank_process() || (v != nullptr && strcmp(v, "single") == 0)) return kGemmSingle;
+  if (v != nullptr && strcmp(v, "mcast4") == 0) return kGemmMcast4;
   return kGemmMcast;
 }
 
@@ -463,6 +473,15 @@ int set_last_error(int code, const char* msg) { return fail(code, "%s", msg); }
 extern "C" {
 
 const char* alr_version(void) { return "libalr 0.1 (sm_103a)"; }
+
+int alr_kernel_forms(int32_t* gemm, int32_t* loss) {
+  if (gemm == nullptr || loss == nullptr) return fail(ALR_ERR_INVALID_ARG, "gemm and loss must be non-NULL");
+  alr_params p{};
+  p.dtype = ALR_BF16;
+  *gemm = int32_t(gemm_form(ALR_BF16));
+  *loss = loss_multicast(&p) ? 1 : 0;
+  return ALR_OK;
+}
 
 int alr_debug_withhold_next_stage(int enable) {
   g_withhold_next.store(enable ? 1 : 0);

@@ -204,3 +204,21 @@ def test_error_paths_reject_before_any_device_work(libalr):
         msg = lib.alr_last_error().decode()
         assert rc == code, (name, rc, msg)
         assert text in msg, (name, msg)
+
+
+def test_multi_rank_processes_use_no_multicast_forms(libalr, monkeypatch):
+    """One rank of a multi-rank launch (WORLD_SIZE > 1) never takes a kernel form with TMA
+    multicast loads, whatever the environment asks; a single process keeps its choice."""
+    for world, gemm_env, loss_env, want in (
+            (None, None, None, ("mcast", "single")),
+            ("1", "mcast4", "mcast", ("mcast4", "mcast")),
+            ("2", None, None, ("single", "single")),
+            ("8", "mcast", "mcast", ("single", "single")),
+            ("4", "mcast4", None, ("single", "single")),
+            ("2", "pair", None, ("pair", "single"))):
+        for k, v in (("WORLD_SIZE", world), ("ALR_GEMM_FORM", gemm_env), ("ALR_LOSS_FORM", loss_env)):
+            if v is None:
+                monkeypatch.delenv(k, raising=False)
+            else:
+                monkeypatch.setenv(k, v)
+        assert alr.alr_kernel_forms() == want, (world, gemm_env, loss_env)
