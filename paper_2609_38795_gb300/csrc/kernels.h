@@ -31,10 +31,9 @@ struct LossPlan {
 // epilogue thread (structure of arrays, field-major: part[f * n_parts * N + part * N + row]).
 enum PartField {
   kPMd = 0,   // running max of z_d
-  kPSd,       // sum exp(z_d - m_d) over the part's columns other than its leader (whose
-              // own term is the exact 1 left out)
+  kPSd,       // sum exp(z_d - m_d)
   kPMt,       // running max of z_t
-  kPSt,       // same for z_t
+  kPSt,       // sum exp(z_t - m_t)
   kPU,        // sum exp(z_t - m_t) * (z_d - m_d)
   kPW,        // sum exp(z_t - m_t) * (z_t - m_t)
   kPBd,       // best z_d
@@ -44,6 +43,8 @@ enum PartField {
   kPIt,
   kPSect,
   kPZx,       // z_t at the corpus token if it lies in the split, else NaN
+  kPSdLo,     // rounding error of kPSd (the sum is kPSd + kPSdLo)
+  kPStLo,     // rounding error of kPSt
   kPFields
 };
 

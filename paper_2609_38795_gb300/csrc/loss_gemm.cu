@@ -217,34 +217,36 @@ ALR_DEV void topk_insert(float (&t)[kTopK], int (&ti)[kTopK], float v, int i) {
 }
 
 // Running statistics of one row over the columns one thread sees (full-vocabulary forward).
-// best_x is both the greedy top-1 (the leader) and the online-softmax reference of side x.
-// r_x sums exp(z_x - best_x) over the columns other than the leader, whose own term is the
-// exact 1 (the whole sum is 1 + r_x): once the row's maximum is in, a plain running sum sits at
-// 1 + small and every added term would lose up to half a unit of 1, while r_x keeps the small
-// part, which is what a near-zero loss or entropy is made of, at full relative precision.
+// best_x is both the greedy top-1 and the online-softmax reference of side x; s_x sums
+// exp(z_x - best_x), with the rounding error of its additions kept in c_x: once the row's
+// maximum is in, the sum sits at 1 + small and each added term would otherwise lose up to half
+// a unit of 1, while the small part is what a near-zero loss or entropy is made of.
 // u and w sum exp(z_t - best_t) * (z_d - best_d) and * (z_t - best_t): measured from the
 // running maxima, the terms that carry weight are near zero, so these sums stay small and
-// precise when the logits are large, and the soft CE comes out as log(1 + r_d) - u / (1 + r_t),
-// a sum of two non-negative terms, instead of a difference of two numbers of the logits' size.
+// precise when the logits are large, and the soft CE comes out as log s_d - u / s_t, a sum of
+// two non-negative terms, instead of a difference of two numbers of the logits' size.
 struct RowStats {
-  float best_d, sec_d, r_d, best_t, sec_t, r_t, u, w, zx;
+  float best_d, sec_d, s_d, c_d, best_t, sec_t, s_t, c_t, u, w, zx;
   int i_d, i_t;
 };
 
 ALR_DEV void stats_init(RowStats& st) {
   st.best_d = st.sec_d = st.best_t = st.sec_t = -INFINITY;
-  st.r_d = st.r_t = st.u = st.w = 0.f;
+  st.s_d = st.s_t = st.c_d = st.c_t = st.u = st.w = 0.f;
   st.i_d = st.i_t = 0x7fffffff;
   st.zx = qnan();
 }
 
-// Sum of 2^(z_j log2 e + b) over the sub-chunk's columns other than jj (masked columns are -inf
-// and add 0): the rest-sum of a sub-chunk that brings a new leader at jj.
-ALR_DEV float sum_except(const float (&z)[16], float b, int jj) {
-  float e = 0.f;
-#pragma unroll
-  for (int j = 0; j < kSub; ++j) e += (j == jj) ? 0.f : ex2(fmaf(z[j], kLog2e, b));
-  return e;
+// (s, c) <- (s, c) * sc + x with the rounding error of the addition moved into c (Knuth's
+// TwoSum, branch-free: s + c holds the sum to about twice fp32 precision).  The error of the
+// product s * sc (sc < 1 only when the running maximum moves) is not kept.
+ALR_DEV void sum2_scaled(float& s, float& c, float sc, float x) {
+  const float t = s * sc;
+  const float y = t + x;
+  const float xb = y - t;
+  const float e = (t - (y - xb)) + (x - xb);
+  s = y;
+  c = fmaf(c, sc, e);
 }
 
 // Fold one 16-column sub-chunk (nv valid columns) into the full-vocabulary statistics.
@@ -295,33 +297,18 @@ ALR_DEV void stats_sub(RowStats& st, const uint32_t (&rd)[16], const uint32_t (&
   }
   // u, w: move to the new references (skipped while nothing has been summed: the old
   // reference is still -inf), rescale, add this sub-chunk
-  const bool any = st.best_t > -INFINITY;
-  const float u_sh = any ? fmaf(st.best_d - nbd, 1.f + st.r_t, st.u) : 0.f;
-  const float w_sh = any ? fmaf(st.best_t - nbt, 1.f + st.r_t, st.w) : 0.f;
+  const bool any = st.s_t > 0.f;
+  const float u_sh = any ? fmaf(st.best_d - nbd, st.s_t + st.c_t, st.u) : 0.f;
+  const float w_sh = any ? fmaf(st.best_t - nbt, st.s_t + st.c_t, st.w) : 0.f;
   const float sct = ex2((st.best_t - nbt) * kLog2e);
+  const float scd = ex2((st.best_d - nbd) * kLog2e);
   st.u = fmaf(u_sh, sct, (u0 + u1) * kLn2);
   st.w = fmaf(w_sh, sct, (w0 + w1) * kLn2);
-  // rest-sums and greedy top-2.  Without a new leader all of the sub-chunk's terms join the
-  // rest.  A new leader (rare: a few times per thread) leaves the sub-chunk's sum, and the old
-  // leader's exact 1 joins the rest, both rescaled to the new reference.
-  if (ct > st.best_t) {
-    const int jj = first_at(zt, ct);
-    const float e = sum_except(zt, bt, jj);
-    st.r_t = any ? fmaf(st.r_t + 1.f, sct, e) : e;
-    top2_lead(st.best_t, st.sec_t, st.i_t, zt, ct, jj, v0);
-  } else {
-    st.r_t += s0 + s1;
-    st.sec_t = fmaxf(st.sec_t, ct);
-  }
-  if (cd > st.best_d) {
-    const int jj = first_at(zd, cd);
-    const float e = sum_except(zd, bd, jj);
-    st.r_d = st.best_d > -INFINITY ? fmaf(st.r_d + 1.f, ex2((st.best_d - nbd) * kLog2e), e) : e;
-    top2_lead(st.best_d, st.sec_d, st.i_d, zd, cd, jj, v0);
-  } else {
-    st.r_d += d0 + d1;
-    st.sec_d = fmaxf(st.sec_d, cd);
-  }
+  sum2_scaled(st.s_t, st.c_t, sct, s0 + s1);
+  sum2_scaled(st.s_d, st.c_d, scd, d0 + d1);
+  // greedy top-2 of both sides (moves best_d / best_t to the new maxima nbd / nbt)
+  top2_update(st.best_d, st.sec_d, st.i_d, zd, cd, v0);
+  top2_update(st.best_t, st.sec_t, st.i_t, zt, ct, v0);
   const int xr = x - v0;
   if (xr >= 0 && xr < (kFull ? kSub : nv)) {
 #pragma unroll
@@ -881,9 +868,11 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
         float* o = args.part + part * P.N + row;
         if constexpr (is_fwd(kMode)) {
           o[kPMd * fs] = st.best_d;
-          o[kPSd * fs] = st.r_d;
+          o[kPSd * fs] = st.s_d;
+          o[kPSdLo * fs] = st.c_d;
           o[kPMt * fs] = st.best_t;
-          o[kPSt * fs] = st.r_t;
+          o[kPSt * fs] = st.s_t;
+          o[kPStLo * fs] = st.c_t;
           o[kPU * fs] = st.u;
           o[kPW * fs] = st.w;
           o[kPBd * fs] = st.best_d;

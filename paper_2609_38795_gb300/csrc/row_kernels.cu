@@ -106,9 +106,10 @@ __global__ void __launch_bounds__(256) combine_kernel(
   if (active) {
     for (int k = 0; k < P.n_parts; ++k) {
       const float* p = part + size_t(k) * P.N + r;
-      // a part's sum of exponentials is its leader's exact 1 plus the rest it kept
+      // a part's sums of exponentials, from their two-float parts
       const float md = p[kPMd * fs], mt = p[kPMt * fs];
-      const double sd = 1.0 + double(p[kPSd * fs]), st = 1.0 + double(p[kPSt * fs]);
+      const double sd = double(p[kPSd * fs]) + double(p[kPSdLo * fs]);
+      const double st = double(p[kPSt * fs]) + double(p[kPStLo * fs]);
       const float nmd = fmaxf(Md, md), nmt = fmaxf(Mt, mt);
       const float so = ex2((Mt - nmt) * kLog2e), sn = ex2((mt - nmt) * kLog2e);
       // U, Wt and the parts' u, w are measured from their own maxima (z_d - M_d, z_t - M_t):
