@@ -415,9 +415,9 @@ size_t alr_topk_fwd_workspace_size(const alr_params* p);
  *   tail contributes nothing), q = softmax(h_d W) over the whole vocabulary.
  * omega_r = weight_in[r] when weight_in is given (e.g. erase weights from alr_erase_weights),
  * else w_k * row_mask[r] (row_mask nullable = ones).  Label tokens must lie in [0, V).
- * tail_q is computed as (S - sum_i e^{z_i - m}) / S from the fp32 running sum S; when the
- * drafter puts almost all its mass on the label tokens (tail_q below ~1e-5) its relative
- * error grows accordingly.
+ * tail_q is the drafter's mass outside the label tokens, summed from the same exponentials as
+ * the log-sum-exp (the label tokens' own terms taken out as they were added), so its relative
+ * precision holds however little mass the drafter leaves outside the label.
  */
 int alr_topk_loss_fwd(const alr_params* p, const void* Hd, const void* W, const int32_t* top_idx,
                       const float* top_prob, const float* tail, const float* row_mask,

@@ -53,11 +53,19 @@ constexpr int kTopK = 8;
 
 // Partial record of the label readout: log-sum-exp state, the k best target logits with their
 // token ids, z_t at the corpus token.
-enum ReadoutField { kRM = 0, kRS, kRTop, kRIdx = kRTop + kTopK, kRZx = kRIdx + kTopK, kRFields };
+// kRSLo: the rounding error of the sum kRS (the sum is kRS + kRSLo); kRR: the exponent
+// residual r of the reference kRM (every summed exponential carries the factor 2^r).
+enum ReadoutField {
+  kRM = 0, kRS, kRTop, kRIdx = kRTop + kTopK, kRZx = kRIdx + kTopK, kRSLo, kRR, kRFields
+};
 
 // Partial record of the top-k loss forward: log-sum-exp state and greedy top-2 of z_d, and
 // z_d at the row's k label tokens (NaN where the token is outside the part's columns).
-enum TopkField { kKM = 0, kKS, kKBest, kKIdx, kKSec, kKZ, kKFields = kKZ + kTopK };
+// kKSLo: the rounding error of the sum kKS; kKSIn: the part of kKS that the row's label
+// tokens contributed (the same rounded terms); kKR: the exponent residual of kKM.
+enum TopkField {
+  kKM = 0, kKS, kKBest, kKIdx, kKSec, kKZ, kKSLo = kKZ + kTopK, kKSIn, kKR, kKFields
+};
 
 // What one launch of the fused loss kernel computes.
 enum LossMode {

@@ -155,10 +155,30 @@ ALR_DEV void load_masked(float (&z)[16], const uint32_t (&r)[16], int nv) {
   for (int j = 0; j < kSub; ++j) z[j] = (kFull || j < nv) ? f32(r[j]) : -INFINITY;
 }
 
+// (s, c) <- (s, c) * sc + x with the rounding error of the addition moved into c (Knuth's
+// TwoSum, branch-free: s + c holds the sum to about twice fp32 precision).  The error of the
+// product s * sc (sc < 1 only when the running maximum moves) is not kept.
+ALR_DEV void sum2_scaled(float& s, float& c, float sc, float x) {
+  const float t = s * sc;
+  const float y = t + x;
+  const float xb = y - t;
+  const float e = (t - (y - xb)) + (x - xb);
+  s = y;
+  c = fmaf(c, sc, e);
+}
+
+// The exponent every column gets relative to the reference m is fma(z, log2 e, -m log2 e),
+// which at z = m is not 0 but the rounding residual of m log2 e (exactly representable, up to
+// ~4e-6 at |m| ~ 40): every exponential summed against m carries the factor 2^r.  The merge
+// divides it out, so that log S and the log-probabilities taken from it keep their precision.
+ALR_DEV float exp_residual(float m) { return fmaf(m, kLog2e, -m * kLog2e); }
+
 // Online log-sum-exp: move the reference from m to max(m, cm) and add the sub-chunk's
-// exp(z - ref) (masked -inf columns add 0).  Even and odd columns are summed in the two lanes
-// of packed registers.
-ALR_DEV void lse_update(float& m, float& s, const float (&z)[16], float cm) {
+// exp(z - ref) (masked -inf columns add 0) to the compensated sum (s, c).  Even and odd
+// columns are summed in the two lanes of packed registers; each lane's exponential equals the
+// scalar ex2(fmaf(z, kLog2e, -m * kLog2e)) of its column.  Returns the factor the old sums
+// were rescaled by.
+ALR_DEV float lse_update(float& m, float& s, float& c, const float (&z)[16], float cm) {
   const float nm = fmaxf(m, cm);
   const float sc = ex2((m - nm) * kLog2e);
   const float b = -nm * kLog2e;
@@ -169,8 +189,9 @@ ALR_DEV void lse_update(float& m, float& s, const float (&z)[16], float cm) {
     r = f2_add(r, f2_ex2(f2_fma(f2_pack(z[j], z[j + 1]), l2e, b2)));
   float r0, r1;
   f2_unpack(r, r0, r1);
-  s = fmaf(s, sc, r0 + r1);
+  sum2_scaled(s, c, sc, r0 + r1);
   m = nm;
+  return sc;
 }
 
 // Greedy top-2 with lowest-index ties, given the sub-chunk maximum cm.  Columns reach a
@@ -235,18 +256,6 @@ ALR_DEV void stats_init(RowStats& st) {
   st.s_d = st.s_t = st.c_d = st.c_t = st.u = st.w = 0.f;
   st.i_d = st.i_t = 0x7fffffff;
   st.zx = qnan();
-}
-
-// (s, c) <- (s, c) * sc + x with the rounding error of the addition moved into c (Knuth's
-// TwoSum, branch-free: s + c holds the sum to about twice fp32 precision).  The error of the
-// product s * sc (sc < 1 only when the running maximum moves) is not kept.
-ALR_DEV void sum2_scaled(float& s, float& c, float sc, float x) {
-  const float t = s * sc;
-  const float y = t + x;
-  const float xb = y - t;
-  const float e = (t - (y - xb)) + (x - xb);
-  s = y;
-  c = fmaf(c, sc, e);
 }
 
 // Fold one 16-column sub-chunk (nv valid columns) into the full-vocabulary statistics.
@@ -672,7 +681,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
 
       // ---- per-row state for this unit ----
       RowStats st;                       // forward modes
-      float m = -INFINITY, s = 0.f;      // single-operand log-sum-exp state
+      float m = -INFINITY, s = 0.f, sc = 0.f;   // single-operand log-sum-exp state (s + sc)
+      float s_in = 0.f;                  // top-k forward: the label tokens' part of s
       float best = -INFINITY, sec = -INFINITY, zx = qnan();
       int bidx = 0x7fffffff, x = -1;
       float tk[kTopK];                   // readout: k best values / top-k forward: z_d at labels
@@ -779,7 +789,7 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
                 keep_logits_f32(r0, args.zd_out, size_t(row) * size_t(P.V) + size_t(v0), nv);
               }
             }
-            lse_update(m, s, z, cm);
+            const float resc = lse_update(m, s, sc, z, cm);
             if constexpr (kMode == kModeReadout) {
               const int xr = x - v0;
               if (xr >= 0 && xr < nv) {
@@ -803,16 +813,24 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
               }
             } else {
               top2_update(best, sec, bidx, z, cm, v0);
+              // the label tokens' exponentials, the very terms lse_update added to s, so that
+              // s - s_in is the drafter's mass outside the label (the tail bin's q) without a
+              // cancellation between separately rounded sums
+              s_in *= resc;
               bool hit = false;
 #pragma unroll
               for (int i = 0; i < kTopK; ++i) hit |= unsigned(ti[i] - v0) < unsigned(nv);
               if (hit) {
+                const float b = -m * kLog2e;
 #pragma unroll
                 for (int i = 0; i < kTopK; ++i) {
                   const int rel = ti[i] - v0;
 #pragma unroll
                   for (int j = 0; j < kSub; ++j)
-                    if (j == rel) tk[i] = z[j];
+                    if (j == rel) {
+                      tk[i] = z[j];
+                      s_in += ex2(fmaf(z[j], kLog2e, b));
+                    }
                 }
               }
             }
@@ -885,6 +903,8 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
         } else if constexpr (kMode == kModeReadout) {
           o[kRM * fs] = m;
           o[kRS * fs] = s;
+          o[kRSLo * fs] = sc;
+          o[kRR * fs] = exp_residual(m);
 #pragma unroll
           for (int i = 0; i < kTopK; ++i) {
             o[(kRTop + i) * fs] = tk[i];
@@ -894,6 +914,9 @@ __global__ void __launch_bounds__(Shape<kMode, kBN, is_staged(kMode, sizeof(Elem
         } else if constexpr (is_topk_fwd(kMode)) {
           o[kKM * fs] = m;
           o[kKS * fs] = s;
+          o[kKSLo * fs] = sc;
+          o[kKSIn * fs] = s_in;
+          o[kKR * fs] = exp_residual(m);
           o[kKBest * fs] = best;
           o[kKIdx * fs] = __int_as_float(bidx);
           o[kKSec * fs] = sec;

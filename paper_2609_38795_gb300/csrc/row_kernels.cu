@@ -304,6 +304,13 @@ __device__ __forceinline__ void insert_ranked(float (&t)[kTopK], int (&ti)[kTopK
   }
 }
 
+// 2^-r for the exponent residual r of a reference (|r| <= 4e-3 over the fp16 range of logits):
+// 1 - x + x^2 / 2 with x = r ln 2, within 5e-9 relative (1e-15 for |r| <= 3e-5, |logit| < 1000).
+__device__ __forceinline__ double inv_exp2_small(float r) {
+  const double x = double(r) * 0.6931471805599453;
+  return 1.0 - x + 0.5 * x * x;
+}
+
 // Label readout merge, one thread per row: log-sum-exp over all parts, the k best target
 // logits (ties to the lower id), their probabilities and the tail mass
 //   tail = (S - sum_k exp(t_k - M)) / S,
@@ -315,7 +322,8 @@ __global__ void __launch_bounds__(256) readout_combine_kernel(
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= P.N) return;
   const size_t fs = size_t(P.n_parts) * P.N;
-  float M = -INFINITY, S = 0.f, zx = quiet_nan();
+  float M = -INFINITY, zx = quiet_nan();
+  double S = 0.0;   // merged in fp64 from the parts' two-float sums
   float t[kTopK];
   int ti[kTopK];
 #pragma unroll
@@ -327,7 +335,9 @@ __global__ void __launch_bounds__(256) readout_combine_kernel(
     const float* p = part + size_t(k) * P.N + r;
     const float m = p[kRM * fs];
     const float nm = fmaxf(M, m);
-    S = S * ex2((M - nm) * kLog2e) + p[kRS * fs] * ex2((m - nm) * kLog2e);
+    const double sp = (double(p[kRS * fs]) + double(p[kRSLo * fs])) * inv_exp2_small(p[kRR * fs]);
+    S = (M > -INFINITY ? S * double(ex2((M - nm) * kLog2e)) : 0.0) +
+        (m > -INFINITY ? sp * double(ex2((m - nm) * kLog2e)) : 0.0);
     M = nm;
 #pragma unroll
     for (int i = 0; i < kTopK; ++i) {
@@ -337,20 +347,22 @@ __global__ void __launch_bounds__(256) readout_combine_kernel(
     const float z = p[kRZx * fs];
     if (z == z) zx = z;
   }
-  const float lse = M + logf(S);
+  const double ls = log(S);
+  const float lse = M + float(ls);
   double inside = 0.0;
 #pragma unroll
   for (int i = 0; i < kTopK; ++i) {
+    const double e = exp(double(t[i]) - double(M));
     top_idx[size_t(r) * kTopK + i] = ti[i];
-    top_prob[size_t(r) * kTopK + i] = expf(t[i] - lse);
-    inside += exp(double(t[i]) - double(M));
+    top_prob[size_t(r) * kTopK + i] = float(e / S);
+    inside += e;
   }
   // with V <= k every token is in the list and the tail is empty by definition
-  tail[r] = P.V <= kTopK ? 0.f : float(fmax(0.0, (double(S) - inside) / double(S)));
+  tail[r] = P.V <= kTopK ? 0.f : float(fmax(0.0, (S - inside) / S));
   if (lse_t) lse_t[r] = lse;
   if (argmax_t) argmax_t[r] = ti[0];
   if (gap_t) gap_t[r] = t[0] - t[1];
-  if (has_corpus && logp_x) logp_x[r] = zx - lse;
+  if (has_corpus && logp_x) logp_x[r] = float((double(zx) - double(M)) - ls);
 }
 
 // Top-k loss merge, one warp per anchor: log-sum-exp and greedy top-2 of z_d, the label
@@ -371,7 +383,10 @@ __global__ void __launch_bounds__(256) topk_combine_kernel(
   const bool active = lane < P.B;
   const int r = a * P.B + (active ? lane : 0);
   const size_t fs = size_t(P.n_parts) * P.N;
-  float M = -INFINITY, S = 0.f, bd = -INFINITY, secd = -INFINITY;
+  // the sum of exponentials is merged in fp64 from its two-float parts: with a sharp drafter
+  // its logarithm is the near-zero part of every log q
+  float M = -INFINITY, bd = -INFINITY, secd = -INFINITY;
+  double S = 0.0, Sout = 0.0;   // all columns; the columns outside the row's label tokens
   int id = 0x7fffffff;
   float zk[kTopK];
 #pragma unroll
@@ -381,7 +396,15 @@ __global__ void __launch_bounds__(256) topk_combine_kernel(
       const float* p = part + size_t(k) * P.N + r;
       const float m = p[kKM * fs];
       const float nm = fmaxf(M, m);
-      S = S * ex2((M - nm) * kLog2e) + p[kKS * fs] * ex2((m - nm) * kLog2e);
+      // the part's sums without the factor 2^r its exponentials carry
+      const double unr = inv_exp2_small(p[kKR * fs]);
+      const double sp = (double(p[kKS * fs]) + double(p[kKSLo * fs])) * unr;
+      const double so =
+          ((double(p[kKS * fs]) - double(p[kKSIn * fs])) + double(p[kKSLo * fs])) * unr;
+      const double f_old = M > -INFINITY ? double(ex2((M - nm) * kLog2e)) : 0.0;
+      const double f_new = m > -INFINITY ? double(ex2((m - nm) * kLog2e)) : 0.0;
+      S = S * f_old + sp * f_new;
+      Sout = Sout * f_old + so * f_new;
       M = nm;
       const float b2 = p[kKBest * fs], s2 = p[kKSec * fs];
       const int i2 = __float_as_int(p[kKIdx * fs]);
@@ -401,13 +424,13 @@ __global__ void __launch_bounds__(256) topk_combine_kernel(
   }
   float loss = 0.f, w = 0.f;
   if (active) {
-    const float lse = M + logf(S);
-    double inside = 0.0, ce = 0.0;
-    for (int i = 0; i < kTopK; ++i) {
-      inside += exp(double(zk[i]) - double(M));
-      ce -= double(top_prob[size_t(r) * kTopK + i]) * (double(zk[i]) - double(lse));
-    }
-    const double tq = fmax((double(S) - inside) / double(S), 1e-30);
+    const double ls = log(S);
+    const float lse = M + float(ls);
+    // log q_i = (z_i - M) - log S: the difference z_i - M is exact in fp64
+    double ce = 0.0;
+    for (int i = 0; i < kTopK; ++i)
+      ce -= double(top_prob[size_t(r) * kTopK + i]) * ((double(zk[i]) - double(M)) - ls);
+    const double tq = fmax(Sout / S, 1e-30);
     const float tl = tail[r];
     if (tl > 0.f) ce -= double(tl) * log(tq);
     loss = float(ce);

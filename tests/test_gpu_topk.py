@@ -343,3 +343,48 @@ def test_topk_logit_grad_from_logits_elementwise(scale):
     tol = 2.0 ** -8 * np.abs(ref) + 1e-5 * c[:, None] * (q + 1e-3) + P.FLUSH_FLOOR
     assert np.all(np.abs(got - ref) <= tol), np.abs(got - ref).max()
     assert np.all(got[5] == 0)
+
+
+@pytest.mark.parametrize("sigma", [0.1, 0.5])
+def test_text8b_sub_batch_sharp_head_compact_labels(sigma):
+    """The compact-label step's calls on 8 anchors (128 rows) at the text8b head with a head
+    scaled to trained-head logit sizes (|z| up to ~40): readout of H_t, top-8 forward keeping
+    z_d, G from the kept z_d in place, dH and dW through alr_gemm.  Labels, per-row losses and
+    every G, dH, dW entry against the oracle (1e-3 relative, 2e-2 max-norm)."""
+    wl = synthetic.WORKLOADS["text8b"]
+    A, B, lam = 8, wl.B, 1.013441
+    b = synthetic.sharpen(synthetic.slot_batch(wl.d, wl.V, A, B, sigma, device="cuda", seed=81))
+    Hd, Ht, W = b["Hd"], b["Ht"], b["W"]
+    N = A * B
+    Hd64, Ht64, W64 = P.np64(Hd), P.np64(Ht), P.np64(W)
+    g = gpu_readout(Ht, W, B)
+    r = orc.label_readout(Ht64, W64, k=K)
+    assert np.abs(r["z_t"]).max() > 30.0
+    compare_readout(g, r)
+    lab = dict(idx=g["top_idx"], prob=g["top_prob"], tail=g["tail"])
+    idx, prob, tail = host_labels(lab)
+    Zd = torch.empty(N, wl.V, dtype=torch.float16, device="cuda")
+    Rd = torch.empty(alr.alr_kept_ref_groups(wl.V), N, dtype=torch.float16, device="cuda")
+    params, out = gpu_topk_forward(Hd, W, B, lab, lam=lam, Zd=Zd, Zd_ref=Rd)
+    z_d = Hd64 @ W64
+    P.check_kept(Zd, Rd, z_d)
+    loss_r, tq_r = orc.top_k_soft_cross_entropy(z_d, idx, prob, tail)
+    assert P.rel_err(P.np64(out["loss_row"]), loss_r).max() <= P.LOSS_RTOL
+    w_r = orc.slot_weights(orc.MODE_ALR, B, 2.0, N)
+    G = Zd.view(torch.bfloat16)
+    alr.alr_topk_logit_grad_from_logits(params, Zd, Rd, lab["idx"], lab["prob"], lab["tail"],
+                                        out["weight"], out["weight_sum"], out["lse_d"],
+                                        out["tail_q"], G)
+    dH = torch.empty(N, wl.d, device="cuda")
+    dW = torch.zeros(wl.d, wl.V, device="cuda")
+    alr.alr_gemm(G, W, dH, N, wl.d, wl.V)
+    alr.alr_gemm(Hd, G, dW, wl.d, wl.V, N, a_mn=True, b_mn=True, accumulate=True)
+    torch.cuda.synchronize()
+    G_r = orc.top_k_logit_grad(z_d, idx, prob, tail, w_r, lam)
+    dH_r, dW_r = orc.slot_loss_backward(Hd64, W64, G_r)
+    errs = (P.max_norm_rel(P.np64(G), G_r), P.max_norm_rel(P.np64(dH), dH_r),
+            P.max_norm_rel(P.np64(dW), dW_r))
+    print(f"compact labels, sharp head, sigma={sigma}: loss rel err "
+          f"{P.rel_err(P.np64(out['loss_row']), loss_r).max():.2e}, G/dH/dW {errs}")
+    assert max(errs) <= P.GRAD_RTOL
+    assert alr.alr_device_status() == alr.ALR_OK
