@@ -245,7 +245,7 @@ int alr_slot_loss_fwd(const alr_params* p, const void* Hd, const void* Ht, const
  *
  *   - Limit: problems whose alr_fwd_workspace_size exceeds ALR_NOALLOC_SCRATCH_BYTES are
  *     rejected with ALR_ERR_INVALID_ARG and a message naming both sizes (bf16 at d=4096,
- *     B=16 on a 152-SM GB300: about 16 900 rows).
+ *     V=151936, B=16 on a 152-SM GB300: about 14 700 rows).
  *   - Memory: every device that loads the library holds the array until the process exits.
  *   - Set-up: the first call on a device (with that device current) looks up the array's
  *     device address; make that first call before any stream capture.  The address is kept
