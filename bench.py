@@ -945,28 +945,30 @@ def run_gpu(args, rank, world, local_rank):
         "clocks": clk,
         "cpu_baseline": cpu,
     }
-    # The step the hot path's outline describes (logits never stored; the backward recomputes
-    # its logit tiles), with its own roofline record: timed here as `recompute` beside the
-    # default kept-logits step, or as the main step under --step recompute.
-    ns = other if keep else {"ms_per_step": ms_step, "rows_per_s": rows_per_s, "phase_ms": phase_ms}
-    if ns is not None:
-        ns_flops = {"fwd": 4 * NdV, "logit_grad": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
-        ns_dom = max(ns_flops, key=lambda ph: ns["phase_ms"][ph])
-        ns_ach = ns_flops[ns_dom] / (ns["phase_ms"][ns_dom] / 1e3) / 1e12
-        out["north_star_rows_per_s"] = ns["rows_per_s"]
-        out["north_star"] = {
+    # The step that never stores the logits (the backward recomputes its logit tiles), with
+    # its own roofline record: timed as `recompute` beside the default kept-logits step, or as
+    # the main step under --step recompute.
+    rc = other if keep else {"ms_per_step": ms_step, "rows_per_s": rows_per_s,
+                             "phase_ms": phase_ms}
+    if rc is not None:
+        rc_flops = {"fwd": 4 * NdV, "logit_grad": 4 * NdV, "dH_gemm": 2 * NdV, "dW_gemm": 2 * NdV}
+        rc_dom = max(rc_flops, key=lambda ph: rc["phase_ms"][ph])
+        rc_ach = rc_flops[rc_dom] / (rc["phase_ms"][rc_dom] / 1e3) / 1e12
+        out["recompute_rows_per_s"] = rc["rows_per_s"]
+        rec = out.setdefault("recompute", {}) if not keep else out["recompute"]
+        rec.update({
             "what": "logits never stored: the forward reduces both logit tiles on chip, the "
                     "backward recomputes them (12 NdV tensor flops per step)",
-            "rows_per_s": ns["rows_per_s"], "ms_per_step": ns["ms_per_step"],
-            "executed_tflops_12NdV": 12 * NdV / (ns["ms_per_step"] / 1e3) / 1e12,
-            "algorithmic_tflops_8NdV": 8 * NdV / (ns["ms_per_step"] / 1e3) / 1e12,
-            "roofline": {"bound": "tensor", "kernel": ns_dom, "achieved": ns_ach,
+            "rows_per_s": rc["rows_per_s"], "ms_per_step": rc["ms_per_step"],
+            "executed_tflops_12NdV": 12 * NdV / (rc["ms_per_step"] / 1e3) / 1e12,
+            "algorithmic_tflops_8NdV": 8 * NdV / (rc["ms_per_step"] / 1e3) / 1e12,
+            "roofline": {"bound": "tensor", "kernel": rc_dom, "achieved": rc_ach,
                          "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
-                         "frac": ns_ach / pk["bf16_sustained"],
-                         "frac_of_burst_peak": ns_ach / pk["bf16"],
-                         "traffic": kernel_traffic(ns_dom + "_recompute"),
-                         "flops_per_launch": ns_flops[ns_dom],
-                         "peak_note": f"{pk['source']} sustained bf16"}}
+                         "frac": rc_ach / pk["bf16_sustained"],
+                         "frac_of_burst_peak": rc_ach / pk["bf16"],
+                         "traffic": kernel_traffic(rc_dom + "_recompute"),
+                         "flops_per_launch": rc_flops[rc_dom],
+                         "peak_note": f"{pk['source']} sustained bf16"}})
     if e2e is not None:
         out["e2e"] = {"value": job_rows_per_s(world, wl.N, K, e2e_ms), "unit": UNIT,
                       "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
