@@ -31,9 +31,12 @@
  *              multicast) | single | mcast4 | pair (CTA pairs with M = 256 tcgen05 products)
  *              selects the bf16 GEMM kernel; ALR_LOSS_FORM = single (default) | mcast selects
  *              the fused loss kernels' form.  fp32 (tf32) products always run on single CTAs.
- *              A process launched as one rank of several (environment WORLD_SIZE > 1) never
- *              uses the multicast forms: mcast and mcast4 run as single there, so TMA multicast
- *              loads stay in single-GPU runs.  alr_kernel_forms() reports the choice.
+ *              The cluster forms (mcast, mcast4, pair, and the loss kernels' mcast) are built
+ *              into a second library, libalr_cluster.so, which this library loads from its own
+ *              directory on first use.  A process launched as one rank of several (environment
+ *              WORLD_SIZE > 1) never loads it, so TMA multicast loads stay out of multi-rank
+ *              processes; there, or if it cannot be loaded, every form runs on single CTAs.
+ *              alr_kernel_forms() reports the choice, alr_cluster_forms_error() the reason.
  */
 #ifndef ALR_H
 #define ALR_H
@@ -114,6 +117,13 @@ int alr_device_status(void* stream, int clear);
  *   *loss: 0 single CTAs, 1 clusters of two sharing head tiles by TMA multicast.
  */
 int alr_kernel_forms(int32_t* gemm, int32_t* loss);
+
+/*
+ * "" when libalr_cluster.so (the cluster kernel forms) is loaded in this process, else why it
+ * is not: the process is one rank of several, or the loader's message.  Loads it on first use
+ * (no device needed).  The string is owned by the library and stays valid.
+ */
+const char* alr_cluster_forms_error(void);
 
 /*
  * Test hook for the failure-detection path (the paper has no counterpart).  With enable != 0,

@@ -55,6 +55,7 @@ SIGNATURES = {
     "alr_device_supported": (_c_int, []),
     "alr_device_status": (_c_int, [_c_p, _c_int]),
     "alr_kernel_forms": (_c_int, [_c_p, _c_p]),
+    "alr_cluster_forms_error": (ctypes.c_char_p, []),
     "alr_debug_withhold_next_stage": (_c_int, [_c_int]),
     "alr_gather_ira_blocks": (_c_int, [_c_p, _c_i32, _c_i32, _c_i32, _c_i32, _c_p, _c_p, _c_p,
                                        _c_i32, _c_i32, _c_p, _c_p, _c_p]),
@@ -238,6 +239,12 @@ def alr_kernel_forms():
     g, l = ctypes.c_int32(), ctypes.c_int32()
     _check(lib().alr_kernel_forms(ctypes.byref(g), ctypes.byref(l)))
     return GEMM_FORMS[g.value], LOSS_FORMS[l.value]
+
+
+def alr_cluster_forms_error() -> str:
+    """"" when libalr_cluster.so (the cluster kernel forms) is loaded in this process, else why
+    it is not."""
+    return lib().alr_cluster_forms_error().decode()
 
 
 def alr_debug_withhold_next_stage(enable=True) -> int:

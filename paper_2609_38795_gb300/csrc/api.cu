@@ -12,6 +12,7 @@
 #include <nvtx3/nvToolsExt.h>
 
 #include "alr.h"
+#include "cluster_forms.h"
 #include "kernels.h"
 
 namespace {
@@ -169,24 +170,17 @@ int check_kept(const alr_params* p, const void* Z, const void* ref, const char* 
 #define ALR_LOSS_BN 256
 #endif
 
-// True in a process launched as one rank of several (WORLD_SIZE > 1, as torchrun and
-// torch.distributed set it): such a process uses no kernel form with TMA multicast loads, so
-// that multicast reads of device memory stay in single-GPU runs.
-bool multi_rank_process() {
-  const char* w = getenv("WORLD_SIZE");
-  return w != nullptr && atoi(w) > 1;
-}
-
 // The fused loss kernels run on single CTAs unless the environment variable ALR_LOSS_FORM is
-// "mcast" (bf16 inputs, single-GPU runs): clusters of two CTAs sharing every head tile by TMA
-// multicast.  The
-// dual-product modes already share each head tile between z_d and z_t, and at the power cap
-// the multicast form settles ~4 % lower in clock for ~1 % fewer L2 bytes per product: it is
-// not faster, so it is not the default.  Both forms give bit-identical results.
+// "mcast" (bf16 inputs): clusters of two CTAs sharing every head tile by TMA multicast, from
+// libalr_cluster.so, which only a single-process run loads (alr::cluster_forms() is nullptr in
+// a multi-rank process, and then the single form runs).  The dual-product modes already share
+// each head tile between z_d and z_t, and at the power cap the multicast form settles ~4 %
+// lower in clock for ~1 % fewer L2 bytes per product: it is not faster, so it is not the
+// default.  Both forms give bit-identical results.
 bool loss_multicast(const alr_params* p) {
-  if (p->dtype != ALR_BF16 || ALR_LOSS_BN != 256 || multi_rank_process()) return false;
+  if (p->dtype != ALR_BF16 || ALR_LOSS_BN != 256) return false;
   const char* v = getenv("ALR_LOSS_FORM");
-  return v != nullptr && strcmp(v, "mcast") == 0;
+  return v != nullptr && strcmp(v, "mcast") == 0 && alr::cluster_forms() != nullptr;
 }
 
 // two_rows: the single-operand modes (readout, top-k), whose units hold two row blocks.
@@ -278,23 +272,25 @@ BwdLayout bwd_layout(const alr_params* p, bool with_g = true) {
 
 // Form of the bf16 products, chosen by the environment variable ALR_GEMM_FORM:
 //   "mcast"   clusters of two CTAs, each on a 128 x 256 tile, sharing every B tile by TMA
-//             multicast (plain_gemm.cu), the default;
-//   "single"  one CTA per 128 x 256 tile, each loading its own B tiles;
-//   "pair"    CTA pairs with M = 256 products (pair_gemm.cu).
+//             multicast, the default;
+//   "single"  one CTA per 128 x 256 tile, each loading its own B tiles (plain_gemm.cu);
+//   "pair"    CTA pairs with M = 256 products.
+// The cluster forms ("mcast", "mcast4", "pair") live in libalr_cluster.so (csrc_cluster/),
+// which only a single-process run loads: in a process that is one rank of several, or where
+// that library cannot be loaded, every form runs as "single" (alr_kernel_forms reports it).
 // The step runs at the GB300's power cap, so the form that moves fewest bytes per product
 // wins: multicast halves the B traffic out of L2 and runs 6 % faster than single CTAs at the
 // same clock and power.  The pair form issues more products per clock but draws more power
 // per product and settles at a clock ~20 % lower.  tf32 products always run on single CTAs.
 //   "mcast4"  as "mcast" with clusters of four CTAs, each loading a quarter of the B tile.
-// One rank of a multi-rank launch never takes the multicast forms: "mcast", "mcast4" and the
-// default run as "single" there.
 enum GemmForm { kGemmSingle = 0, kGemmMcast = 1, kGemmPair = 2, kGemmMcast4 = 3 };
 
 GemmForm gemm_form(int dtype) {
   if (dtype != ALR_BF16) return kGemmSingle;
   const char* v = getenv("ALR_GEMM_FORM");
+  if ((v != nullptr && strcmp(v, "single") == 0) || alr::cluster_forms() == nullptr)
+    return kGemmSingle;
   if (v != nullptr && strcmp(v, "pair") == 0) return kGemmPair;
-  if (multi_rank_process() || (v != nullptr && strcmp(v, "single") == 0)) return kGemmSingle;
   if (v != nullptr && strcmp(v, "mcast4") == 0) return kGemmMcast4;
   return kGemmMcast;
 }
@@ -345,16 +341,17 @@ int launch_gemm(int dt, bool a_mn, bool b_mn, bool acc, const CUtensorMap& ma,
                 cudaStream_t s, const char* what) {
   cudaError_t e;
   const GemmForm form = gemm_form(dt);
+  const alr::ClusterForms* cf = alr::cluster_forms();   // non-NULL for every cluster form
   if (form == kGemmPair) {
-    const int pairs = alr::pair_gemm_max_pairs();
+    const int pairs = cf->pair_gemm_max_pairs();
     if (pairs < 1) return fail(ALR_ERR_CUDA, "%s: no CTA pair of the GEMM fits on this device", what);
     alr::GemmArgs g = pair_gemm_plan(M, Nc, K, C, ldc, pairs);
     g.status = alr::device_status_ptr();
     if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
-    e = alr::launch_pair_gemm(a_mn, b_mn, acc, ma, mb, g, s);
+    e = cf->launch_pair_gemm(a_mn, b_mn, acc, &ma, &mb, &g, s);
   } else if (form == kGemmMcast || form == kGemmMcast4) {
     const int cl = form == kGemmMcast4 ? 4 : 2;
-    const int clusters = alr::plain_gemm_mc_max_clusters(cl);
+    const int clusters = cf->gemm_max_clusters(cl);
     if (clusters < 1)
       return fail(ALR_ERR_CUDA, "%s: no CTA cluster of the GEMM fits on this device", what);
     // 128-row blocks in groups of `cl`: n_mb counts groups, raster groups of 16 row blocks
@@ -367,7 +364,7 @@ int launch_gemm(int dt, bool a_mn, bool b_mn, bool acc, const CUtensorMap& ma,
     g.status = alr::device_status_ptr();
     if (g.status == nullptr) return fail(ALR_ERR_CUDA, "status word lookup failed");
     g.withhold_first_stage = g_withhold_next.exchange(0);
-    e = alr::launch_plain_gemm_mc(cl, a_mn, b_mn, acc, ma, mb, g, s);
+    e = cf->launch_gemm(cl, a_mn, b_mn, acc, &ma, &mb, &g, s);
   } else {
     alr::GemmArgs g = gemm_plan(M, Nc, K, C, ldc, sms);
     g.status = alr::device_status_ptr();
@@ -481,6 +478,10 @@ int alr_kernel_forms(int32_t* gemm, int32_t* loss) {
   *gemm = int32_t(gemm_form(ALR_BF16));
   *loss = loss_multicast(&p) ? 1 : 0;
   return ALR_OK;
+}
+
+const char* alr_cluster_forms_error(void) {
+  return alr::cluster_forms() != nullptr ? "" : alr::cluster_forms_error();
 }
 
 int alr_debug_withhold_next_stage(int enable) {

@@ -134,24 +134,8 @@ cudaError_t launch_plain_gemm(int dtype, bool a_mn, bool b_mn, bool accumulate,
                               const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,
                               cudaStream_t s);
 size_t plain_gemm_smem_bytes(int dtype);
-// The multicast form of the same kernel (bf16): clusters of `cluster` (2 or 4) CTAs over row
-// blocks cluster i .. cluster i + cluster - 1 share each B tile (n_mb counts row-block groups,
-// `grid` is `cluster` times the number of clusters; the K-major B map has 256 / cluster-row
-// boxes).
-cudaError_t launch_plain_gemm_mc(int cluster, bool a_mn, bool b_mn, bool accumulate,
-                                 const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,
-                                 cudaStream_t s);
-// Clusters of `cluster` CTAs of the multicast GEMM that can be resident at once (0 on error).
-int plain_gemm_mc_max_clusters(int cluster);
-
-// The same products (bf16 operands only) on CTA pairs with M = 256 tcgen05 products
-// (pair_gemm.cu).  Here n_mb counts 256-row pair blocks, `grid` is twice the number of pairs,
-// and the B tensor map has 128-row boxes (K-major) or 64 x 64 boxes (MN-major).
-cudaError_t launch_pair_gemm(bool a_mn, bool b_mn, bool accumulate, const CUtensorMap& a,
-                             const CUtensorMap& b, const GemmArgs& args, cudaStream_t s);
-// CTA pairs of the pair GEMM that can be resident at once on the current device (0 on error).
-int pair_gemm_max_pairs();
-size_t pair_gemm_smem_bytes();
+// The cluster forms of the same kernel (multicast clusters, CTA pairs) are in
+// libalr_cluster.so (cluster_forms.h).
 
 // Row-level kernels (row_kernels.cu).
 cudaError_t launch_gather(const void* feat, int S, int L, int d, int elem_bytes,

@@ -290,13 +290,11 @@ ALR_DEV void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: 
 
 ALR_DEV bool elect_one_lane() { return (threadIdx.x & 31u) == 0; }
 
-// ------------------------------------------------- CTA pairs (2-SM tensor-core products) ---
-// (The cluster coordinates are constant for a kernel's lifetime: their reads are not volatile,
-// so the compiler may re-read them instead of holding them in registers.)
-// A cluster of two CTAs on neighbouring SMs computes one M = 256 product: each CTA holds 128
-// rows of A and half of the columns of B in its own shared memory, and receives its 128 rows
-// of D in its own tensor memory.  The even CTA issues the MMAs for both; all tcgen05
-// allocation, MMA and commit instructions of such a kernel use .cta_group::2.
+// ------------------------------------------------------------------ cluster coordinates ---
+// (Constant for a kernel's lifetime: their reads are not volatile, so the compiler may re-read
+// them instead of holding them in registers.)  The kernel forms that share operand tiles across
+// the CTAs of a cluster, and their PTX, are built into a library of their own from
+// csrc_cluster/; these sources only name the coordinates and the cluster barrier.
 ALR_DEV uint32_t cluster_ctarank() {
   uint32_t r;
   asm("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -315,126 +313,16 @@ ALR_DEV uint32_t n_clusters_x() {
   return r;
 }
 
-// Shared::cluster address of the object at the same offset as `p` in CTA `rank`'s smem.
-ALR_DEV uint32_t cluster_addr(const void* p, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
-  return r;
-}
-
-// All threads of both CTAs: arrive (release) and wait (acquire).
+// All threads of every CTA of the cluster: arrive (release) and wait (acquire).
 ALR_DEV void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" :::
                    "memory");
 }
 
-// Arrive on an mbarrier in any CTA of the cluster (release at cluster scope).
-ALR_DEV void mbar_arrive_cluster(uint32_t cluster_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar)
-               : "memory");
-}
-
-// As mbar_try_wait, acquiring at cluster scope (arrivals come from the peer CTA too).
-ALR_DEV bool mbar_try_wait_cl(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
-      : "memory");
-  return done != 0;
-}
-
-ALR_DEV bool mbar_wait_cl(uint64_t* bar, uint32_t parity, const AbortFlag& ab) {
-  if (mbar_try_wait_cl(bar, parity)) return true;
-  const uint64_t t0 = global_timer_ns();
-  for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait_cl(bar, parity)) return true;
-    if (i % kWaitCheckEvery == 0) {
-      if (*ab.smem) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
-        *ab.smem = 1;
-        atomicExch(ab.status, kStatusTimeout);
-        return false;
-      }
-    }
-  }
-}
-
-ALR_DEV void mbar_wait_drain_cl(uint64_t* bar, uint32_t parity) {
-  const uint64_t t0 = global_timer_ns();
-  while (!mbar_try_wait_cl(bar, parity)) {
-    if (global_timer_ns() - t0 > kWaitLimitNs) return;
-  }
-}
-
-// TMA tile load into this CTA's shared memory whose completion is counted on an mbarrier of
-// either CTA of the pair (`cluster_bar`, a shared::cluster address).
-ALR_DEV void tma_load_2d_pair(void* smem_dst, const CUtensorMap* map, uint32_t cluster_bar, int x,
-                              int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(cluster_bar), "r"(x), "r"(y)
-      : "memory");
-}
-
-// TMA tile load multicast to the CTAs of `cta_mask`: the tile lands at `smem_dst`'s offset in
-// each of them and completes on the mbarrier at `bar`'s offset in each of them.
-ALR_DEV void tma_load_2d_mc(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
-                            uint16_t cta_mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(cta_mask)
-      : "memory");
-}
-
-// mma_commit that arrives on the mbarrier at `bar`'s offset in every CTA of `cta_mask`.
-ALR_DEV void mma_commit_mc(uint64_t* bar, uint16_t cta_mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(smem_u32(bar)),
-      "h"(cta_mask)
-      : "memory");
-}
-
-// Collective tensor-memory allocation over the pair: one warp of each CTA executes it.
-ALR_DEV void tmem_alloc_pair(uint32_t* smem_result, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(smem_result)),
-               "r"(ncols)
-               : "memory");
-}
-ALR_DEV void tmem_relinquish_pair() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
-}
-ALR_DEV void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-
-// One M = 256 product for the pair (bf16 operands), issued by the even CTA.
-ALR_DEV void mma_issue_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                            uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// Arrive once on the mbarrier at `bar`'s offset in every CTA of `cta_mask` when all pair
-// products this thread issued so far have completed.
-ALR_DEV void mma_commit_pair(uint64_t* bar, uint16_t cta_mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(smem_u32(bar)),
-      "h"(cta_mask)
-      : "memory");
-}
+// The form of a kernel that runs without clusters: no CTA shares its operand tiles.
+struct NoCluster {
+  static constexpr int kCtas = 1;
+};
 
 ALR_DEV uint8_t* align_1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));

@@ -13,11 +13,12 @@
 // stage counts the bytes of both CTAs' loads (TMA .cta_group::2 completes on the peer's
 // barrier); the products' commit releases the stage in both CTAs at once (multicast), and
 // the epilogue warps of both CTAs release an accumulator buffer on the even CTA's barrier.
-// Every wait is bounded (tc_common.cuh).
+// Every wait is bounded (tc_common.cuh, cluster_ptx.cuh).  Built into libalr_cluster.so only.
 #include <atomic>
 
+#include "cluster_forms.h"
+#include "cluster_ptx.cuh"
 #include "kernels.h"
-#include "tc_common.cuh"
 
 namespace alr {
 namespace {
@@ -288,9 +289,12 @@ cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs&
 
 }  // namespace
 
-size_t pair_gemm_smem_bytes() { return kSmemBytes; }
+}  // namespace alr
 
-int pair_gemm_max_pairs() {
+extern "C" {
+
+int alr_cluster_pair_gemm_max_pairs(void) {
+  using namespace alr;
   // per-device occupancy, computed once (concurrent first calls compute the same value)
   static std::atomic<int> cached[64];
   int dev = 0;
@@ -318,19 +322,22 @@ int pair_gemm_max_pairs() {
   return n;
 }
 
-cudaError_t launch_pair_gemm(bool a_mn, bool b_mn, bool accumulate, const CUtensorMap& a,
-                             const CUtensorMap& b, const GemmArgs& args, cudaStream_t s) {
+cudaError_t alr_cluster_launch_pair_gemm(int a_mn, int b_mn, int accumulate, const CUtensorMap* a,
+                                         const CUtensorMap* b, const alr::GemmArgs* args,
+                                         cudaStream_t s) {
+  using namespace alr;
+  if (a == nullptr || b == nullptr || args == nullptr) return cudaErrorInvalidValue;
   const int key = (a_mn ? 4 : 0) | (b_mn ? 2 : 0) | (accumulate ? 1 : 0);
   switch (key) {
-    case 0: return launch_t<false, false, false>(a, b, args, s);
-    case 1: return launch_t<false, false, true>(a, b, args, s);
-    case 2: return launch_t<false, true, false>(a, b, args, s);
-    case 3: return launch_t<false, true, true>(a, b, args, s);
-    case 4: return launch_t<true, false, false>(a, b, args, s);
-    case 5: return launch_t<true, false, true>(a, b, args, s);
-    case 6: return launch_t<true, true, false>(a, b, args, s);
-    default: return launch_t<true, true, true>(a, b, args, s);
+    case 0: return launch_t<false, false, false>(*a, *b, *args, s);
+    case 1: return launch_t<false, false, true>(*a, *b, *args, s);
+    case 2: return launch_t<false, true, false>(*a, *b, *args, s);
+    case 3: return launch_t<false, true, true>(*a, *b, *args, s);
+    case 4: return launch_t<true, false, false>(*a, *b, *args, s);
+    case 5: return launch_t<true, false, true>(*a, *b, *args, s);
+    case 6: return launch_t<true, true, false>(*a, *b, *args, s);
+    default: return launch_t<true, true, true>(*a, *b, *args, s);
   }
 }
 
-}  // namespace alr
+}  // extern "C"

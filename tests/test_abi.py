@@ -3,8 +3,11 @@
 No kernel is launched here (these run without a GPU)."""
 
 import ctypes
+import json
 import os
 import re
+import subprocess
+import sys
 
 import pytest
 
@@ -206,19 +209,69 @@ def test_error_paths_reject_before_any_device_work(libalr):
         assert text in msg, (name, msg)
 
 
-def test_multi_rank_processes_use_no_multicast_forms(libalr, monkeypatch):
-    """One rank of a multi-rank launch (WORLD_SIZE > 1) never takes a kernel form with TMA
-    multicast loads, whatever the environment asks; a single process keeps its choice."""
+_FORMS_CHILD = r"""
+import ctypes, json, sys
+h = ctypes.CDLL(sys.argv[1])
+h.alr_cluster_forms_error.restype = ctypes.c_char_p
+g, l = ctypes.c_int32(), ctypes.c_int32()
+assert h.alr_kernel_forms(ctypes.byref(g), ctypes.byref(l)) == 0
+why = h.alr_cluster_forms_error().decode()
+maps = open("/proc/self/maps").read()
+print(json.dumps({"forms": [g.value, l.value], "why": why,
+                  "cluster_mapped": "libalr_cluster.so" in maps}))
+"""
+
+
+def _forms_in_child(env_over):
+    env = {k: v for k, v in os.environ.items()
+           if k not in ("WORLD_SIZE", "ALR_GEMM_FORM", "ALR_LOSS_FORM")}
+    env.update(env_over)
+    r = subprocess.run([sys.executable, "-c", _FORMS_CHILD, build_lib.LIB], env=env,
+                       capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0, r.stderr
+    out = json.loads(r.stdout.strip().splitlines()[-1])
+    g, l = out["forms"]
+    return (alr.GEMM_FORMS[g], alr.LOSS_FORMS[l]), out["why"], out["cluster_mapped"]
+
+
+def test_multi_rank_processes_never_load_the_cluster_forms(libalr):
+    """The kernel forms with TMA multicast loads (and the CTA-pair GEMM) live in
+    libalr_cluster.so.  A single process loads it and keeps its choice of form; one rank of a
+    multi-rank launch (WORLD_SIZE > 1) never maps it and runs every form on single CTAs,
+    whatever the environment asks.  Each case is a fresh process: the library decides once."""
     for world, gemm_env, loss_env, want in (
             (None, None, None, ("mcast", "single")),
             ("1", "mcast4", "mcast", ("mcast4", "mcast")),
+            (None, "pair", None, ("pair", "single")),
+            (None, "single", "single", ("single", "single")),
             ("2", None, None, ("single", "single")),
             ("8", "mcast", "mcast", ("single", "single")),
             ("4", "mcast4", None, ("single", "single")),
-            ("2", "pair", None, ("pair", "single"))):
-        for k, v in (("WORLD_SIZE", world), ("ALR_GEMM_FORM", gemm_env), ("ALR_LOSS_FORM", loss_env)):
-            if v is None:
-                monkeypatch.delenv(k, raising=False)
-            else:
-                monkeypatch.setenv(k, v)
-        assert alr.alr_kernel_forms() == want, (world, gemm_env, loss_env)
+            ("2", "pair", None, ("single", "single"))):
+        env = {k: v for k, v in (("WORLD_SIZE", world), ("ALR_GEMM_FORM", gemm_env),
+                                 ("ALR_LOSS_FORM", loss_env)) if v is not None}
+        forms, why, mapped = _forms_in_child(env)
+        multi = world is not None and int(world) > 1
+        assert forms == want, (env, forms, why)
+        assert mapped == (not multi), (env, why)
+        assert (why == "") == (not multi) and (not multi or "rank" in why), (env, why)
+
+
+def test_cluster_forms_are_built_apart():
+    """No source of libalr.so issues a multicast copy or commit, or a 2-SM product; the cluster
+    library's sources do, and it exports the loader's entry points."""
+    pat = re.compile(r"multicast::cluster|cta_group::2")
+    for d in (build_lib.CSRC, build_lib.INCLUDE):
+        for f in os.listdir(d):
+            with open(os.path.join(d, f)) as fh:
+                code = re.sub(r"/\*.*?\*/", "", fh.read(), flags=re.S)   # PTX, not comments
+            code = "\n".join(line.split("//")[0] for line in code.splitlines())
+            assert not pat.search(code), f
+    cl = "".join(open(os.path.join(build_lib.CSRC_CLUSTER, f)).read()
+                 for f in os.listdir(build_lib.CSRC_CLUSTER))
+    assert pat.search(cl)
+    h = ctypes.CDLL(build_lib.LIB_CLUSTER)
+    for name in ("alr_cluster_args_size", "alr_cluster_launch_loss", "alr_cluster_launch_gemm",
+                 "alr_cluster_gemm_max_clusters", "alr_cluster_launch_pair_gemm",
+                 "alr_cluster_pair_gemm_max_pairs"):
+        assert hasattr(h, name), name

@@ -30,6 +30,7 @@ def test_withheld_stage_times_out_and_context_survives(form, monkeypatch):
     other's stages by multicast (every CTA of the cluster then runs out on its own barriers
     and both meet at the closing cluster barrier)."""
     monkeypatch.setenv("ALR_LOSS_FORM", form)
+    assert alr.alr_kernel_forms()[1] == form, alr.alr_cluster_forms_error()
     A, B, d, V = 16, 16, 256, 1024
     b = synthetic.slot_batch(d, V, A, B, 0.5, dtype=torch.bfloat16, device="cuda", seed=9)
     sl = alr.SlotLoss(A * B, d, V, B)
@@ -56,6 +57,7 @@ def test_withheld_gemm_stage_times_out_and_context_survives(form, monkeypatch):
     makes every CTA give up (one epilogue warp sees the abort and the others follow it out of
     their named barrier), the timeout is reported, and the next product is correct."""
     monkeypatch.setenv("ALR_GEMM_FORM", form)
+    assert alr.alr_kernel_forms()[0] == form, alr.alr_cluster_forms_error()
     M, Nc, K = 1024, 768, 512
     g = torch.Generator(device="cuda").manual_seed(5)
     A = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)

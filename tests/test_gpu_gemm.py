@@ -44,6 +44,7 @@ def test_gemm_layouts(form, dtype, a_mn, b_mn, shape, monkeypatch):
     if dtype == torch.float32 and form != "single":
         pytest.skip("tf32 products have one form")
     monkeypatch.setenv("ALR_GEMM_FORM", form)
+    assert alr.alr_kernel_forms()[0] == form, alr.alr_cluster_forms_error()
     M, Nc, K = shape
     if dtype == torch.float32 and (a_mn or b_mn):
         A_st, B_st, _ = _operands(M, Nc, K, dtype, a_mn, b_mn, seed=1)

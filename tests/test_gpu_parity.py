@@ -391,6 +391,7 @@ def test_loss_kernel_forms_agree_bit_for_bit(N, monkeypatch):
     monkeypatch.setenv("ALR_LOSS_FORM", "single")
     single = _all_outputs(Hd, Ht, W, B, alr.ALR_MODE_ERASE_SOFT, tok)
     monkeypatch.setenv("ALR_LOSS_FORM", "mcast")
+    assert alr.alr_kernel_forms()[1] == "mcast", alr.alr_cluster_forms_error()
     mcast = _all_outputs(Hd, Ht, W, B, alr.ALR_MODE_ERASE_SOFT, tok)
     for k in single:
         a, b = single[k].cpu(), mcast[k].cpu()
