@@ -84,7 +84,7 @@ def peaks():
 
 # ------------------------------------------------------------------ DRAM traffic ---
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "loss_gemm_traffic.json")
-KERNEL_SOURCES = ["paper_2609_38795_gb300/csrc/loss_gemm.cu",
+KERNEL_SOURCES = ["paper_2609_38795_gb300/csrc/loss_gemm_kernel.cuh",
                   "paper_2609_38795_gb300/csrc/row_kernels.cu",
                   "paper_2609_38795_gb300/csrc/tc_common.cuh",
                   "paper_2609_38795_gb300/csrc/kernels.h"]
