@@ -32,7 +32,7 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ f
   const int sq = seq[a], p0 = pos[a];
   int lim = L;
   if (valid_len != nullptr) lim = min(lim, valid_len[a]);
-  const bool ok = sq >= 0 && sq < S && p0 >= 0 && p0 + s < lim;
+  const bool ok = sq >= 0 && sq < S && p0 >= 0 && (long long)p0 + s < lim;   // no int overflow
   uint4* dst = out + r * vec_per_row;
   if (lane == 0 && row_valid != nullptr) row_valid[r] = ok ? 1.f : 0.f;
   if (!ok) {

@@ -40,9 +40,7 @@ def _operands(M, Nc, K, dtype, a_mn, b_mn, seed):
 def test_gemm_layouts(form, dtype, a_mn, b_mn, shape, monkeypatch):
     """Every form of the bf16 product (ALR_GEMM_FORM): single CTAs, clusters sharing B by
     multicast, CTA pairs with M = 256 products; fp32 (tf32) runs on single CTAs whatever the
-    setting."""
-    if dtype == torch.float32 and form != "single":
-        pytest.skip("tf32 products have one form")
+    setting, so its cases check that a cluster-form setting leaves the tf32 path intact."""
     monkeypatch.setenv("ALR_GEMM_FORM", form)
     assert alr.alr_kernel_forms()[0] == form, alr.alr_cluster_forms_error()
     M, Nc, K = shape

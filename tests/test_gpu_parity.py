@@ -46,6 +46,12 @@ def test_gather_matches_oracle_bit_for_bit(dtype):
     seq = torch.randint(-1, S + 1, (A,), generator=g, dtype=torch.int32)      # some invalid
     pos = torch.randint(-2, L - 4, (A,), generator=g, dtype=torch.int32)      # some past L-B
     vlen = torch.randint(0, L + 3, (A,), generator=g, dtype=torch.int32)
+    # extreme values: positions whose row index would overflow int32, the int32 ends as valid
+    # lengths and sequence ids; all give zero rows, as in the oracle's unbounded integers
+    i32 = torch.iinfo(torch.int32)
+    pos[0], pos[1], pos[2] = i32.max - 5, i32.max, i32.min
+    vlen[3], vlen[4] = i32.min, i32.max
+    seq[5], seq[6] = i32.max, i32.min
     for use_vlen in (False, True):
         out = torch.full((A * B, d), 7.0, dtype=dtype, device="cuda")
         valid = torch.full((A * B,), -1.0, device="cuda")
