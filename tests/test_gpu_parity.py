@@ -186,6 +186,35 @@ def test_large_ragged_step(keep):
     assert np.all(P.np64(dH)[7::B] == 0)
 
 
+@pytest.mark.parametrize("keep", [True, False])
+def test_paper_block_of_fifteen_predicted_slots(keep):
+    """The paper's own block (Sec. 3: K = 15 predicted slots after the anchor, App. A: blocks
+    of 16 with slot 0 the anchor) as B = 15 rows per anchor, so anchors straddle the 128-row
+    tiles (40 anchors, 600 rows, 4.7 row tiles), in the soft erase mode with gamma = 0.5 (the
+    alternative erase schedule) and lambda = 1.013441, through the whole step, logits kept and
+    recomputed: every row of the forward, the accepted lengths, dH and dW against the oracle."""
+    A, B, d, V, lam, gamma = 40, 15, 256, 3000, 1.013441, 0.5
+    mode = alr.ALR_MODE_ERASE_SOFT
+    Hd, Ht, W = _inputs(d, V, A, B, 0.5, torch.bfloat16, seed=15)
+    tok = _erase_tokens(Ht, W, 0.2, seed=15)
+    sl = alr.SlotLoss(A * B, d, V, B, lam=lam, gamma=gamma, mode=mode, keep_logits=keep)
+    sl.forward(Hd, Ht, W, corpus_tok=tok)
+    acc, hist = sl.accept()
+    dH = torch.empty(A * B, d, device="cuda")
+    dW = torch.zeros(d, V, device="cuda")
+    sl.backward(Hd, Ht, W, dH, dW)
+    torch.cuda.synchronize()
+    assert alr.alr_device_status() == alr.ALR_OK
+    r = _oracle_fwd(Hd, Ht, W, B, mode=mode, gamma=gamma, lam=lam, corpus_tok=P.npi(tok))
+    P.compare_forward(P.fwd_to_numpy(sl), r, mode=mode)
+    acc_r, _ = orc.accept_len(r["argmax_d"], r["argmax_t"], B)
+    P.compare_accept(P.npi(acc), P.npi(hist), acc_r, r["gap_d"], r["gap_t"], B)
+    G = orc.logit_grad(r["z_d"], r["z_t"], r["weight"], lam)
+    dH_r, dW_r = orc.slot_loss_backward(P.np64(Hd), P.np64(W), G)
+    assert P.max_norm_rel(P.np64(dH), dH_r) <= P.GRAD_RTOL
+    assert P.max_norm_rel(P.np64(dW), dW_r) <= P.GRAD_RTOL
+
+
 def test_small_bf16_forward_full_parity():
     """The small workload (d=2048, V=32000, B=16, 256 anchors): every row, forward only."""
     wl = synthetic.WORKLOADS["small"]
