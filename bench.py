@@ -84,10 +84,12 @@ def peaks():
 
 # ------------------------------------------------------------------ DRAM traffic ---
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "loss_gemm_traffic.json")
-KERNEL_SOURCES = ["paper_2609_38795_gb300/csrc/loss_gemm_kernel.cuh",
-                  "paper_2609_38795_gb300/csrc/row_kernels.cu",
-                  "paper_2609_38795_gb300/csrc/tc_common.cuh",
-                  "paper_2609_38795_gb300/csrc/kernels.h"]
+_CSRC = "paper_2609_38795_gb300/csrc/"
+_LOSS_KERNEL = [_CSRC + "loss_gemm_kernel.cuh", _CSRC + "tc_common.cuh", _CSRC + "kernels.h"]
+_ROW_KERNELS = [_CSRC + "row_kernels.cu", _CSRC + "tc_common.cuh", _CSRC + "kernels.h"]
+# the sources each recorded kernel is built from: its counters stay valid while their code does
+KERNEL_SOURCES = {"fwd": _LOSS_KERNEL, "fwd_recompute": _LOSS_KERNEL,
+                  "logit_grad_recompute": _LOSS_KERNEL, "logit_grad": _ROW_KERNELS}
 
 
 def _code_only(text):
@@ -99,33 +101,36 @@ def _code_only(text):
     return " ".join(text.split())
 
 
-def kernel_sources_sha256(read=None):
-    """Digest of the kernel sources' code.  `read(rel)` returns a file's text (default: the
-    working tree)."""
+def kernel_sources_sha256(files, read=None):
+    """Digest of the code of `files` (repository-relative).  `read(rel)` returns a file's text
+    (default: the working tree)."""
     import hashlib
     if read is None:
         def read(rel):
             with open(os.path.join(ROOT, rel), encoding="utf-8") as f:
                 return f.read()
     h = hashlib.sha256()
-    for rel in KERNEL_SOURCES:
+    for rel in files:
         h.update(_code_only(read(rel)).encode())
     return h.hexdigest()
 
 
 def kernel_traffic(phase):
     """DRAM bytes per full-size launch of the kernel of a step phase ("fwd": the fused forward
-    keeping the logits; "logit_grad": G from the kept logits), from the committed ncu summary,
-    or None when that summary is missing or was taken from other kernel sources."""
+    keeping the logits; "logit_grad": G from the kept logits; "*_recompute": the step that keeps
+    nothing), from the committed ncu summary, or None when that summary is missing or the
+    kernel's sources changed since its capture."""
     try:
         with open(TRAFFIC_FILE) as f:
             j = json.load(f)
     except (OSError, ValueError):
         return None
-    if j.get("sources_sha256") != kernel_sources_sha256():
-        return None
     k = j.get("kernels", {}).get(phase)
-    return None if k is None else k["bytes_per_full_launch"]
+    if k is None or phase not in KERNEL_SOURCES:
+        return None
+    if k.get("sources_sha256") != kernel_sources_sha256(KERNEL_SOURCES[phase]):
+        return None
+    return k["bytes_per_full_launch"]
 
 
 # ------------------------------------------------------------------ rank reductions ---

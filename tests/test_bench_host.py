@@ -1,3 +1,4 @@
+import os
 """Host-side helpers of bench.py (no GPU): the mean accepted tokens reported from an
 acceptance histogram, the clock-sample summary that decides whether a run is kept, and the
 digest that ties the committed DRAM-traffic record to the kernel code."""
@@ -42,18 +43,19 @@ def test_clock_samples_summary_and_throttle_reasons():
 
 
 def test_traffic_record_follows_kernel_code_not_comments():
-    """The DRAM-traffic record is tied to a digest of the kernel sources' code: a comment or
-    a blank line leaves it valid, a changed token invalidates it."""
+    """The DRAM-traffic record of a kernel is tied to a digest of its sources' code: a comment
+    or a blank line leaves it valid, a changed token invalidates it."""
     src = {"a.cu": "int f(int x) {\n  return x + 1;  // add one\n}\n", "b.h": "/* doc */ int g;"}
     names = list(src)
-    saved = bench.KERNEL_SOURCES
-    try:
-        bench.KERNEL_SOURCES = names
-        h0 = bench.kernel_sources_sha256(read=lambda rel: src[rel])
-        commented = dict(src, **{"a.cu": "// header\nint f(int x) {\n\n"
-                                          "  return x + 1; /* one */\n}\n"})
-        assert bench.kernel_sources_sha256(read=lambda rel: commented[rel]) == h0
-        changed = dict(src, **{"a.cu": "int f(int x) {\n  return x + 2;\n}\n"})
-        assert bench.kernel_sources_sha256(read=lambda rel: changed[rel]) != h0
-    finally:
-        bench.KERNEL_SOURCES = saved
+    h0 = bench.kernel_sources_sha256(names, read=lambda rel: src[rel])
+    commented = dict(src, **{"a.cu": "// header\nint f(int x) {\n\n"
+                                      "  return x + 1; /* one */\n}\n"})
+    assert bench.kernel_sources_sha256(names, read=lambda rel: commented[rel]) == h0
+    changed = dict(src, **{"a.cu": "int f(int x) {\n  return x + 2;\n}\n"})
+    assert bench.kernel_sources_sha256(names, read=lambda rel: changed[rel]) != h0
+
+
+def test_every_recorded_kernel_names_existing_sources():
+    for phase, files in bench.KERNEL_SOURCES.items():
+        for rel in files:
+            assert os.path.exists(os.path.join(bench.ROOT, rel)), (phase, rel)
