@@ -86,10 +86,10 @@ def peaks():
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "loss_gemm_traffic.json")
 _CSRC = "paper_2609_38795_gb300/csrc/"
 _LOSS_KERNEL = [_CSRC + "loss_gemm_kernel.cuh", _CSRC + "tc_common.cuh", _CSRC + "kernels.h"]
-_ROW_KERNELS = [_CSRC + "row_kernels.cu", _CSRC + "tc_common.cuh", _CSRC + "kernels.h"]
+_GRAD_KERNELS = [_CSRC + "grad_kernels.cu", _CSRC + "tc_common.cuh", _CSRC + "kernels.h"]
 # the sources each recorded kernel is built from: its counters stay valid while their code does
 KERNEL_SOURCES = {"fwd": _LOSS_KERNEL, "fwd_recompute": _LOSS_KERNEL,
-                  "logit_grad_recompute": _LOSS_KERNEL, "logit_grad": _ROW_KERNELS}
+                  "logit_grad_recompute": _LOSS_KERNEL, "logit_grad": _GRAD_KERNELS}
 
 
 def _code_only(text):
