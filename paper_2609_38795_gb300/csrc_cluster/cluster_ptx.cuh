@@ -125,6 +125,24 @@ ALR_DEV void mma_commit_pair(uint64_t* bar, uint16_t cta_mask) {
       : "memory");
 }
 
+// Host side: the launch configuration of a kernel on clusters of `ctas` CTAs along x (attr
+// must outlive the launch).
+inline cudaLaunchConfig_t cluster_config(cudaLaunchAttribute* attr, unsigned ctas, unsigned grid,
+                                         unsigned threads, size_t smem, cudaStream_t s) {
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = ctas;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
 // Cluster policies of the fused loss and plain GEMM kernels: clusters of kCtas CTAs in which
 // each CTA loads a 1 / kCtas share of every head (B) tile, multicast into all of them, and each
 // MMA issuer's commit releases the stage in all of them.

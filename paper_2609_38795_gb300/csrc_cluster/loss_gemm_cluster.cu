@@ -9,22 +9,6 @@
 namespace alr {
 namespace {
 
-cudaLaunchConfig_t cluster2_config(cudaLaunchAttribute* attr, unsigned grid, unsigned threads,
-                                   size_t smem, cudaStream_t s) {
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(threads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cfg;
-}
-
 template <int kMode>
 cudaError_t launch_cluster(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& w,
                            const CUtensorMap& g, const CUtensorMap& g2, const LossArgs& args,
@@ -44,7 +28,7 @@ cudaError_t launch_cluster(const CUtensorMap& a0, const CUtensorMap& a1, const C
   cudaLaunchAttribute attr[1];
   int known = max_clusters[dev].load(std::memory_order_relaxed);
   if (known == 0) {
-    cudaLaunchConfig_t q = cluster2_config(attr, 2, S::kThreads, S::kSmem, s);
+    cudaLaunchConfig_t q = cluster_config(attr, 2, 2, S::kThreads, S::kSmem, s);
     int n = 0;
     if ((e = cudaOccupancyMaxActiveClusters(&n, kern, &q)) != cudaSuccess) return e;
     if (n < 1) return cudaErrorInvalidConfiguration;
@@ -52,7 +36,7 @@ cudaError_t launch_cluster(const CUtensorMap& a0, const CUtensorMap& a1, const C
     known = n;
   }
   const int clusters = known < args.plan.n_units ? known : args.plan.n_units;
-  cudaLaunchConfig_t cfg = cluster2_config(attr, unsigned(2 * clusters), S::kThreads, S::kSmem, s);
+  cudaLaunchConfig_t cfg = cluster_config(attr, 2, unsigned(2 * clusters), S::kThreads, S::kSmem, s);
   return cudaLaunchKernelEx(&cfg, kern, a0, a1, w, g, g2, args);
 }
 

@@ -9,22 +9,6 @@
 namespace alr {
 namespace {
 
-template <int kMc>
-cudaLaunchConfig_t cluster_config(cudaLaunchAttribute* attr, unsigned grid, cudaStream_t s) {
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kMc;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
-  cfg.stream = s;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cfg;
-}
-
 template <bool kAMN, bool kBMN, bool kAcc, int kMc>
 cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs& args,
                      cudaStream_t s) {
@@ -33,7 +17,7 @@ cudaError_t launch_t(const CUtensorMap& a, const CUtensorMap& b, const GemmArgs&
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes));
   if (e != cudaSuccess) return e;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = cluster_config<kMc>(attr, unsigned(args.grid), s);
+  cudaLaunchConfig_t cfg = cluster_config(attr, kMc, unsigned(args.grid), kThreads, kSmemBytes, s);
   return cudaLaunchKernelEx(&cfg, kern, a, b, args);
 }
 
@@ -50,7 +34,7 @@ int max_clusters() {
                            int(kSmemBytes)) != cudaSuccess)
     return 0;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = cluster_config<kMc>(attr, unsigned(kMc), nullptr);
+  cudaLaunchConfig_t cfg = cluster_config(attr, kMc, unsigned(kMc), kThreads, kSmemBytes, nullptr);
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) return 0;
   cached[dev].store(n, std::memory_order_relaxed);
