@@ -63,6 +63,38 @@ def test_gather_matches_oracle_bit_for_bit(dtype):
         assert np.array_equal(valid.cpu().numpy(), rv)
 
 
+def test_chained_gathers_see_each_others_writes():
+    """The gathers are launched with programmatic dependent launch: a gather may be scheduled
+    while the one before it still runs, and must wait for it before any access.  Each gather
+    here reads the previous one's output as its feature buffer (read after write), and the last
+    one also overwrites the buffer its predecessor read (write after read); every buffer
+    matches the oracle applied in the same order."""
+    g = torch.Generator().manual_seed(8)
+    S, L, d, A, B = 3, 256, 512, 48, 16                   # A * B = S * L: outputs are buffers
+    draws = [(torch.randint(0, S, (A,), generator=g, dtype=torch.int32),
+              torch.randint(0, L - B + 1, (A,), generator=g, dtype=torch.int32)) for _ in range(4)]
+    F0 = torch.randn(S, L, d, generator=g).to(torch.bfloat16)
+    bufs = [F0.cuda()] + [torch.empty(S, L, d, dtype=torch.bfloat16, device="cuda")
+                          for _ in range(3)]
+    for i in range(3):                                    # bufs[i + 1] = gather(bufs[i])
+        seq, pos = draws[i]
+        alr.alr_gather_ira_blocks(bufs[i], seq.cuda(), pos.cuda(), B, bufs[i + 1].view(A * B, d))
+    seq, pos = draws[3]                                   # reads bufs[3], overwrites bufs[2]
+    alr.alr_gather_ira_blocks(bufs[3], seq.cuda(), pos.cuda(), B, bufs[2].view(A * B, d))
+    torch.cuda.synchronize()
+    ref = [F0.float().numpy()]
+    for i in range(3):
+        r, v = orc.gather_ira_blocks(ref[i], draws[i][0].numpy(), draws[i][1].numpy(), B)
+        assert v.all()
+        ref.append(r.reshape(S, L, d))
+    last, _ = orc.gather_ira_blocks(ref[3], draws[3][0].numpy(), draws[3][1].numpy(), B)
+    assert np.array_equal(bufs[1].float().cpu().numpy(), ref[1])
+    assert np.array_equal(bufs[3].float().cpu().numpy(), ref[3])
+    assert np.array_equal(bufs[2].float().cpu().numpy(), last.reshape(S, L, d))
+    assert not np.array_equal(ref[2], last.reshape(S, L, d))
+    assert alr.alr_device_status() == alr.ALR_OK
+
+
 def test_gather_ira_secondary_blocks_mask():
     """Secondary blocks at offsets j in 2..14 of 15 stored rows: valid rows are 1[j+k <= K]."""
     K, d, A = 15, 64, 13
