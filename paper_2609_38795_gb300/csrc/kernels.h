@@ -107,7 +107,8 @@ struct LossArgs {
 // R[v / 16, r] at (v / 16) * N + r, so that one warp's 32 rows of a group are contiguous.
 constexpr int kKeepGroup = 16;
 
-// Fused loss kernels (loss_gemm.cu).  dtype: 0 bf16, 1 fp32 (tf32 products).
+// Fused loss kernels (loss_gemm_kernel.cuh, launched from loss_gemm.cu).  dtype: 0 bf16, 1 fp32
+// (tf32 products).
 //   a0: the first hidden-state operand (H_d; H_t for the readout), a1: H_t (dual modes).
 //   g_store: bf16 G [N, V] as 16-column x 32-row boxes without swizzle (gradient modes, bf16),
 //            or fp16 z_d [N, V] in the same boxes (kModeFwdKeep, bf16);
@@ -116,7 +117,8 @@ cudaError_t launch_loss_kernel(int mode, int dtype, const CUtensorMap& a0, const
                                const CUtensorMap& w, const CUtensorMap& g_store,
                                const CUtensorMap& g_store2, const LossArgs& args, cudaStream_t s);
 
-// Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm.cu).
+// Plain GEMM C[M, Nc] (+)= A[M, K] B[K, Nc] with fp32 output (plain_gemm_kernel.cuh, single-CTA
+// form launched from plain_gemm.cu).
 struct GemmArgs {
   int M, Nc, K;
   float* C;

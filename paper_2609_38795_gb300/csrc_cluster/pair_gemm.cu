@@ -6,7 +6,7 @@
 // N = 256): CTA r of the pair loads rows [128 r, 128 r + 128) of the A tile and columns
 // [128 r, 128 r + 128) of the B tile into its own shared memory, the even CTA issues the
 // products for both, and each CTA finds its 128 rows of the tile in its own tensor memory
-// (two 256-column buffers).  Against the one-CTA kernel (plain_gemm.cu) every CTA reads half
+// (two 256-column buffers).  Against the one-CTA kernel (plain_gemm_kernel.cuh) every CTA reads half
 // the B bytes per product from shared memory and from L2.
 //
 // Pipeline: 6 stages of (A 16 KB + B half 16 KB) per CTA.  The even CTA's full barrier of a
